@@ -1,0 +1,238 @@
+"""Seeded synthetic inputs for the verifier: logit rows, emitted-token ids,
+ragged request layouts (CSR offsets), decode traces and scorer weights.
+
+This module is shared by the GPU tests, the benchmark and the oracle tests.  It
+holds none of the verifier's arithmetic: it only draws random numbers.  The
+paper evaluates on 15 benchmark suites whose model outputs are not available
+here; these generators stand in for the small model's per-token distributions
+with the shapes and value mixes listed below.
+
+Workloads (vocabulary widths are the small model's output widths):
+
+  tiny    8 requests, T ~ U{16..64}, V = 32,000 float32, x = 2 N(0,1) plus one
+          spike +U(0,8) per row at a random index.
+  full    64 requests, T ~ U{32..256}, V = 151,936 bfloat16, x = s N(0,1) with a
+          per-row scale s ~ U(1,4); 70% of rows get a spike +U(0,12).
+  decode  256 live slots for 1,000 steps, request lengths ~ U{64..1000}, a slot is
+          refilled by a new request when its request ends; rows as in ``full``.
+  ragged  1,024 requests, T = clip(round(lognormal(ln 128, 0.8)), 8, 1024),
+          rows as in ``full``, processed in 8,192-row chunks.
+  wide    512 requests, T ~ U{64..512}, V = 262,144 float32, x = 2 t_3 (Student-t,
+          3 degrees of freedom); on 10% of rows the maximum is copied to a second
+          random index (an exact tie for the top token).
+
+Every row is a pure function of (workload seed, global row index): rows are
+drawn in blocks of ``BLOCK`` rows from a generator seeded by the block index,
+so any chunking of the batch sees identical values.  The emitted token is
+sampled from the softmax of the *stored* (rounded) row at temperature 1 with
+the Gumbel-max construction, which needs no normalisation.
+
+Scorer: w (11 weights) then b are 12 draws of N(0, 0.1^2) from PCG64(seed+100),
+rounded to float32; tau = 0.5.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass, field
+
+import numpy as np
+import torch
+
+BLOCK = 256  # rows per seeded generation block
+
+
+@dataclass
+class Workload:
+    name: str
+    dtype: str  # "bf16" | "f32"
+    vocab: int
+    lengths: np.ndarray  # int64 [n_req]
+    seed_host: int
+    seed_dev: int
+    dist: str  # "tiny" | "full" | "wide"
+    chunk_rows: int = 0  # 0: whole batch in one call
+    w: np.ndarray = field(default=None)  # float32 [11]
+    b: float = 0.0
+    tau: float = 0.5
+
+    @property
+    def n_req(self) -> int:
+        return int(self.lengths.size)
+
+    @property
+    def offsets(self) -> np.ndarray:
+        return np.concatenate([[0], np.cumsum(self.lengths)]).astype(np.int64)
+
+    @property
+    def n_rows(self) -> int:
+        return int(self.lengths.sum())
+
+    @property
+    def elem_bytes(self) -> int:
+        return 2 if self.dtype == "bf16" else 4
+
+    @property
+    def torch_dtype(self):
+        return torch.bfloat16 if self.dtype == "bf16" else torch.float32
+
+
+def scorer(seed_host: int):
+    g = np.random.Generator(np.random.PCG64(seed_host + 100))
+    d = g.normal(0.0, 0.1, size=12).astype(np.float32)
+    return d[:11].copy(), float(d[11])
+
+
+def _finish(wl: Workload) -> Workload:
+    wl.w, wl.b = scorer(wl.seed_host)
+    return wl
+
+
+def make(name: str, n_req: int | None = None, vocab: int | None = None,
+         max_len: int | None = None) -> Workload:
+    """One of the five named workloads; ``n_req``/``vocab``/``max_len`` shrink it
+    (same distributions) for tests that must finish quickly on the oracle."""
+    if name == "tiny":
+        g = np.random.Generator(np.random.PCG64(1001))
+        n = n_req or 8
+        lengths = g.integers(16, 64, size=n, endpoint=True)
+        wl = Workload(name, "f32", vocab or 32000, lengths, 1001, 2001, "tiny")
+    elif name == "full":
+        g = np.random.Generator(np.random.PCG64(1002))
+        n = n_req or 64
+        lengths = g.integers(32, 256, size=n, endpoint=True)
+        wl = Workload(name, "bf16", vocab or 151936, lengths, 1002, 2002, "full")
+    elif name == "ragged":
+        g = np.random.Generator(np.random.PCG64(1004))
+        n = n_req or 1024
+        raw = np.exp(g.normal(np.log(128.0), 0.8, size=n))
+        lengths = np.clip(np.round(raw), 8, 1024).astype(np.int64)
+        wl = Workload(name, "bf16", vocab or 151936, lengths, 1004, 2004, "full",
+                      chunk_rows=8192)
+    elif name == "wide":
+        g = np.random.Generator(np.random.PCG64(1005))
+        n = n_req or 512
+        lengths = g.integers(64, 512, size=n, endpoint=True)
+        wl = Workload(name, "f32", vocab or 262144, lengths, 1005, 2005, "wide")
+    else:
+        raise KeyError(name)
+    wl.lengths = np.asarray(wl.lengths, np.int64)
+    if max_len is not None:
+        wl.lengths = np.minimum(wl.lengths, max_len)
+    return _finish(wl)
+
+
+# ---- rows ------------------------------------------------------------------
+
+def _block(wl: Workload, blk: int, device) -> tuple[torch.Tensor, torch.Tensor]:
+    """Rows [blk*BLOCK, (blk+1)*BLOCK) in storage dtype, and their emitted ids."""
+    dev = torch.device(device)
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(wl.seed_dev * 1_000_003 + blk)
+    n, V = BLOCK, wl.vocab
+    rows = torch.arange(n, device=dev)
+    if wl.dist == "tiny":
+        x = torch.randn(n, V, generator=gen, device=dev) * 2.0
+        pos = torch.randint(0, V, (n,), generator=gen, device=dev)
+        amp = torch.rand(n, generator=gen, device=dev) * 8.0
+        x[rows, pos] += amp
+    elif wl.dist == "full":
+        s = 1.0 + 3.0 * torch.rand(n, 1, generator=gen, device=dev)
+        x = torch.randn(n, V, generator=gen, device=dev) * s
+        pos = torch.randint(0, V, (n,), generator=gen, device=dev)
+        amp = torch.rand(n, generator=gen, device=dev) * 12.0
+        has = torch.rand(n, generator=gen, device=dev) < 0.7
+        x[rows, pos] += torch.where(has, amp, torch.zeros_like(amp))
+    elif wl.dist == "wide":
+        z = torch.randn(n, V, generator=gen, device=dev)
+        c = torch.zeros(n, V, device=dev)
+        for _ in range(3):
+            c += torch.randn(n, V, generator=gen, device=dev).square_()
+        x = 2.0 * z / torch.sqrt(c / 3.0)
+        del z, c
+        tie = torch.rand(n, generator=gen, device=dev) < 0.10
+        other = torch.randint(0, V - 1, (n,), generator=gen, device=dev)
+        top = torch.argmax(x, dim=1)
+        other = other + (other >= top).long()  # a second index, never the top one
+        r = rows[tie]
+        x[r, other[tie]] = x[r, top[tie]]
+    else:
+        raise KeyError(wl.dist)
+    xs = x.to(wl.torch_dtype)
+    del x
+    # emitted token ~ softmax(stored row) at T = 1, via Gumbel-max
+    u = torch.rand(n, V, generator=gen, device=dev).clamp_(min=1e-30)
+    g = -torch.log(-torch.log(u))
+    chosen = torch.argmax(xs.float() + g, dim=1).to(torch.int32)
+    return xs, chosen
+
+
+def rows(wl: Workload, lo: int, hi: int, device="cuda", out: torch.Tensor | None = None,
+         chosen_out: torch.Tensor | None = None):
+    """Global rows [lo, hi) of the workload: (logits [hi-lo, V], chosen [hi-lo])."""
+    n = hi - lo
+    if out is None:
+        out = torch.empty(n, wl.vocab, dtype=wl.torch_dtype, device=device)
+    if chosen_out is None:
+        chosen_out = torch.empty(n, dtype=torch.int32, device=device)
+    b0, b1 = lo // BLOCK, (hi - 1) // BLOCK if n > 0 else -1
+    for blk in range(b0, b1 + 1):
+        x, c = _block(wl, blk, device)
+        s = max(lo, blk * BLOCK)
+        e = min(hi, (blk + 1) * BLOCK)
+        out[s - lo:e - lo].copy_(x[s - blk * BLOCK:e - blk * BLOCK])
+        chosen_out[s - lo:e - lo].copy_(c[s - blk * BLOCK:e - blk * BLOCK])
+        del x, c
+    return out, chosen_out
+
+
+def to_oracle_array(t: torch.Tensor) -> np.ndarray:
+    """Host copy in the oracle's input format: float32, or uint16 bit patterns for bf16."""
+    t = t.detach().cpu().contiguous()
+    if t.dtype == torch.bfloat16:
+        return t.view(torch.int16).numpy().view(np.uint16)
+    return t.numpy()
+
+
+# ---- decode traces -----------------------------------------------------------
+
+@dataclass
+class DecodeTrace:
+    n_slots: int
+    n_steps: int
+    vocab: int
+    dtype: str
+    seed_dev: int
+    dist: str
+    requests: list  # (slot, start_step, length) for every request that started
+    eos: np.ndarray  # uint8 [n_steps, n_slots]
+    w: np.ndarray
+    b: float
+    tau: float = 0.5
+
+    @property
+    def torch_dtype(self):
+        return torch.bfloat16 if self.dtype == "bf16" else torch.float32
+
+    def as_workload(self) -> Workload:
+        """Row generator view: global row id = step * n_slots + slot."""
+        wl = Workload("decode", self.dtype, self.vocab, np.zeros(0, np.int64), 1003,
+                      self.seed_dev, self.dist)
+        wl.w, wl.b, wl.tau = self.w, self.b, self.tau
+        return wl
+
+
+def decode_trace(n_slots: int = 256, n_steps: int = 1000, lo: int = 64, hi: int = 1000,
+                 vocab: int = 151936, seed_host: int = 1003, seed_dev: int = 2003) -> DecodeTrace:
+    """Every slot is always live: when a request ends the slot takes a new one."""
+    g = np.random.Generator(np.random.PCG64(seed_host))
+    eos = np.zeros((n_steps, n_slots), np.uint8)
+    reqs = []
+    for s in range(n_slots):
+        t = 0
+        while t < n_steps:
+            L = int(g.integers(lo, hi, endpoint=True))
+            reqs.append((s, t, L))
+            if t + L - 1 < n_steps:
+                eos[t + L - 1, s] = 1
+            t += L
+    w, b = scorer(seed_host)
+    return DecodeTrace(n_slots, n_steps, vocab, "bf16", seed_dev, "full", reqs, eos, w, b)
