@@ -1,0 +1,370 @@
+"""Benchmark of the verifier data path: verified tokens/s on the full-response
+workload (64 requests, response lengths U{32..256}, 8,847 logit rows of
+V = 151,936 bf16, 2.69 GB) and achieved HBM bandwidth of the fused kernel.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl gb300|reference]
+
+A step is one fused verification of the whole batch (pr_route: row features,
+pooling, score, ship rule; one kernel launch) with the logits resident in HBM.
+The batch is larger than L2, so no flush is needed between steps.  Under
+torchrun every rank verifies its own batch (weak scaling, no collective on
+the data path); rank 0 prints one JSON line.  ``--impl reference`` times the
+float64 CPU oracle on the host cores instead (a bounded sample per step).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2608_28726_gb300 import workloads as W  # noqa: E402
+
+WORKLOAD = "full"
+METRIC = "verified tokens/sec at V=151,936 bf16 and achieved HBM GB/s vs peak (1xGB300)"
+UNIT = "tokens/s"
+KERNEL_FILES = ("pr_device.cuh", "pr_kernels.cuh", "pro_router.cu")
+PROFILE = os.path.join(ROOT, "profiles", "verify_rows_bf16_full_response.md")
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def reduce_max(value: float, world: int, device) -> float:
+    """Max over ranks (the slowest rank sets the job time)."""
+    if world == 1:
+        return value
+    import torch.distributed as dist
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world: int):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def workload_desc(wl) -> str:
+    return ("full-response verify: %d requests, T~U{32..256} (%d rows), V=%d %s, "
+            "N(0,1)*s, s~U(1,4), spike +U(0,12) on 70%% of rows" % (
+                wl.n_req, wl.n_rows, wl.vocab, wl.dtype))
+
+
+def algorithmic_bytes(wl) -> int:
+    """Bytes one fused launch must move: each row's logits, its token id and
+    its 36-byte record (8 floats + flags) written and read back once by the
+    pooling epilogue; per request two offsets, 11 aggregates, score, ship and
+    flags."""
+    per_row = wl.vocab * wl.elem_bytes + 4 + 36 + 36
+    per_req = 16 + 44 + 4 + 1 + 4
+    return wl.n_rows * per_row + wl.n_req * per_req
+
+
+def kernel_sha() -> str:
+    h = hashlib.sha256()
+    for f in KERNEL_FILES:
+        with open(os.path.join(ROOT, "paper_2608_28726_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic():
+    """DRAM bytes per launch from the committed ncu summary, if it was taken on
+    the current kernel source (else None)."""
+    try:
+        text = open(PROFILE).read()
+    except OSError:
+        return None
+    vals = {}
+    for line in text.splitlines():
+        if ":" in line and line.strip().startswith("- "):
+            k, v = line.strip()[2:].split(":", 1)
+            vals[k.strip()] = v.strip().strip("`")
+    if vals.get("kernel_source_sha") != kernel_sha():
+        return None
+    try:
+        return int(vals["dram_bytes_per_full_launch"])
+    except (KeyError, ValueError):
+        return None
+
+
+class ClockSampler:
+    """nvidia-smi clocks / throttle reasons every 100 ms while the bench runs."""
+
+    FIELDS = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.samples = []
+        self.proc = None
+        self.index = index
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.samples.append((time.time(), [p.strip() for p in line.split(",")]))
+
+    def stop(self):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+        if self.thread:
+            self.thread.join(timeout=2)
+
+    def summary(self, t0: float, t1: float):
+        inside = [s for (t, s) in self.samples if t0 <= t <= t1]
+        window = "timed"
+        if len(inside) < 3:
+            inside = [s for (_, s) in self.samples]
+            window = "whole run (timed region shorter than 3 samples)"
+        if not inside:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        sm = [float(s[1]) for s in inside if s[1].replace(".", "").isdigit()]
+        mx = [float(s[2]) for s in inside if s[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for s in inside for i in range(4)
+                          if len(s) > 5 + i and s[5 + i].lower().startswith("active")})
+        pw = [float(s[3]) for s in inside if s[3].replace(".", "").isdigit()]
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None,
+                "power_w_max": max(pw) if pw else None,
+                "reasons": reasons, "samples": len(inside), "window": window}
+
+
+def oracle_sample(wl, x_host_rows, chosen_host, req_lo: int, req_hi: int, n_threads: int):
+    """Oracle on whole requests [req_lo, req_hi) of the workload."""
+    import oracle
+    off = wl.offsets
+    lo, hi = int(off[req_lo]), int(off[req_hi])
+    sub_off = off[req_lo:req_hi + 1] - lo
+    t0 = time.perf_counter()
+    o = oracle.route(x_host_rows, chosen_host, sub_off, wl.w.astype(np.float64), wl.b, wl.tau,
+                     n_threads=n_threads)
+    dt = time.perf_counter() - t0
+    return o, dt, hi - lo
+
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    import oracle
+    oracle.build()
+    wl = W.make(WORKLOAD)
+    cores = os.cpu_count() or 1
+    # one step = the oracle on one bounded sample of whole requests
+    req_hi = 2
+    lo, hi = 0, int(wl.offsets[req_hi])
+    x, ch = W.rows(wl, lo, hi, device="cpu")
+    xs, cs = W.to_oracle_array(x), ch.numpy()
+    for _ in range(args.warmup):
+        oracle_sample(wl, xs, cs, 0, req_hi, cores)
+    times = []
+    for _ in range(args.steps):
+        _, dt, rows = oracle_sample(wl, xs, cs, 0, req_hi, cores)
+        times.append(dt)
+    total = sum(times)
+    value = (hi - lo) * args.steps / total
+    sample = "requests 0..%d of the workload (%d rows of V=%d bf16) per step" % (
+        req_hi - 1, hi - lo, wl.vocab)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic",
+        "config": {"workload": workload_desc(wl), "sample_rows_per_step": hi - lo},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+    return 0
+
+
+def run_gb300(args):
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", init_method="env://")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    from paper_2608_28726_gb300 import build as prbuild
+    prbuild.build()
+    from paper_2608_28726_gb300 import binding as B
+
+    wl = W.make(WORKLOAD)
+    x, ch = W.rows(wl, 0, wl.n_rows, device=dev)
+    off = torch.from_numpy(wl.offsets).to(dev)
+    w = torch.from_numpy(wl.w).to(dev)
+    ctx = B.pr_ctx_create(local, max_rows=wl.n_rows, max_requests=wl.n_req)
+    stream = torch.cuda.current_stream(dev)
+    score = torch.empty(wl.n_req, device=dev)
+    ship = torch.empty(wl.n_req, dtype=torch.uint8, device=dev)
+    rflags = torch.empty(wl.n_req, dtype=torch.int32, device=dev)
+    agg = torch.empty(wl.n_req, 11, device=dev)
+
+    def step():
+        B.pr_route(ctx, x, ch, off, w, wl.b, wl.tau, score=score, ship=ship, req_flags=rflags,
+                   agg=agg, stream=stream)
+
+    sampler = ClockSampler(local)
+    sampler.start()
+    for _ in range(max(3, args.warmup)):
+        step()
+    torch.cuda.synchronize(dev)
+
+    K = args.steps
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(K + 1)]
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    n_launch0 = B.launch_count()
+    t_wall0 = time.time()
+    ev[0].record(stream)
+    for i in range(K):
+        step()
+        ev[i + 1].record(stream)
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    t_wall1 = time.time()
+    launches = B.launch_count() - n_launch0
+    per_launch = [ev[i].elapsed_time(ev[i + 1]) for i in range(K)]
+    total_ms = ev[0].elapsed_time(ev[K])
+    total_ms = reduce_max(total_ms, world, dev)
+    clocks = sampler.summary(t_wall0, t_wall1)
+
+    # end to end from pinned host memory through the public C ABI
+    hx = x.cpu().pin_memory()
+    hc = ch.cpu().pin_memory()
+    hoff = torch.from_numpy(wl.offsets)
+    hw = torch.from_numpy(wl.w)
+    hs = torch.empty(wl.n_req).pin_memory()
+    hsh = torch.empty(wl.n_req, dtype=torch.uint8).pin_memory()
+    hf = torch.empty(wl.n_req, dtype=torch.int32).pin_memory()
+    ctx_h = B.pr_ctx_create(local, max_rows=wl.n_rows, max_requests=wl.n_req)
+    e2e_steps = max(3, min(K, 10))
+
+    def e2e_step():
+        B.pr_route_host(ctx_h, hx, hc, hoff, hw, wl.b, wl.tau, chunk_rows=512, score=hs, ship=hsh,
+                        req_flags=hf, stream=stream)
+
+    e2e_step()
+    barrier(world)
+    t0 = time.perf_counter()
+    for _ in range(e2e_steps):
+        e2e_step()
+    barrier(world)
+    e2e_s = reduce_max(time.perf_counter() - t0, world, dev)
+    sampler.stop()
+
+    h2d = hx.numel() * hx.element_size() + hc.numel() * 4 + hoff.numel() * 8 + hw.numel() * 4
+    d2h = hs.numel() * 4 + hsh.numel() + hf.numel() * 4
+    rows_all = wl.n_rows * world
+    value = rows_all * K / (total_ms / 1e3)
+    e2e_value = rows_all * e2e_steps / e2e_s
+
+    avg_launch_ms = sum(per_launch) / len(per_launch)
+    abytes = algorithmic_bytes(wl)
+    achieved = abytes / (avg_launch_ms / 1e3) / 1e9
+    peaks_file = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    peak, peak_src = 6800.0, "fallback"
+    if os.path.exists(peaks_file):
+        peak = float(json.load(open(peaks_file))["hbm_gbs"])
+        peak_src = "measured"
+
+    line = None
+    if rank == 0:
+        # parity of the timed run's outputs on a sample of whole requests, and
+        # the oracle's own speed on that sample (the CPU baseline)
+        import oracle
+        oracle.build()
+        cores = os.cpu_count() or 1
+        req_hi = 8
+        lo, hi = 0, int(wl.offsets[req_hi])
+        xs = W.to_oracle_array(x[lo:hi])
+        cs = ch[lo:hi].cpu().numpy()
+        o, dt, rows = oracle_sample(wl, xs, cs, 0, req_hi, cores)
+        g_agg = agg[:req_hi].cpu().numpy().astype(np.float64)
+        g_score = score[:req_hi].cpu().numpy().astype(np.float64)
+        ok = bool(np.all(np.abs(g_agg - o["agg"]) <= 1e-5 + 1e-4 * np.abs(o["agg"])) and
+                  np.all(np.abs(g_score - o["score"]) <= 1e-5 + 1e-4 * np.abs(o["score"])) and
+                  np.all((ship[:req_hi].cpu().numpy() == o["ship"]) |
+                         (np.abs(o["score"] - wl.tau) < 1e-6)) and
+                  np.all(hsh[:req_hi].numpy() == ship[:req_hi].cpu().numpy()))
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
+            "warmup": max(3, args.warmup), "ms_per_step": total_ms / K, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": workload_desc(wl), "rows_per_step_per_gpu": wl.n_rows,
+                       "logit_bytes_per_step_per_gpu": wl.n_rows * wl.vocab * 2,
+                       "l2": "inputs (2.69 GB) larger than L2 (129 MB), no flush",
+                       "parallelism": "dp%d (independent batches)" % world},
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                         "frac": achieved / peak, "traffic": profiled_traffic(),
+                         "kernel": "verify_rows<bf16, route>", "peak_source": peak_src,
+                         "algorithmic_bytes_per_launch": abytes,
+                         "avg_launch_ms": avg_launch_ms},
+            "cpu_baseline": {"value": rows / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": "requests 0..%d (%d rows), float64 C oracle, %d threads" % (
+                                 req_hi - 1, rows, cores)},
+            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d // world * world,
+                    "d2h_bytes_per_step": d2h, "api": "pr_route_host (pinned host buffers)"},
+            "gpu_launches": launches,
+            "clocks": clocks,
+            "parity": {"requests_checked": req_hi, "rows_checked": rows, "ok": ok},
+        }
+        print(json.dumps(line))
+    B.pr_ctx_destroy(ctx_h)
+    B.pr_ctx_destroy(ctx)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    args = ap.parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_gb300(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

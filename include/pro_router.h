@@ -1,0 +1,256 @@
+/*
+ * pro_router.h — C ABI of the GB300 data path of Pro-Router's token-aware
+ * verifier (arXiv 2608.28726, Section 3.1).
+ *
+ * The verifier reads, for every generated token t, the small model's logit row
+ * x_t over the vocabulary (V entries) and reduces it to the per-token features
+ * of Eq. 3:
+ *     l_t   = log p_t(y_t)            log-probability of the emitted token y_t
+ *     m_t   = max_v p_t(v)            maximum probability
+ *     h_t   = -H_t^K,  H_t^K = -sum_{v in top-K} p_t(v) log p_t(v),  K = 20
+ *     rho_t = t / T                   position fraction (t is 1-based)
+ * with p_t = softmax(x_t).  The data path also reports the probability margin
+ * p(i1) - p(i2) between the first two tokens, the full-vocabulary entropy H,
+ * log-sum-exp and the two top indices.  Per request (a ragged run of T rows)
+ * the features are pooled, scored by a linear scorer and thresholded: a
+ * request ships when its confidence is >= tau (Section 3.1, the ship rule
+ * "p >= tau"); otherwise it escalates to the large model.
+ *
+ * Conventions shared by every call
+ *   - Pointers named as device buffers are caller-owned CUDA device memory on
+ *     the context's device; the library never frees them.  The library
+ *     allocates only inside a context (pr_ctx_create) and, for
+ *     pr_route_host, a staging area held by the context.
+ *   - Calls are asynchronous on the caller's CUDA stream (`stream` is a
+ *     cudaStream_t; NULL is the legacy default stream) unless stated.
+ *   - Argument and launch problems return a pr_status; problems in the data
+ *     (non-finite rows, bad token ids, bad offsets) never trap: they set the
+ *     PR_FLAG_* bits in the per-row / per-request flag outputs and in the
+ *     context's flag word (pr_ctx_flags).
+ *   - Logits are row-major [n_rows][row_stride] elements, bf16 or fp32;
+ *     only the first `vocab` entries of a row count.  Any element alignment is
+ *     accepted; rows whose start is 16-byte aligned (base pointer and
+ *     row_stride * element size multiples of 16) take the vector path.
+ *   - Token ids are int32 (V < 2^31); request offsets are int64 CSR: request r
+ *     owns rows [offsets[r], offsets[r+1]).
+ *   - Features are written as PR_NFEAT floats per row, in the order of the
+ *     PR_F_* slot names; pooled aggregates as PR_NAGG floats per request in
+ *     the order of the PR_A_* slot names.
+ *   - A row with NaN or +inf, or with no finite entry, has NaN features and
+ *     top indices -1 (PR_FLAG_NONFINITE); -inf is a masked token with p = 0.
+ *     A request with such a row, or with an out-of-range token id, has NaN
+ *     aggregates and score and does not ship.  An empty request (T = 0) has
+ *     NaN aggregates, score 0 and does not ship (PR_FLAG_EMPTY_REQ).
+ *   - All floating-point accumulation is fp32.
+ */
+#ifndef PRO_ROUTER_H
+#define PRO_ROUTER_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  PR_OK = 0,
+  PR_ERR_INVALID_ARG = -1, /* a null, negative, out-of-range or misaligned argument */
+  PR_ERR_UNSUPPORTED = -2, /* a device or mode this build cannot run */
+  PR_ERR_CUDA = -3,        /* a CUDA runtime call failed; see pr_last_cuda_error */
+  PR_ERR_NO_MEMORY = -4    /* a context allocation failed */
+} pr_status;
+
+typedef enum { PR_DTYPE_F32 = 0, PR_DTYPE_BF16 = 1 } pr_dtype;
+
+/* flag bits written on the device (never a trap) */
+#define PR_FLAG_NONFINITE 1u   /* NaN or +inf in the row, or no finite entry */
+#define PR_FLAG_BAD_CHOSEN 2u  /* emitted token id outside [0, vocab): l = NaN */
+#define PR_FLAG_EMPTY_REQ 4u   /* request with T = 0 */
+#define PR_FLAG_BAD_OFFSETS 8u /* offsets not monotone / outside the row range */
+#define PR_FLAG_BAD_SLOT 16u   /* decode slot id outside [0, n_slots) */
+
+/* per-row feature record, PR_NFEAT floats */
+#define PR_NFEAT 8
+#define PR_F_LOGP 0   /* l = log p(y)              (Eq. 3) */
+#define PR_F_MAXP 1   /* m = max_v p(v)            (Eq. 3) */
+#define PR_F_MARGIN 2 /* p(i1) - p(i2) */
+#define PR_F_ENT 3    /* H = -sum_v p log p        (full vocabulary) */
+#define PR_F_TOPK 4   /* h = -H^K                  (Eq. 3, K = topk) */
+#define PR_F_RHO 5    /* rho = t / T               (Eq. 3) */
+#define PR_F_LSE 6    /* log sum_v exp(x_v) */
+#define PR_F_X1 7     /* x_{i1}, the largest logit */
+
+/* per-request pooled aggregates, PR_NAGG floats: mean / min over t */
+#define PR_NAGG 11
+#define PR_A_MEAN_LOGP 0
+#define PR_A_MIN_LOGP 1
+#define PR_A_MEAN_MAXP 2
+#define PR_A_MIN_MAXP 3
+#define PR_A_MEAN_MARGIN 4
+#define PR_A_MIN_MARGIN 5
+#define PR_A_MEAN_NEGENT 6 /* mean of -H */
+#define PR_A_MIN_NEGENT 7  /* min of -H */
+#define PR_A_MEAN_TOPK 8   /* mean of h */
+#define PR_A_MIN_TOPK 9    /* min of h */
+#define PR_A_MEAN_RHO 10   /* (T + 1) / (2T) */
+
+#define PR_MAX_TOPK 32 /* largest K accepted (the paper uses K = 20) */
+
+/* options (pr_ctx_set_option) */
+#define PR_OPT_TOPK 0        /* K of the top-K entropy for pr_route / pr_decode_step; default 20 */
+#define PR_OPT_TOPK_RENORM 1 /* 0 (default): raw p over the top K; 1: renormalised over the top K */
+#define PR_OPT_SPLIT 2       /* CTAs per row (thread-block cluster): 0 = automatic, or 1, 2, 4, 8 */
+
+typedef struct pr_ctx pr_ctx;
+
+/* ---- context -------------------------------------------------------------- */
+
+/*
+ * Create a context on CUDA device `device`.  It owns the workspace of the
+ * fused and incremental calls: per-row records for up to `max_rows` rows of
+ * one routed batch (pr_route's global row index, row_base + local row, must
+ * stay below it), per-request completion counters for up to `max_requests`
+ * requests, and `max_requests` decode slots (pr_decode_step).  Everything is
+ * zeroed.  Synchronous.  Returns PR_ERR_INVALID_ARG for a null `ctx`, a
+ * negative size or a bad device, PR_ERR_NO_MEMORY if an allocation fails.
+ */
+pr_status pr_ctx_create(pr_ctx** ctx, int device, int64_t max_rows, int32_t max_requests);
+
+/* Free the context and its workspace (synchronises the device first). */
+pr_status pr_ctx_destroy(pr_ctx* ctx);
+
+/* Zero counters, decode slots and the flag word, on `stream`.  Needed only
+ * after a call that was given inconsistent offsets, slots or row ranges. */
+pr_status pr_ctx_reset(pr_ctx* ctx, void* stream);
+
+/* Set an option (PR_OPT_*).  Takes effect for calls issued afterwards. */
+pr_status pr_ctx_set_option(pr_ctx* ctx, int32_t option, int32_t value);
+
+/*
+ * OR of every flag bit any call on this context has raised since the last
+ * clear.  Synchronises `stream`.  With `clear` != 0 the word is zeroed.
+ */
+pr_status pr_ctx_flags(pr_ctx* ctx, void* stream, int32_t clear, uint32_t* flags);
+
+/* ---- the three verifier calls ----------------------------------------------- */
+
+/*
+ * Per-token features (Eq. 3) of n_rows logit rows.
+ *   logits     device, [n_rows][row_stride] elements of type `dt`
+ *   vocab      V, 1 <= V <= row_stride, V < 2^31
+ *   chosen     device int32 [n_rows], the emitted token y_t of each row
+ *   topk       K in [1, PR_MAX_TOPK] (the paper's K = 20)
+ *   offsets    device int64 [n_req + 1] or NULL; with offsets the position
+ *              fraction rho = t/T is filled in, without it rho = 0
+ *   feat       device float [n_rows][PR_NFEAT]           (output)
+ *   top2       device int32 [n_rows][2] = {i1, i2}: the first two tokens in
+ *              the order (value descending, index ascending); i2 = -1 if V = 1
+ *   row_flags  device uint32 [n_rows]                     (output)
+ * Every row is read once from device memory.  Uses the context's PR_OPT_SPLIT
+ * and PR_OPT_TOPK_RENORM options.
+ */
+pr_status pr_token_features(pr_ctx* ctx, const void* logits, pr_dtype dt, int64_t n_rows,
+                            int64_t vocab, int64_t row_stride, const int32_t* chosen,
+                            int32_t topk, const int64_t* offsets, int32_t n_req, float* feat,
+                            int32_t* top2, uint32_t* row_flags, void* stream);
+
+/*
+ * Pool per-row features into per-request aggregates, score and threshold
+ * (Section 3.1: mean pool, sigmoid score, ship iff score >= tau).
+ *   feat       device float [n_rows][PR_NFEAT] as written by pr_token_features,
+ *              16-byte aligned
+ *   row_flags  device uint32 [n_rows] or NULL (then no row is flagged)
+ *   n_rows     rows in feat; a request reaching past it gets PR_FLAG_BAD_OFFSETS
+ *   offsets    device int64 [n_req + 1]; rows [offsets[r], offsets[r+1]) are read
+ *   w          device float [PR_NAGG], b: bias; z = w . a + b, score = sigmoid(z)
+ *   tau        threshold in (0, 1); ship = (z >= log(tau / (1 - tau)))
+ *   agg        device float [n_req][PR_NAGG] or NULL      (output)
+ *   score      device float [n_req]                       (output)
+ *   ship       device uint8 [n_req], 1 = ship, 0 = escalate (output)
+ *   req_flags  device uint32 [n_req]                      (output)
+ * Sums run in a fixed order per request, so results do not depend on timing.
+ */
+pr_status pr_aggregate_score(pr_ctx* ctx, const float* feat, const uint32_t* row_flags,
+                             int64_t n_rows, const int64_t* offsets, int32_t n_req,
+                             const float* w, float b, float tau, float* agg, float* score,
+                             uint8_t* ship, uint32_t* req_flags, void* stream);
+
+/*
+ * Fused verification: logit rows -> ship / escalate, in one launch.  Rows are
+ * rows [row_base, row_base + n_rows) of a batch whose requests are described
+ * by `offsets` (global row indices, n_req + 1 entries, offsets[n_req] <=
+ * max_rows).  A batch may be fed in several chunks on one stream, each call
+ * with its own row_base, in any order, each row exactly once; a request that
+ * straddles chunks is finished by the call that delivers its last row.  Per
+ * request, when all its rows are done, the kernel that finished the last row
+ * pools, scores and writes score / ship / req_flags (and agg if not NULL).
+ * Empty requests are written by every call whose row range touches their
+ * offset.  K and the entropy mode come from the context options.
+ */
+pr_status pr_route(pr_ctx* ctx, const void* logits, pr_dtype dt, int64_t row_base,
+                   int64_t n_rows, int64_t vocab, int64_t row_stride, const int32_t* chosen,
+                   const int64_t* offsets, int32_t n_req, const float* w, float b, float tau,
+                   float* score, uint8_t* ship, uint32_t* req_flags, float* agg, void* stream);
+
+/*
+ * The same verification from HOST memory, end to end: the logits, token ids,
+ * offsets and weights are host buffers (pinned memory copies fastest); rows
+ * are copied to the device in chunks of `chunk_rows` rows through a
+ * double-buffered staging area owned by the context, overlapped with the
+ * fused kernel, and score / ship / req_flags (and agg if not NULL) are copied
+ * back to the host buffers.  Synchronous: returns when the host outputs are
+ * written.  The first call allocates the staging area (2 * chunk_rows rows).
+ */
+pr_status pr_route_host(pr_ctx* ctx, const void* logits, pr_dtype dt, int64_t n_rows,
+                        int64_t vocab, int64_t row_stride, const int32_t* chosen,
+                        const int64_t* offsets, int32_t n_req, const float* w, float b, float tau,
+                        int64_t chunk_rows, float* score, uint8_t* ship, uint32_t* req_flags,
+                        float* agg, void* stream);
+
+/* ---- incremental decode-step mode --------------------------------------------- */
+
+/*
+ * One decode step over n_live live requests, each in its own slot of the
+ * context (0 <= slot < max_requests, no slot twice in one step).  Row i of
+ * `logits` is the distribution that produced token chosen[i] of the request in
+ * slot[i].  Each row's features are folded in place into that slot's running
+ * accumulators (count, compensated sums, minima) in step order.  When eos[i]
+ * is non-zero the request ends with this row: its aggregates (mean rho =
+ * (T+1)/(2T)) are scored and thresholded, score_out / ship_out / slot_flags
+ * (and agg_out if not NULL) at index slot[i] are written, and the slot is
+ * cleared for the next request.  Output arrays have max_requests entries;
+ * entries of slots that did not end in this step are left untouched.
+ */
+pr_status pr_decode_step(pr_ctx* ctx, const void* logits, pr_dtype dt, int32_t n_live,
+                         int64_t vocab, int64_t row_stride, const int32_t* slot,
+                         const int32_t* chosen, const uint8_t* eos, const float* w, float b,
+                         float tau, float* score_out, uint8_t* ship_out, uint32_t* slot_flags,
+                         float* agg_out, void* stream);
+
+/*
+ * Checkpoint of the decode slots.  pr_state_export with host_buf == NULL
+ * stores the needed size in *bytes; otherwise it copies the state into
+ * host_buf (*bytes must be at least that size).  pr_state_import restores a
+ * state exported from a context with the same max_requests.  Both synchronise
+ * the device.
+ */
+pr_status pr_state_export(pr_ctx* ctx, void* host_buf, size_t* bytes);
+pr_status pr_state_import(pr_ctx* ctx, const void* host_buf, size_t bytes);
+
+/* ---- diagnostics ------------------------------------------------------------------ */
+
+/* Static description of a status code. */
+const char* pr_status_string(pr_status status);
+
+/* The CUDA error string of the last PR_ERR_CUDA on this thread ("" if none). */
+const char* pr_last_cuda_error(void);
+
+/* Number of kernel launches this library has issued in this process. */
+uint64_t pr_launch_count(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PRO_ROUTER_H */

@@ -1,0 +1,239 @@
+"""ctypes binding of libprorouter.so with the C ABI's call names.
+
+Argument marshalling only: tensors are passed as raw pointers, every step of
+the verifier runs in the library's CUDA kernels.  PyTorch provides device
+memory and streams.  Importing this module raises if the library is missing:
+there is no fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+import torch
+
+from .build import LIB
+
+PR_OK, PR_ERR_INVALID_ARG, PR_ERR_UNSUPPORTED, PR_ERR_CUDA, PR_ERR_NO_MEMORY = 0, -1, -2, -3, -4
+PR_DTYPE_F32, PR_DTYPE_BF16 = 0, 1
+PR_FLAG_NONFINITE, PR_FLAG_BAD_CHOSEN, PR_FLAG_EMPTY_REQ = 1, 2, 4
+PR_FLAG_BAD_OFFSETS, PR_FLAG_BAD_SLOT = 8, 16
+PR_NFEAT, PR_NAGG, PR_MAX_TOPK = 8, 11, 32
+PR_OPT_TOPK, PR_OPT_TOPK_RENORM, PR_OPT_SPLIT = 0, 1, 2
+
+# every symbol include/pro_router.h declares
+EXPORTS = (
+    "pr_ctx_create", "pr_ctx_destroy", "pr_ctx_reset", "pr_ctx_set_option", "pr_ctx_flags",
+    "pr_token_features", "pr_aggregate_score", "pr_route", "pr_route_host", "pr_decode_step",
+    "pr_state_export", "pr_state_import", "pr_status_string", "pr_last_cuda_error",
+    "pr_launch_count",
+)
+
+if not os.path.exists(LIB):
+    raise ImportError("libprorouter.so has not been built (python -m paper_2608_28726_gb300.build)")
+
+_P = ctypes.c_void_p
+_I32, _I64, _F32, _SZ = ctypes.c_int32, ctypes.c_int64, ctypes.c_float, ctypes.c_size_t
+_lib = ctypes.CDLL(LIB)
+_SIGS = {
+    "pr_ctx_create": [ctypes.POINTER(_P), ctypes.c_int, _I64, _I32],
+    "pr_ctx_destroy": [_P],
+    "pr_ctx_reset": [_P, _P],
+    "pr_ctx_set_option": [_P, _I32, _I32],
+    "pr_ctx_flags": [_P, _P, _I32, ctypes.POINTER(ctypes.c_uint32)],
+    "pr_token_features": [_P, _P, ctypes.c_int, _I64, _I64, _I64, _P, _I32, _P, _I32, _P, _P, _P,
+                          _P],
+    "pr_aggregate_score": [_P, _P, _P, _I64, _P, _I32, _P, _F32, _F32, _P, _P, _P, _P, _P],
+    "pr_route": [_P, _P, ctypes.c_int, _I64, _I64, _I64, _I64, _P, _P, _I32, _P, _F32, _F32, _P, _P,
+                 _P, _P, _P],
+    "pr_route_host": [_P, _P, ctypes.c_int, _I64, _I64, _I64, _P, _P, _I32, _P, _F32, _F32, _I64,
+                      _P, _P, _P, _P, _P],
+    "pr_decode_step": [_P, _P, ctypes.c_int, _I32, _I64, _I64, _P, _P, _P, _P, _F32, _F32, _P, _P,
+                       _P, _P, _P],
+    "pr_state_export": [_P, _P, ctypes.POINTER(_SZ)],
+    "pr_state_import": [_P, _P, _SZ],
+}
+for _name, _args in _SIGS.items():
+    _fn = getattr(_lib, _name)
+    _fn.argtypes = _args
+    _fn.restype = ctypes.c_int
+_lib.pr_status_string.argtypes = [ctypes.c_int]
+_lib.pr_status_string.restype = ctypes.c_char_p
+_lib.pr_last_cuda_error.argtypes = []
+_lib.pr_last_cuda_error.restype = ctypes.c_char_p
+_lib.pr_launch_count.argtypes = []
+_lib.pr_launch_count.restype = ctypes.c_uint64
+
+
+class PRError(RuntimeError):
+    def __init__(self, status: int, call: str):
+        msg = _lib.pr_status_string(status).decode()
+        if status == PR_ERR_CUDA:
+            msg += " (" + _lib.pr_last_cuda_error().decode() + ")"
+        super().__init__("%s: %s" % (call, msg))
+        self.status = status
+
+
+def _check(st: int, call: str):
+    if st != PR_OK:
+        raise PRError(st, call)
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    if isinstance(t, torch.Tensor):
+        return ctypes.c_void_p(t.data_ptr())
+    if isinstance(t, np.ndarray):
+        return t.ctypes.data_as(ctypes.c_void_p)
+    raise TypeError(type(t))
+
+
+def _stream(stream):
+    if stream is None:
+        return ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    if isinstance(stream, torch.cuda.Stream):
+        return ctypes.c_void_p(stream.cuda_stream)
+    return ctypes.c_void_p(int(stream))
+
+
+def _dtype(t: torch.Tensor) -> int:
+    if t.dtype == torch.bfloat16:
+        return PR_DTYPE_BF16
+    if t.dtype == torch.float32:
+        return PR_DTYPE_F32
+    raise TypeError("logits must be bfloat16 or float32")
+
+
+def _rows(logits: torch.Tensor, vocab):
+    if logits.dim() != 2 or (logits.size(1) > 1 and logits.stride(1) != 1):
+        raise ValueError("logits must be 2-D with unit stride along the vocabulary")
+    stride = logits.stride(0) if logits.size(0) > 1 else logits.size(1)
+    V = logits.size(1) if vocab is None else int(vocab)
+    return V, max(stride, V)
+
+
+def launch_count() -> int:
+    return int(_lib.pr_launch_count())
+
+
+def pr_status_string(status: int) -> str:
+    return _lib.pr_status_string(status).decode()
+
+
+# ---- context ---------------------------------------------------------------------
+
+def pr_ctx_create(device: int = 0, max_rows: int = 0, max_requests: int = 0):
+    h = ctypes.c_void_p()
+    _check(_lib.pr_ctx_create(ctypes.byref(h), int(device), int(max_rows), int(max_requests)),
+           "pr_ctx_create")
+    return h
+
+
+def pr_ctx_destroy(ctx):
+    _check(_lib.pr_ctx_destroy(ctx), "pr_ctx_destroy")
+
+
+def pr_ctx_reset(ctx, stream=None):
+    _check(_lib.pr_ctx_reset(ctx, _stream(stream)), "pr_ctx_reset")
+
+
+def pr_ctx_set_option(ctx, option: int, value: int):
+    _check(_lib.pr_ctx_set_option(ctx, int(option), int(value)), "pr_ctx_set_option")
+
+
+def pr_ctx_flags(ctx, stream=None, clear: bool = False) -> int:
+    v = ctypes.c_uint32(0)
+    _check(_lib.pr_ctx_flags(ctx, _stream(stream), int(bool(clear)), ctypes.byref(v)),
+           "pr_ctx_flags")
+    return int(v.value)
+
+
+# ---- verifier calls ------------------------------------------------------------------
+
+def pr_token_features(ctx, logits, chosen, topk: int = 20, offsets=None, feat=None, top2=None,
+                      row_flags=None, vocab=None, stream=None):
+    n = logits.size(0)
+    V, stride = _rows(logits, vocab)
+    dev = logits.device
+    feat = torch.empty(n, PR_NFEAT, dtype=torch.float32, device=dev) if feat is None else feat
+    top2 = torch.empty(n, 2, dtype=torch.int32, device=dev) if top2 is None else top2
+    row_flags = torch.empty(n, dtype=torch.int32, device=dev) if row_flags is None else row_flags
+    n_req = 0 if offsets is None else offsets.numel() - 1
+    _check(_lib.pr_token_features(ctx, _ptr(logits), _dtype(logits), n, V, stride, _ptr(chosen),
+                                  int(topk), _ptr(offsets), n_req, _ptr(feat), _ptr(top2),
+                                  _ptr(row_flags), _stream(stream)), "pr_token_features")
+    return feat, top2, row_flags
+
+
+def pr_aggregate_score(ctx, feat, offsets, w, b: float, tau: float, row_flags=None, agg=None,
+                       score=None, ship=None, req_flags=None, stream=None):
+    n_req = offsets.numel() - 1
+    dev = feat.device
+    agg = torch.empty(n_req, PR_NAGG, dtype=torch.float32, device=dev) if agg is None else agg
+    score = torch.empty(n_req, dtype=torch.float32, device=dev) if score is None else score
+    ship = torch.empty(n_req, dtype=torch.uint8, device=dev) if ship is None else ship
+    req_flags = torch.empty(n_req, dtype=torch.int32, device=dev) if req_flags is None else req_flags
+    _check(_lib.pr_aggregate_score(ctx, _ptr(feat), _ptr(row_flags), feat.size(0), _ptr(offsets),
+                                   n_req, _ptr(w), float(b), float(tau), _ptr(agg), _ptr(score),
+                                   _ptr(ship), _ptr(req_flags), _stream(stream)),
+           "pr_aggregate_score")
+    return agg, score, ship, req_flags
+
+
+def pr_route(ctx, logits, chosen, offsets, w, b: float, tau: float, row_base: int = 0, score=None,
+             ship=None, req_flags=None, agg=None, vocab=None, stream=None, want_agg: bool = True):
+    n = logits.size(0)
+    V, stride = _rows(logits, vocab)
+    n_req = offsets.numel() - 1
+    dev = logits.device
+    score = torch.empty(n_req, dtype=torch.float32, device=dev) if score is None else score
+    ship = torch.empty(n_req, dtype=torch.uint8, device=dev) if ship is None else ship
+    req_flags = torch.empty(n_req, dtype=torch.int32, device=dev) if req_flags is None else req_flags
+    if agg is None and want_agg:
+        agg = torch.empty(n_req, PR_NAGG, dtype=torch.float32, device=dev)
+    _check(_lib.pr_route(ctx, _ptr(logits), _dtype(logits), int(row_base), n, V, stride,
+                         _ptr(chosen), _ptr(offsets), n_req, _ptr(w), float(b), float(tau),
+                         _ptr(score), _ptr(ship), _ptr(req_flags), _ptr(agg), _stream(stream)),
+           "pr_route")
+    return score, ship, req_flags, agg
+
+
+def pr_route_host(ctx, logits, chosen, offsets, w, b: float, tau: float, chunk_rows: int = 8192,
+                  score=None, ship=None, req_flags=None, agg=None, vocab=None, stream=None):
+    """Host tensors in, host tensors out (pinned host memory copies fastest)."""
+    n = logits.size(0)
+    V, stride = _rows(logits, vocab)
+    n_req = offsets.numel() - 1
+    score = torch.empty(n_req, dtype=torch.float32) if score is None else score
+    ship = torch.empty(n_req, dtype=torch.uint8) if ship is None else ship
+    req_flags = torch.empty(n_req, dtype=torch.int32) if req_flags is None else req_flags
+    _check(_lib.pr_route_host(ctx, _ptr(logits), _dtype(logits), n, V, stride, _ptr(chosen),
+                              _ptr(offsets), n_req, _ptr(w), float(b), float(tau), int(chunk_rows),
+                              _ptr(score), _ptr(ship), _ptr(req_flags), _ptr(agg),
+                              _stream(stream)), "pr_route_host")
+    return score, ship, req_flags, agg
+
+
+def pr_decode_step(ctx, logits, slot, chosen, eos, w, b: float, tau: float, score_out, ship_out,
+                   slot_flags, agg_out=None, vocab=None, stream=None):
+    n = logits.size(0)
+    V, stride = _rows(logits, vocab)
+    _check(_lib.pr_decode_step(ctx, _ptr(logits), _dtype(logits), n, V, stride, _ptr(slot),
+                               _ptr(chosen), _ptr(eos), _ptr(w), float(b), float(tau),
+                               _ptr(score_out), _ptr(ship_out), _ptr(slot_flags), _ptr(agg_out),
+                               _stream(stream)), "pr_decode_step")
+
+
+def pr_state_export(ctx) -> bytes:
+    size = ctypes.c_size_t(0)
+    _check(_lib.pr_state_export(ctx, None, ctypes.byref(size)), "pr_state_export")
+    buf = ctypes.create_string_buffer(size.value)
+    _check(_lib.pr_state_export(ctx, buf, ctypes.byref(size)), "pr_state_export")
+    return buf.raw[:size.value]
+
+
+def pr_state_import(ctx, state: bytes):
+    buf = ctypes.create_string_buffer(state, len(state))
+    _check(_lib.pr_state_import(ctx, buf, len(state)), "pr_state_import")

@@ -1,0 +1,568 @@
+// Host side of the C ABI declared in include/pro_router.h: argument checks,
+// context workspace, launch configuration and the host-memory pipeline.
+#include <cuda_runtime.h>
+
+#include <atomic>
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <new>
+
+#include "pr_kernels.cuh"
+#include "pro_router.h"
+
+namespace {
+
+thread_local char g_cuda_err[256] = "";
+std::atomic<uint64_t> g_launches{0};
+
+pr_status cuda_fail(cudaError_t e, const char* what) {
+  snprintf(g_cuda_err, sizeof g_cuda_err, "%s: %s", what, cudaGetErrorString(e));
+  return PR_ERR_CUDA;
+}
+
+#define PR_CUDA(call)                                   \
+  do {                                                  \
+    cudaError_t e_ = (call);                            \
+    if (e_ != cudaSuccess) return cuda_fail(e_, #call); \
+  } while (0)
+
+constexpr uint32_t STATE_MAGIC = 0x50525354u;  // "PRST"
+constexpr uint32_t STATE_VERSION = 1u;
+
+}  // namespace
+
+struct pr_ctx {
+  int device = 0;
+  int num_sms = 0;
+  int64_t max_rows = 0;
+  int32_t max_requests = 0;
+  // options
+  int32_t topk = 20, renorm = 0, split = 0;
+  // workspace
+  float* rec = nullptr;          // [max_rows][8] per-row records of pr_route
+  uint32_t* rec_flags = nullptr; // [max_rows]
+  int32_t* req_cnt = nullptr;    // [max_requests] completion counters
+  float* acc = nullptr;          // [max_requests][ACC_WORDS] decode slots
+  uint32_t* flags = nullptr;     // flag word
+  // pr_route_host staging (allocated on first use)
+  void* stage[2] = {nullptr, nullptr};
+  int32_t* stage_chosen[2] = {nullptr, nullptr};
+  int64_t stage_rows = 0;
+  size_t stage_row_bytes = 0;
+  int64_t* h_offsets_dev = nullptr;
+  int32_t h_offsets_cap = 0;
+  float* h_w_dev = nullptr;
+  float* h_out = nullptr;        // [max_requests][NAGG + 1] scores and aggregates
+  uint8_t* h_ship_dev = nullptr;
+  uint32_t* h_flags_dev = nullptr;
+  cudaStream_t copy_stream = nullptr;
+  cudaEvent_t ev_copied[2] = {nullptr, nullptr};
+  cudaEvent_t ev_free[2] = {nullptr, nullptr};
+  // occupancy cache per (dtype, mode)
+  int bps[2][3] = {{0, 0, 0}, {0, 0, 0}};
+};
+
+namespace {
+
+template <typename T, int MODE>
+void* kernel_ptr() {
+  return reinterpret_cast<void*>(&prk::verify_rows<T, MODE>);
+}
+
+void* row_kernel(pr_dtype dt, int mode) {
+  if (dt == PR_DTYPE_BF16) {
+    if (mode == prk::MODE_FEATURES) return kernel_ptr<__nv_bfloat16, prk::MODE_FEATURES>();
+    if (mode == prk::MODE_ROUTE) return kernel_ptr<__nv_bfloat16, prk::MODE_ROUTE>();
+    return kernel_ptr<__nv_bfloat16, prk::MODE_DECODE>();
+  }
+  if (mode == prk::MODE_FEATURES) return kernel_ptr<float, prk::MODE_FEATURES>();
+  if (mode == prk::MODE_ROUTE) return kernel_ptr<float, prk::MODE_ROUTE>();
+  return kernel_ptr<float, prk::MODE_DECODE>();
+}
+
+int blocks_per_sm(pr_ctx* c, pr_dtype dt, int mode) {
+  int& v = c->bps[dt == PR_DTYPE_BF16 ? 1 : 0][mode];
+  if (v == 0) {
+    int n = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, row_kernel(dt, mode), prk::NT, 0) !=
+            cudaSuccess ||
+        n <= 0)
+      n = 1;
+    v = n;
+  }
+  return v;
+}
+
+// CTAs per row: the forced option, or enough to put two waves of CTAs on the GPU
+int choose_split(pr_ctx* c, pr_dtype dt, int mode, int64_t n_rows) {
+  if (c->split == 1 || c->split == 2 || c->split == 4 || c->split == 8) return c->split;
+  const int64_t slots = (int64_t)c->num_sms * blocks_per_sm(c, dt, mode);
+  int s = 1;
+  while (s < prk::MAXC && n_rows * s < 2 * slots) s <<= 1;
+  return s;
+}
+
+pr_status launch_rows(pr_ctx* c, pr_dtype dt, int mode, const prk::Args& a, cudaStream_t st) {
+  if (a.n_rows == 0) return PR_OK;
+  const int C = choose_split(c, dt, mode, a.n_rows);
+  if (a.n_rows * C > 0x7fffffffLL) return PR_ERR_INVALID_ARG;
+  cudaLaunchConfig_t cfg;
+  memset(&cfg, 0, sizeof cfg);
+  cfg.gridDim = dim3((unsigned)(a.n_rows * C), 1, 1);
+  cfg.blockDim = dim3(prk::NT, 1, 1);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = (unsigned)C;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = C > 1 ? 1 : 0;
+  void* args[] = {const_cast<prk::Args*>(&a)};
+  PR_CUDA(cudaLaunchKernelExC(&cfg, row_kernel(dt, mode), args));
+  g_launches.fetch_add(1, std::memory_order_relaxed);
+  return PR_OK;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+size_t esize(pr_dtype dt) { return dt == PR_DTYPE_BF16 ? 2 : 4; }
+
+bool valid_dtype(pr_dtype dt) { return dt == PR_DTYPE_F32 || dt == PR_DTYPE_BF16; }
+
+// the part of the row checks shared by every entry point
+pr_status check_rows(pr_dtype dt, const void* logits, int64_t n_rows, int64_t vocab,
+                     int64_t row_stride) {
+  if (!valid_dtype(dt)) return PR_ERR_INVALID_ARG;
+  if (n_rows < 0 || vocab <= 0 || vocab > 0x7fffffffLL || row_stride < vocab)
+    return PR_ERR_INVALID_ARG;
+  if (n_rows > 0 && !logits) return PR_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(logits) % esize(dt)) != 0) return PR_ERR_INVALID_ARG;
+  return PR_OK;
+}
+
+void fill_row_args(prk::Args& a, const void* logits, pr_dtype dt, int64_t n_rows, int64_t vocab,
+                   int64_t row_stride, const int32_t* chosen, int32_t topk, int32_t renorm) {
+  memset(&a, 0, sizeof a);
+  a.logits = logits;
+  a.n_rows = n_rows;
+  a.vocab = vocab;
+  a.row_stride = row_stride;
+  a.chosen = chosen;
+  a.topk = topk;
+  a.kc = topk > 2 ? topk : 2;
+  a.renorm = renorm;
+  a.aligned = aligned16(logits) && ((row_stride * (int64_t)esize(dt)) % 16) == 0;
+}
+
+float zthreshold(float tau) {
+  const double t = (double)tau;
+  if (!(t > 0.0)) return -INFINITY;
+  if (!(t < 1.0)) return INFINITY;
+  return (float)std::log(t / (1.0 - t));
+}
+
+pr_status set_device(pr_ctx* c) {
+  PR_CUDA(cudaSetDevice(c->device));
+  return PR_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* pr_status_string(pr_status s) {
+  switch (s) {
+    case PR_OK:
+      return "ok";
+    case PR_ERR_INVALID_ARG:
+      return "invalid argument";
+    case PR_ERR_UNSUPPORTED:
+      return "unsupported";
+    case PR_ERR_CUDA:
+      return "CUDA error";
+    case PR_ERR_NO_MEMORY:
+      return "out of memory";
+  }
+  return "unknown status";
+}
+
+const char* pr_last_cuda_error(void) { return g_cuda_err; }
+
+uint64_t pr_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
+
+pr_status pr_ctx_create(pr_ctx** out, int device, int64_t max_rows, int32_t max_requests) {
+  if (!out || max_rows < 0 || max_requests < 0) return PR_ERR_INVALID_ARG;
+  *out = nullptr;
+  int ndev = 0;
+  if (cudaGetDeviceCount(&ndev) != cudaSuccess || device < 0 || device >= ndev)
+    return PR_ERR_INVALID_ARG;
+  pr_ctx* c = new (std::nothrow) pr_ctx();
+  if (!c) return PR_ERR_NO_MEMORY;
+  c->device = device;
+  c->max_rows = max_rows;
+  c->max_requests = max_requests;
+  pr_status st = set_device(c);
+  if (st != PR_OK) {
+    delete c;
+    return st;
+  }
+  cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, device);
+  int major = 0;
+  cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, device);
+  if (major < 10) {
+    delete c;
+    return PR_ERR_UNSUPPORTED;
+  }
+  bool ok = true;
+  auto alloc = [&](void** p, size_t bytes) {
+    if (!ok) return;
+    if (bytes == 0) bytes = 16;
+    if (cudaMalloc(p, bytes) != cudaSuccess || cudaMemset(*p, 0, bytes) != cudaSuccess) ok = false;
+  };
+  alloc(reinterpret_cast<void**>(&c->rec), (size_t)max_rows * prk::NFEAT * sizeof(float));
+  alloc(reinterpret_cast<void**>(&c->rec_flags), (size_t)max_rows * sizeof(uint32_t));
+  alloc(reinterpret_cast<void**>(&c->req_cnt), (size_t)max_requests * sizeof(int32_t));
+  alloc(reinterpret_cast<void**>(&c->acc), (size_t)max_requests * prk::ACC_WORDS * sizeof(float));
+  alloc(reinterpret_cast<void**>(&c->flags), sizeof(uint32_t));
+  if (!ok || cudaDeviceSynchronize() != cudaSuccess) {
+    cudaGetLastError();
+    pr_ctx_destroy(c);
+    return PR_ERR_NO_MEMORY;
+  }
+  *out = c;
+  return PR_OK;
+}
+
+pr_status pr_ctx_destroy(pr_ctx* c) {
+  if (!c) return PR_ERR_INVALID_ARG;
+  cudaSetDevice(c->device);
+  cudaDeviceSynchronize();
+  cudaFree(c->rec);
+  cudaFree(c->rec_flags);
+  cudaFree(c->req_cnt);
+  cudaFree(c->acc);
+  cudaFree(c->flags);
+  for (int i = 0; i < 2; ++i) {
+    cudaFree(c->stage[i]);
+    cudaFree(c->stage_chosen[i]);
+    if (c->ev_copied[i]) cudaEventDestroy(c->ev_copied[i]);
+    if (c->ev_free[i]) cudaEventDestroy(c->ev_free[i]);
+  }
+  cudaFree(c->h_offsets_dev);
+  cudaFree(c->h_w_dev);
+  cudaFree(c->h_out);
+  cudaFree(c->h_ship_dev);
+  cudaFree(c->h_flags_dev);
+  if (c->copy_stream) cudaStreamDestroy(c->copy_stream);
+  delete c;
+  return PR_OK;
+}
+
+pr_status pr_ctx_reset(pr_ctx* c, void* stream) {
+  if (!c) return PR_ERR_INVALID_ARG;
+  pr_status st = set_device(c);
+  if (st != PR_OK) return st;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  PR_CUDA(cudaMemsetAsync(c->req_cnt, 0, (size_t)c->max_requests * sizeof(int32_t) + 0, s));
+  PR_CUDA(cudaMemsetAsync(c->acc, 0, (size_t)c->max_requests * prk::ACC_WORDS * sizeof(float), s));
+  PR_CUDA(cudaMemsetAsync(c->flags, 0, sizeof(uint32_t), s));
+  return PR_OK;
+}
+
+pr_status pr_ctx_set_option(pr_ctx* c, int32_t option, int32_t value) {
+  if (!c) return PR_ERR_INVALID_ARG;
+  switch (option) {
+    case PR_OPT_TOPK:
+      if (value < 1 || value > PR_MAX_TOPK) return PR_ERR_INVALID_ARG;
+      c->topk = value;
+      return PR_OK;
+    case PR_OPT_TOPK_RENORM:
+      if (value != 0 && value != 1) return PR_ERR_INVALID_ARG;
+      c->renorm = value;
+      return PR_OK;
+    case PR_OPT_SPLIT:
+      if (value != 0 && value != 1 && value != 2 && value != 4 && value != 8)
+        return PR_ERR_INVALID_ARG;
+      c->split = value;
+      return PR_OK;
+  }
+  return PR_ERR_INVALID_ARG;
+}
+
+pr_status pr_ctx_flags(pr_ctx* c, void* stream, int32_t clear, uint32_t* flags) {
+  if (!c || !flags) return PR_ERR_INVALID_ARG;
+  pr_status st = set_device(c);
+  if (st != PR_OK) return st;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  uint32_t v = 0;
+  PR_CUDA(cudaMemcpyAsync(&v, c->flags, sizeof v, cudaMemcpyDeviceToHost, s));
+  if (clear) PR_CUDA(cudaMemsetAsync(c->flags, 0, sizeof(uint32_t), s));
+  PR_CUDA(cudaStreamSynchronize(s));
+  *flags = v;
+  return PR_OK;
+}
+
+pr_status pr_token_features(pr_ctx* c, const void* logits, pr_dtype dt, int64_t n_rows,
+                            int64_t vocab, int64_t row_stride, const int32_t* chosen,
+                            int32_t topk, const int64_t* offsets, int32_t n_req, float* feat,
+                            int32_t* top2, uint32_t* row_flags, void* stream) {
+  if (!c) return PR_ERR_INVALID_ARG;
+  pr_status st = check_rows(dt, logits, n_rows, vocab, row_stride);
+  if (st != PR_OK) return st;
+  if (topk < 1 || topk > PR_MAX_TOPK || n_req < 0) return PR_ERR_INVALID_ARG;
+  if (n_rows > 0 && (!chosen || !feat || !top2 || !row_flags)) return PR_ERR_INVALID_ARG;
+  if (offsets && n_req < 1) return PR_ERR_INVALID_ARG;
+  if ((st = set_device(c)) != PR_OK) return st;
+  prk::Args a;
+  fill_row_args(a, logits, dt, n_rows, vocab, row_stride, chosen, topk, c->renorm);
+  a.offsets = offsets;
+  a.n_req = offsets ? n_req : 0;
+  a.feat = feat;
+  a.top2 = top2;
+  a.row_flags = row_flags;
+  a.ctx_flags = c->flags;
+  return launch_rows(c, dt, prk::MODE_FEATURES, a, reinterpret_cast<cudaStream_t>(stream));
+}
+
+pr_status pr_aggregate_score(pr_ctx* c, const float* feat, const uint32_t* row_flags,
+                             int64_t n_rows, const int64_t* offsets, int32_t n_req,
+                             const float* w, float b, float tau, float* agg, float* score,
+                             uint8_t* ship, uint32_t* req_flags, void* stream) {
+  if (!c || n_req < 0 || n_rows < 0) return PR_ERR_INVALID_ARG;
+  if (n_req == 0) return PR_OK;
+  if (!offsets || !w || !score || !ship || !req_flags) return PR_ERR_INVALID_ARG;
+  if (n_rows > 0 && !feat) return PR_ERR_INVALID_ARG;
+  if (!aligned16(feat)) return PR_ERR_INVALID_ARG;
+  pr_status st = set_device(c);
+  if (st != PR_OK) return st;
+  prk::AggArgs a;
+  memset(&a, 0, sizeof a);
+  a.feat = feat;
+  a.row_flags = row_flags;
+  a.n_rows = n_rows;
+  a.offsets = offsets;
+  a.n_req = n_req;
+  a.w = w;
+  a.b = b;
+  a.zthr = zthreshold(tau);
+  a.agg = agg;
+  a.score = score;
+  a.ship = ship;
+  a.req_flags = req_flags;
+  a.ctx_flags = c->flags;
+  const unsigned grid = (unsigned)((n_req + prk::NWARP - 1) / prk::NWARP);
+  prk::pool_requests<<<grid, prk::NT, 0, reinterpret_cast<cudaStream_t>(stream)>>>(a);
+  PR_CUDA(cudaGetLastError());
+  g_launches.fetch_add(1, std::memory_order_relaxed);
+  return PR_OK;
+}
+
+pr_status pr_route(pr_ctx* c, const void* logits, pr_dtype dt, int64_t row_base,
+                   int64_t n_rows, int64_t vocab, int64_t row_stride, const int32_t* chosen,
+                   const int64_t* offsets, int32_t n_req, const float* w, float b, float tau,
+                   float* score, uint8_t* ship, uint32_t* req_flags, float* agg, void* stream) {
+  if (!c) return PR_ERR_INVALID_ARG;
+  pr_status st = check_rows(dt, logits, n_rows, vocab, row_stride);
+  if (st != PR_OK) return st;
+  if (n_req < 1 || n_req > c->max_requests || row_base < 0 || row_base + n_rows > c->max_rows)
+    return PR_ERR_INVALID_ARG;
+  if (!offsets || !w || !score || !ship || !req_flags || (n_rows > 0 && !chosen))
+    return PR_ERR_INVALID_ARG;
+  if ((st = set_device(c)) != PR_OK) return st;
+  prk::Args a;
+  fill_row_args(a, logits, dt, n_rows, vocab, row_stride, chosen, c->topk, c->renorm);
+  a.offsets = offsets;
+  a.n_req = n_req;
+  a.row_base = row_base;
+  a.rec = c->rec;
+  a.rec_flags = c->rec_flags;
+  a.req_cnt = c->req_cnt;
+  a.max_rows = c->max_rows;
+  a.w = w;
+  a.b = b;
+  a.zthr = zthreshold(tau);
+  a.score = score;
+  a.ship = ship;
+  a.req_flags = req_flags;
+  a.agg = agg;
+  a.ctx_flags = c->flags;
+  return launch_rows(c, dt, prk::MODE_ROUTE, a, reinterpret_cast<cudaStream_t>(stream));
+}
+
+pr_status pr_decode_step(pr_ctx* c, const void* logits, pr_dtype dt, int32_t n_live,
+                         int64_t vocab, int64_t row_stride, const int32_t* slot,
+                         const int32_t* chosen, const uint8_t* eos, const float* w, float b,
+                         float tau, float* score_out, uint8_t* ship_out, uint32_t* slot_flags,
+                         float* agg_out, void* stream) {
+  if (!c) return PR_ERR_INVALID_ARG;
+  pr_status st = check_rows(dt, logits, n_live, vocab, row_stride);
+  if (st != PR_OK) return st;
+  if (n_live > c->max_requests) return PR_ERR_INVALID_ARG;
+  if (n_live > 0 && (!slot || !chosen || !eos || !w || !score_out || !ship_out || !slot_flags))
+    return PR_ERR_INVALID_ARG;
+  if ((st = set_device(c)) != PR_OK) return st;
+  prk::Args a;
+  fill_row_args(a, logits, dt, n_live, vocab, row_stride, chosen, c->topk, c->renorm);
+  a.slot = slot;
+  a.eos = eos;
+  a.acc = c->acc;
+  a.n_slots = c->max_requests;
+  a.w = w;
+  a.b = b;
+  a.zthr = zthreshold(tau);
+  a.score = score_out;
+  a.ship = ship_out;
+  a.req_flags = slot_flags;
+  a.agg = agg_out;
+  a.ctx_flags = c->flags;
+  return launch_rows(c, dt, prk::MODE_DECODE, a, reinterpret_cast<cudaStream_t>(stream));
+}
+
+pr_status pr_state_export(pr_ctx* c, void* host_buf, size_t* bytes) {
+  if (!c || !bytes) return PR_ERR_INVALID_ARG;
+  const size_t body = (size_t)c->max_requests * prk::ACC_WORDS * sizeof(float);
+  const size_t need = 4 * sizeof(uint32_t) + body;
+  if (!host_buf) {
+    *bytes = need;
+    return PR_OK;
+  }
+  if (*bytes < need) return PR_ERR_INVALID_ARG;
+  pr_status st = set_device(c);
+  if (st != PR_OK) return st;
+  PR_CUDA(cudaDeviceSynchronize());
+  uint32_t hdr[4] = {STATE_MAGIC, STATE_VERSION, (uint32_t)c->max_requests,
+                     (uint32_t)prk::ACC_WORDS};
+  memcpy(host_buf, hdr, sizeof hdr);
+  if (body) PR_CUDA(cudaMemcpy(static_cast<char*>(host_buf) + sizeof hdr, c->acc, body,
+                               cudaMemcpyDeviceToHost));
+  *bytes = need;
+  return PR_OK;
+}
+
+pr_status pr_state_import(pr_ctx* c, const void* host_buf, size_t bytes) {
+  if (!c || !host_buf) return PR_ERR_INVALID_ARG;
+  const size_t body = (size_t)c->max_requests * prk::ACC_WORDS * sizeof(float);
+  uint32_t hdr[4];
+  if (bytes != sizeof hdr + body) return PR_ERR_INVALID_ARG;
+  memcpy(hdr, host_buf, sizeof hdr);
+  if (hdr[0] != STATE_MAGIC || hdr[1] != STATE_VERSION || hdr[2] != (uint32_t)c->max_requests ||
+      hdr[3] != (uint32_t)prk::ACC_WORDS)
+    return PR_ERR_INVALID_ARG;
+  pr_status st = set_device(c);
+  if (st != PR_OK) return st;
+  PR_CUDA(cudaDeviceSynchronize());
+  if (body) PR_CUDA(cudaMemcpy(c->acc, static_cast<const char*>(host_buf) + sizeof hdr, body,
+                               cudaMemcpyHostToDevice));
+  return PR_OK;
+}
+
+pr_status pr_route_host(pr_ctx* c, const void* logits, pr_dtype dt, int64_t n_rows,
+                        int64_t vocab, int64_t row_stride, const int32_t* chosen,
+                        const int64_t* offsets, int32_t n_req, const float* w, float b, float tau,
+                        int64_t chunk_rows, float* score, uint8_t* ship, uint32_t* req_flags,
+                        float* agg, void* stream) {
+  if (!c) return PR_ERR_INVALID_ARG;
+  pr_status st = check_rows(dt, logits, n_rows, vocab, row_stride);
+  if (st != PR_OK) return st;
+  if (n_req < 1 || n_req > c->max_requests || n_rows > c->max_rows || chunk_rows < 1)
+    return PR_ERR_INVALID_ARG;
+  if (!offsets || !w || !score || !ship || !req_flags || (n_rows > 0 && !chosen))
+    return PR_ERR_INVALID_ARG;
+  if ((st = set_device(c)) != PR_OK) return st;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const size_t row_bytes = (size_t)row_stride * esize(dt);
+
+  // staging: two chunks of rows, token ids, the offsets, weights and outputs
+  if (c->stage_rows < chunk_rows || c->stage_row_bytes != row_bytes) {
+    for (int i = 0; i < 2; ++i) {
+      cudaFree(c->stage[i]);
+      cudaFree(c->stage_chosen[i]);
+      c->stage[i] = nullptr;
+      c->stage_chosen[i] = nullptr;
+    }
+    c->stage_rows = 0;
+    for (int i = 0; i < 2; ++i) {
+      if (cudaMalloc(&c->stage[i], (size_t)chunk_rows * row_bytes) != cudaSuccess ||
+          cudaMalloc(reinterpret_cast<void**>(&c->stage_chosen[i]),
+                     (size_t)chunk_rows * sizeof(int32_t)) != cudaSuccess) {
+        cudaGetLastError();
+        return PR_ERR_NO_MEMORY;
+      }
+    }
+    c->stage_rows = chunk_rows;
+    c->stage_row_bytes = row_bytes;
+  }
+  if (!c->copy_stream) {
+    PR_CUDA(cudaStreamCreateWithFlags(&c->copy_stream, cudaStreamNonBlocking));
+    for (int i = 0; i < 2; ++i) {
+      PR_CUDA(cudaEventCreateWithFlags(&c->ev_copied[i], cudaEventDisableTiming));
+      PR_CUDA(cudaEventCreateWithFlags(&c->ev_free[i], cudaEventDisableTiming));
+    }
+  }
+  if (c->h_offsets_cap < n_req + 1) {
+    cudaFree(c->h_offsets_dev);
+    c->h_offsets_dev = nullptr;
+    c->h_offsets_cap = 0;
+    if (cudaMalloc(reinterpret_cast<void**>(&c->h_offsets_dev), (size_t)(n_req + 1) * sizeof(int64_t)) !=
+        cudaSuccess) {
+      cudaGetLastError();
+      return PR_ERR_NO_MEMORY;
+    }
+    c->h_offsets_cap = n_req + 1;
+  }
+  if (!c->h_w_dev) {
+    bool ok = cudaMalloc(reinterpret_cast<void**>(&c->h_w_dev), prk::NAGG * sizeof(float)) == cudaSuccess &&
+              cudaMalloc(reinterpret_cast<void**>(&c->h_out),
+                         (size_t)(c->max_requests > 0 ? c->max_requests : 1) * (prk::NAGG + 1) *
+                             sizeof(float)) == cudaSuccess &&
+              cudaMalloc(reinterpret_cast<void**>(&c->h_ship_dev), (size_t)(c->max_requests + 1)) ==
+                  cudaSuccess &&
+              cudaMalloc(reinterpret_cast<void**>(&c->h_flags_dev),
+                         (size_t)(c->max_requests + 1) * sizeof(uint32_t)) == cudaSuccess;
+    if (!ok) {
+      cudaGetLastError();
+      return PR_ERR_NO_MEMORY;
+    }
+  }
+  float* d_score = c->h_out;
+  float* d_agg = c->h_out + c->max_requests;
+  PR_CUDA(cudaMemcpyAsync(c->h_offsets_dev, offsets, (size_t)(n_req + 1) * sizeof(int64_t),
+                          cudaMemcpyHostToDevice, s));
+  PR_CUDA(cudaMemcpyAsync(c->h_w_dev, w, prk::NAGG * sizeof(float), cudaMemcpyHostToDevice, s));
+
+  // chunk i: copy on copy_stream into buffer i % 2, route on s
+  const int64_t nchunks = (n_rows + chunk_rows - 1) / chunk_rows;
+  PR_CUDA(cudaEventRecord(c->ev_free[0], s));
+  PR_CUDA(cudaEventRecord(c->ev_free[1], s));
+  for (int64_t i = 0; i < nchunks; ++i) {
+    const int j = (int)(i & 1);
+    const int64_t r0 = i * chunk_rows;
+    const int64_t nr = (r0 + chunk_rows <= n_rows) ? chunk_rows : n_rows - r0;
+    PR_CUDA(cudaStreamWaitEvent(c->copy_stream, c->ev_free[j], 0));
+    PR_CUDA(cudaMemcpyAsync(c->stage[j], static_cast<const char*>(logits) + (size_t)r0 * row_bytes,
+                            (size_t)nr * row_bytes, cudaMemcpyHostToDevice, c->copy_stream));
+    PR_CUDA(cudaMemcpyAsync(c->stage_chosen[j], chosen + r0, (size_t)nr * sizeof(int32_t),
+                            cudaMemcpyHostToDevice, c->copy_stream));
+    PR_CUDA(cudaEventRecord(c->ev_copied[j], c->copy_stream));
+    PR_CUDA(cudaStreamWaitEvent(s, c->ev_copied[j], 0));
+    st = pr_route(c, c->stage[j], dt, r0, nr, vocab, row_stride, c->stage_chosen[j],
+                  c->h_offsets_dev, n_req, c->h_w_dev, b, tau, d_score, c->h_ship_dev,
+                  c->h_flags_dev, agg ? d_agg : nullptr, stream);
+    if (st != PR_OK) return st;
+    PR_CUDA(cudaEventRecord(c->ev_free[j], s));
+  }
+  PR_CUDA(cudaMemcpyAsync(score, d_score, (size_t)n_req * sizeof(float), cudaMemcpyDeviceToHost, s));
+  PR_CUDA(cudaMemcpyAsync(ship, c->h_ship_dev, (size_t)n_req, cudaMemcpyDeviceToHost, s));
+  PR_CUDA(cudaMemcpyAsync(req_flags, c->h_flags_dev, (size_t)n_req * sizeof(uint32_t),
+                          cudaMemcpyDeviceToHost, s));
+  if (agg)
+    PR_CUDA(cudaMemcpyAsync(agg, d_agg, (size_t)n_req * prk::NAGG * sizeof(float),
+                            cudaMemcpyDeviceToHost, s));
+  PR_CUDA(cudaStreamSynchronize(s));
+  return PR_OK;
+}
+
+}  // extern "C"

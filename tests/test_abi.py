@@ -1,0 +1,82 @@
+"""The C-ABI library builds for sm_103a, loads, and exports every symbol the
+header declares; host-side argument checks answer without touching a GPU."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2608_28726_gb300 import build as prbuild
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "pro_router.h")
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(pr_[a-z_0-9]+)\s*\(", text)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    path = prbuild.build()
+    return ctypes.CDLL(path)
+
+
+def test_header_declares_the_three_verifier_calls():
+    names = declared_functions()
+    for n in ("pr_token_features", "pr_aggregate_score", "pr_route"):
+        assert n in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+
+
+def test_binding_covers_the_header(lib):
+    from paper_2608_28726_gb300 import binding
+    assert sorted(binding.EXPORTS) == declared_functions()
+
+
+def test_library_targets_sm_103a_only():
+    assert prbuild.ARCH == ["-gencode", "arch=compute_103a,code=sm_103a"]
+
+
+def test_status_strings(lib):
+    lib.pr_status_string.restype = ctypes.c_char_p
+    lib.pr_status_string.argtypes = [ctypes.c_int]
+    assert lib.pr_status_string(0) == b"ok"
+    assert lib.pr_status_string(-1) == b"invalid argument"
+    assert lib.pr_status_string(-3) == b"CUDA error"
+    assert lib.pr_status_string(12345) == b"unknown status"
+
+
+def test_null_context_is_rejected(lib):
+    P = ctypes.c_void_p
+    lib.pr_route.argtypes = [P, P, ctypes.c_int, ctypes.c_int64, ctypes.c_int64, ctypes.c_int64,
+                             ctypes.c_int64, P, P, ctypes.c_int32, P, ctypes.c_float,
+                             ctypes.c_float, P, P, P, P, P]
+    assert lib.pr_route(None, None, 1, 0, 0, 1, 1, None, None, 1, None, 0.0, 0.5, None, None, None,
+                        None, None) == -1
+    lib.pr_ctx_create.argtypes = [ctypes.POINTER(P), ctypes.c_int, ctypes.c_int64, ctypes.c_int32]
+    assert lib.pr_ctx_create(None, 0, 1, 1) == -1
+    h = P()
+    assert lib.pr_ctx_create(ctypes.byref(h), 0, -5, 1) == -1
+    lib.pr_ctx_set_option.argtypes = [P, ctypes.c_int32, ctypes.c_int32]
+    assert lib.pr_ctx_set_option(None, 0, 20) == -1
+    lib.pr_launch_count.restype = ctypes.c_uint64
+    assert lib.pr_launch_count() == 0
+
+
+def test_no_gpu_means_no_context(lib):
+    """Without a device the context cannot be made, and says so (no fallback)."""
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    P = ctypes.c_void_p
+    lib.pr_ctx_create.argtypes = [ctypes.POINTER(P), ctypes.c_int, ctypes.c_int64, ctypes.c_int32]
+    h = P()
+    assert lib.pr_ctx_create(ctypes.byref(h), 0, 16, 4) == -1
+    assert not h.value

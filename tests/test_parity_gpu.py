@@ -1,0 +1,438 @@
+"""GPU parity of the three verifier calls against the float64 oracle, on
+small inputs that still span several tiles and a ragged tail, plus the edge
+cases: odd and tiny vocabularies, unaligned rows, every K, masked / tied /
+non-finite rows, bad ids and offsets, row splits, chunking, decode steps,
+checkpoints, the host-memory path and buffer guards.  Everything goes
+through the C ABI (ctypes binding)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from _util import as_oracle, assert_close, assert_ship, random_rows
+
+pytestmark = pytest.mark.gpu
+
+B = None  # the binding, imported once a GPU is known to be present
+
+
+@pytest.fixture(scope="module")
+def ctx():
+    global B
+    assert torch.cuda.is_available(), "the GPU tests need a CUDA device"
+    from paper_2608_28726_gb300 import build
+    build.build()
+    from paper_2608_28726_gb300 import binding
+    B = binding
+    h = B.pr_ctx_create(0, max_rows=1 << 16, max_requests=1024)
+    yield h
+    B.pr_ctx_destroy(h)
+
+
+def _set(ctx, split=0, renorm=0, topk=20):
+    B.pr_ctx_set_option(ctx, B.PR_OPT_SPLIT, split)
+    B.pr_ctx_set_option(ctx, B.PR_OPT_TOPK_RENORM, renorm)
+    B.pr_ctx_set_option(ctx, B.PR_OPT_TOPK, topk)
+
+
+def _oracle_rows(x, chosen, K=20, renorm=False, vocab=None):
+    xs = as_oracle(x)
+    ch = chosen.cpu().numpy()
+    feats, idxs, flags = [], [], []
+    for r in range(xs.shape[0]):
+        row = xs[r] if vocab is None else xs[r, :vocab]
+        f, i, fl = oracle.row_features(row, int(ch[r]), K=K, renorm=renorm)
+        feats.append(f)
+        idxs.append(i)
+        flags.append(fl)
+    return np.array(feats), np.array(idxs), np.array(flags)
+
+
+def _check_features(feat, top2, rflags, of, oi, ofl, what):
+    feat = feat.cpu().numpy()
+    top2 = top2.cpu().numpy()
+    rflags = rflags.cpu().numpy().astype(np.uint32)
+    assert np.array_equal(rflags, ofl), "%s flags %s vs %s" % (what, rflags, ofl)
+    assert np.array_equal(top2, oi), "%s top2 differ at rows %s" % (
+        what, np.argwhere((top2 != oi).any(1)).ravel()[:8])
+    for s in (oracle.LOGP, oracle.MAXP, oracle.MARGIN, oracle.ENT, oracle.TOPK, oracle.LSE,
+              oracle.X1):
+        assert_close(feat[:, s], of[:, s], "%s feature %d" % (what, s))
+
+
+# ---- per-token features ----------------------------------------------------------------
+
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+@pytest.mark.parametrize("V", [1, 2, 7, 8, 9, 31, 160, 1000, 4097, 32000, 70001])
+def test_features_vocab_sizes(ctx, dtype, V):
+    _set(ctx)
+    x, ch = random_rows(24, V, dtype, seed=V)
+    feat, top2, rf = B.pr_token_features(ctx, x, ch, topk=20)
+    of, oi, ofl = _oracle_rows(x, ch)
+    _check_features(feat, top2, rf, of, oi, ofl, "V=%d" % V)
+
+
+@pytest.mark.parametrize("K", [1, 2, 3, 19, 20, 21, 32])
+@pytest.mark.parametrize("renorm", [0, 1])
+def test_features_topk(ctx, K, renorm):
+    _set(ctx, renorm=renorm)
+    x, ch = random_rows(16, 3001, torch.bfloat16, seed=100 + K)
+    feat, top2, rf = B.pr_token_features(ctx, x, ch, topk=K)
+    of, oi, ofl = _oracle_rows(x, ch, K=K, renorm=bool(renorm))
+    _check_features(feat, top2, rf, of, oi, ofl, "K=%d renorm=%d" % (K, renorm))
+    _set(ctx)
+
+
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+@pytest.mark.parametrize("shift", [1, 3])
+def test_features_unaligned_rows(ctx, dtype, shift):
+    """Row starts off the 16-byte grid take the guarded element path."""
+    V = 2053
+    base, ch = random_rows(12, V + shift + 5, dtype, seed=7 + shift)
+    x = base[:, shift:shift + V]  # row stride V + shift + 5, start offset `shift` elements
+    assert x.stride(0) == V + shift + 5
+    feat, top2, rf = B.pr_token_features(ctx, x, ch % V, topk=20)
+    of, oi, ofl = _oracle_rows(x.contiguous(), ch % V)
+    _check_features(feat, top2, rf, of, oi, ofl, "unaligned")
+
+
+def test_features_vocab_narrower_than_stride(ctx):
+    x, ch = random_rows(10, 5000, torch.float32, seed=3)
+    V = 4321
+    feat, top2, rf = B.pr_token_features(ctx, x, ch % V, topk=20, vocab=V)
+    of, oi, ofl = _oracle_rows(x, ch % V, vocab=V)
+    _check_features(feat, top2, rf, of, oi, ofl, "vocab<stride")
+
+
+def _special_rows(V, dtype):
+    rows, chosen = [], []
+    neg = float("-inf")
+    r = torch.full((V,), 1.25)                      # uniform
+    rows.append(r); chosen.append(3)
+    r = torch.full((V,), neg); r[V // 3] = 2.0      # one-hot by masking
+    rows.append(r); chosen.append(V // 3)
+    r = torch.full((V,), neg); r[5] = r[V - 2] = -1.0  # two-way tie, rest masked
+    rows.append(r); chosen.append(V - 2)
+    r = torch.randn(V); r[torch.rand(V) < 0.5] = neg   # half masked
+    rows.append(r); chosen.append(int(torch.nonzero(r > neg)[0]))
+    r = torch.randn(V); r[17] = float("nan")        # NaN
+    rows.append(r); chosen.append(0)
+    r = torch.randn(V); r[V - 1] = float("inf")     # +inf
+    rows.append(r); chosen.append(0)
+    rows.append(torch.full((V,), neg)); chosen.append(0)  # nothing finite
+    r = torch.randn(V); rows.append(r); chosen.append(-1)  # bad chosen
+    r = torch.randn(V); rows.append(r); chosen.append(V)   # bad chosen
+    r = torch.randn(V); m = r.max(); r[[2, 9, 200, V - 1]] = m  # 4-way tie at the top
+    rows.append(r); chosen.append(9)
+    r = torch.zeros(V); r[0] = -200.0               # one low outlier
+    rows.append(r); chosen.append(0)
+    r = torch.randn(V) * 30; rows.append(r); chosen.append(1)  # very peaked
+    r = torch.randn(V) + 1000.0; rows.append(r); chosen.append(4)  # large offset
+    r = torch.randn(V); r[3] = neg; rows.append(r); chosen.append(3)  # chosen is masked
+    x = torch.stack(rows).to(dtype)
+    return x.cuda(), torch.tensor(chosen, dtype=torch.int32).cuda()
+
+
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+@pytest.mark.parametrize("V", [257, 4096])
+def test_features_special_rows(ctx, dtype, V):
+    _set(ctx)
+    x, ch = _special_rows(V, dtype)
+    feat, top2, rf = B.pr_token_features(ctx, x, ch, topk=20)
+    of, oi, ofl = _oracle_rows(x, ch)
+    _check_features(feat, top2, rf, of, oi, ofl, "special V=%d" % V)
+
+
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+def test_split_factor_invariance(ctx, dtype):
+    """1, 2, 4 or 8 CTAs per row: same indices and flags, features to tolerance."""
+    x, ch = random_rows(20, 151936 if dtype == torch.bfloat16 else 65536, dtype, seed=11)
+    of, oi, ofl = _oracle_rows(x, ch)
+    for split in (1, 2, 4, 8):
+        _set(ctx, split=split)
+        feat, top2, rf = B.pr_token_features(ctx, x, ch, topk=20)
+        _check_features(feat, top2, rf, of, oi, ofl, "split=%d" % split)
+    _set(ctx)
+
+
+def test_features_rho(ctx):
+    lengths = [5, 1, 0, 9, 3]
+    off = torch.tensor(np.concatenate([[0], np.cumsum(lengths)]), dtype=torch.int64).cuda()
+    n = int(sum(lengths))
+    x, ch = random_rows(n, 999, torch.float32, seed=5)
+    feat, _, _ = B.pr_token_features(ctx, x, ch, topk=20, offsets=off)
+    rho = feat[:, 5].cpu().numpy()
+    expect = np.concatenate([np.arange(1, T + 1) / T for T in lengths if T > 0])
+    assert_close(rho, expect, "rho", rtol=1e-7, atol=0)
+
+
+# ---- pooling, scoring, the ship rule ---------------------------------------------------------
+
+def _batch(lengths, V, dtype, seed):
+    off = np.concatenate([[0], np.cumsum(lengths)]).astype(np.int64)
+    x, ch = random_rows(int(off[-1]), V, dtype, seed=seed)
+    g = np.random.default_rng(seed)
+    w = (g.standard_normal(11) * 0.1).astype(np.float32)
+    b = float(np.float32(g.standard_normal() * 0.1))
+    return x, ch, off, w, b
+
+
+def _check_requests(score, ship, rflags, agg, o, tau, what):
+    rflags = rflags.cpu().numpy().astype(np.uint32)
+    assert np.array_equal(rflags, o["req_flags"]), what
+    assert_close(agg.cpu().numpy(), o["agg"], what + " agg")
+    assert_close(score.cpu().numpy(), o["score"], what + " score")
+    assert_ship(ship.cpu().numpy(), o["ship"], o["score"], tau)
+
+
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+def test_route_matches_oracle(ctx, dtype):
+    _set(ctx)
+    lengths = [3, 0, 40, 1, 77, 0, 12, 130, 2]
+    x, ch, off, w, b = _batch(lengths, 3001, dtype, seed=21)
+    o = oracle.route(as_oracle(x), ch.cpu().numpy(), off, w.astype(np.float64), b, 0.5)
+    dw = torch.from_numpy(w).cuda()
+    doff = torch.from_numpy(off).cuda()
+    score, ship, rf, agg = B.pr_route(ctx, x, ch, doff, dw, b, 0.5)
+    _check_requests(score, ship, rf, agg, o, 0.5, "route")
+    # and the same through the two separate calls
+    feat, top2, rfl = B.pr_token_features(ctx, x, ch, topk=20, offsets=doff)
+    agg2, score2, ship2, rf2 = B.pr_aggregate_score(ctx, feat, doff, dw, b, 0.5, row_flags=rfl)
+    _check_requests(score2, ship2, rf2, agg2, o, 0.5, "features+aggregate")
+    assert torch.equal(agg.nan_to_num(7.0), agg2.nan_to_num(7.0))
+    assert torch.equal(ship, ship2)
+
+
+def test_route_threshold_and_flags(ctx):
+    """Zero weights give score 1/2, which ships at tau = 1/2 (ship iff p >= tau)."""
+    lengths = [4, 6]
+    x, ch, off, _, _ = _batch(lengths, 500, torch.float32, seed=2)
+    ch[2] = 10_000  # a bad token id escalates request 0
+    w = torch.zeros(11, device="cuda")
+    doff = torch.from_numpy(off).cuda()
+    score, ship, rf, agg = B.pr_route(ctx, x, ch, doff, w, 0.0, 0.5)
+    assert ship.tolist() == [0, 1]
+    assert rf.tolist() == [B.PR_FLAG_BAD_CHOSEN, 0]
+    assert torch.isnan(score[0]) and score[1].item() == 0.5
+    score, ship, rf, agg = B.pr_route(ctx, x, ch, doff, w, 0.0, 0.5000001)
+    assert ship.tolist() == [0, 0]
+
+
+def test_route_bad_offsets(ctx):
+    x, ch, off, w, b = _batch([3, 3], 300, torch.float32, seed=3)
+    B.pr_ctx_flags(ctx, clear=True)
+    doff = torch.tensor([0, 4, 2], dtype=torch.int64, device="cuda")
+    score, ship, rf, agg = B.pr_route(ctx, x[:6], ch[:6], doff, torch.from_numpy(w).cuda(), b, 0.5)
+    torch.cuda.synchronize()
+    assert rf[1].item() == B.PR_FLAG_BAD_OFFSETS and ship[1].item() == 0
+    assert B.pr_ctx_flags(ctx, clear=True) & B.PR_FLAG_BAD_OFFSETS
+    B.pr_ctx_reset(ctx)
+
+
+@pytest.mark.parametrize("chunk", [1, 7, 64, 1000])
+def test_chunked_route_equals_whole(ctx, chunk):
+    """Requests straddling chunks are finished by whichever chunk ends them;
+    chunk order does not matter and the results are bit-identical."""
+    lengths = [5, 0, 33, 1, 64, 17, 0, 120, 9]
+    x, ch, off, w, b = _batch(lengths, 2048, torch.bfloat16, seed=31)
+    _set(ctx, split=2)  # the automatic split depends on the rows per call
+    dw, doff = torch.from_numpy(w).cuda(), torch.from_numpy(off).cuda()
+    ref = B.pr_route(ctx, x, ch, doff, dw, b, 0.5)
+    n = x.size(0)
+    starts = list(range(0, n, chunk))
+    np.random.default_rng(chunk).shuffle(starts)
+    nr = len(lengths)
+    score = torch.full((nr,), -5.0, device="cuda")
+    ship = torch.full((nr,), 9, dtype=torch.uint8, device="cuda")
+    rf = torch.full((nr,), -1, dtype=torch.int32, device="cuda")
+    agg = torch.zeros(nr, 11, device="cuda")
+    for s in starts:
+        e = min(n, s + chunk)
+        B.pr_route(ctx, x[s:e], ch[s:e], doff, dw, b, 0.5, row_base=s, score=score, ship=ship,
+                   req_flags=rf, agg=agg)
+    assert torch.equal(score.nan_to_num(3.0), ref[0].nan_to_num(3.0))
+    assert torch.equal(ship, ref[1]) and torch.equal(rf, ref[2])
+    assert torch.equal(agg.nan_to_num(3.0), ref[3].nan_to_num(3.0))
+    _set(ctx)
+
+
+def test_route_is_one_launch(ctx):
+    x, ch, off, w, b = _batch([10, 20], 1000, torch.bfloat16, seed=4)
+    dw, doff = torch.from_numpy(w).cuda(), torch.from_numpy(off).cuda()
+    n0 = B.launch_count()
+    B.pr_route(ctx, x, ch, doff, dw, b, 0.5)
+    assert B.launch_count() - n0 == 1
+
+
+def test_route_host_matches_route(ctx):
+    lengths = [50, 3, 0, 200, 11]
+    x, ch, off, w, b = _batch(lengths, 4096, torch.bfloat16, seed=41)
+    _set(ctx, split=1)  # the automatic split depends on the rows per call
+    dw, doff = torch.from_numpy(w).cuda(), torch.from_numpy(off).cuda()
+    ref = B.pr_route(ctx, x, ch, doff, dw, b, 0.5)
+    hx = x.cpu().pin_memory()
+    hc = ch.cpu().pin_memory()
+    hoff = torch.from_numpy(off)
+    hw = torch.from_numpy(w)
+    agg = torch.empty(len(lengths), 11)
+    score, ship, rf, _ = B.pr_route_host(ctx, hx, hc, hoff, hw, b, 0.5, chunk_rows=37, agg=agg)
+    assert torch.equal(score.nan_to_num(3.0), ref[0].cpu().nan_to_num(3.0))
+    assert torch.equal(ship, ref[1].cpu()) and torch.equal(rf, ref[2].cpu())
+    assert torch.equal(agg.nan_to_num(3.0), ref[3].cpu().nan_to_num(3.0))
+    _set(ctx)
+
+
+def test_output_guards(ctx):
+    """Nothing is written outside the output slices."""
+    lengths = [7, 0, 19]
+    x, ch, off, w, b = _batch(lengths, 1500, torch.float32, seed=8)
+    dw, doff = torch.from_numpy(w).cuda(), torch.from_numpy(off).cuda()
+    n, nr, G = x.size(0), len(lengths), 64
+    sent = 123456.0
+    feat = torch.full((n + 2 * G // 8, 8), sent, device="cuda")
+    top2 = torch.full((n + 2 * G, 2), 77, dtype=torch.int32, device="cuda")
+    rfl = torch.full((n + 2 * G,), 55, dtype=torch.int32, device="cuda")
+    g8 = G // 8
+    B.pr_token_features(ctx, x, ch, topk=20, feat=feat[g8:g8 + n], top2=top2[G:G + n],
+                        row_flags=rfl[G:G + n])
+    score = torch.full((nr + 2 * G,), sent, device="cuda")
+    ship = torch.full((nr + 2 * G,), 200, dtype=torch.uint8, device="cuda")
+    rf = torch.full((nr + 2 * G,), 99, dtype=torch.int32, device="cuda")
+    agg = torch.full((nr + 2 * G, 11), sent, device="cuda")
+    B.pr_route(ctx, x, ch, doff, dw, b, 0.5, score=score[G:G + nr], ship=ship[G:G + nr],
+               req_flags=rf[G:G + nr], agg=agg[G:G + nr])
+    torch.cuda.synchronize()
+    for t, v, lo, hi in ((feat, sent, g8, g8 + n), (top2, 77, G, G + n), (rfl, 55, G, G + n),
+                         (score, sent, G, G + nr), (ship, 200, G, G + nr), (rf, 99, G, G + nr),
+                         (agg, sent, G, G + nr)):
+        assert (t[:lo] == v).all() and (t[hi:] == v).all()
+
+
+def test_invalid_arguments(ctx):
+    x, ch, off, w, b = _batch([3], 100, torch.float32, seed=1)
+    dw, doff = torch.from_numpy(w).cuda(), torch.from_numpy(off).cuda()
+    with pytest.raises(B.PRError) as e:
+        B.pr_token_features(ctx, x, ch, topk=0)
+    assert e.value.status == B.PR_ERR_INVALID_ARG
+    with pytest.raises(B.PRError):
+        B.pr_token_features(ctx, x, ch, topk=33)
+    with pytest.raises(B.PRError):
+        B.pr_route(ctx, x, ch, doff, dw, b, 0.5, row_base=(1 << 16))
+    with pytest.raises(TypeError):
+        B.pr_token_features(ctx, x.half(), ch)  # fp16 is not a verifier dtype
+    with pytest.raises(B.PRError):
+        B.pr_ctx_set_option(ctx, B.PR_OPT_SPLIT, 3)
+
+
+# ---- incremental decode steps ------------------------------------------------------------------
+
+def _decode_run(ctx, trace_rows, n_slots, steps, eos, w, b, stop=None, state=None):
+    """Run steps [0, stop) (or all) and return per-slot outputs at every EOS."""
+    V = trace_rows[0][0].size(1)
+    score = torch.full((n_slots,), -1.0, device="cuda")
+    ship = torch.zeros(n_slots, dtype=torch.uint8, device="cuda")
+    fl = torch.zeros(n_slots, dtype=torch.int32, device="cuda")
+    agg = torch.zeros(n_slots, 11, device="cuda")
+    slot = torch.arange(n_slots, dtype=torch.int32, device="cuda")
+    dw = torch.from_numpy(w).cuda()
+    ends = {}
+    for s in range(steps if stop is None else stop):
+        x, ch = trace_rows[s]
+        e = torch.from_numpy(eos[s]).cuda()
+        B.pr_decode_step(ctx, x, slot, ch, e, dw, b, 0.5, score, ship, fl, agg_out=agg)
+        for sl in np.nonzero(eos[s])[0]:
+            ends[(int(sl), s)] = (score[sl].item(), ship[sl].item(), fl[sl].item(),
+                                  agg[sl].cpu().numpy().copy())
+    return ends
+
+
+def _small_trace(n_slots=6, steps=80, V=1500, seed=9):
+    g = np.random.default_rng(seed)
+    eos = np.zeros((steps, n_slots), np.uint8)
+    reqs = []
+    for s in range(n_slots):
+        t = 0
+        while t < steps:
+            L = int(g.integers(1, 30))
+            reqs.append((s, t, L))
+            if t + L - 1 < steps:
+                eos[t + L - 1, s] = 1
+            t += L
+    rows = [random_rows(n_slots, V, torch.bfloat16, seed=1000 + k) for k in range(steps)]
+    w = (g.standard_normal(11) * 0.1).astype(np.float32)
+    b = float(np.float32(g.standard_normal() * 0.1))
+    return rows, eos, reqs, w, b
+
+
+def test_decode_matches_oracle(ctx):
+    _set(ctx)
+    n_slots, steps = 6, 80
+    rows, eos, reqs, w, b = _small_trace(n_slots, steps)
+    B.pr_ctx_reset(ctx)
+    ends = _decode_run(ctx, rows, n_slots, steps, eos, w, b)
+    xs = [as_oracle(r[0]) for r in rows]
+    cs = [r[1].cpu().numpy() for r in rows]
+    checked = 0
+    for (sl, t0, L) in reqs:
+        if t0 + L > steps:
+            continue
+        X = np.stack([xs[t][sl] for t in range(t0, t0 + L)])
+        C = np.array([cs[t][sl] for t in range(t0, t0 + L)], np.int32)
+        o = oracle.route(X, C, np.array([0, L]), w.astype(np.float64), b, 0.5)
+        sc, sh, fl, ag = ends[(sl, t0 + L - 1)]
+        assert fl == o["req_flags"][0]
+        assert_close(ag, o["agg"][0], "decode agg")
+        assert_close(sc, o["score"][0], "decode score")
+        assert_ship([sh], o["ship"], o["score"], 0.5)
+        checked += 1
+    assert checked >= 15
+    B.pr_ctx_reset(ctx)
+
+
+def test_decode_checkpoint_resume(ctx):
+    n_slots, steps = 6, 80
+    rows, eos, reqs, w, b = _small_trace(n_slots, steps, seed=12)
+    B.pr_ctx_reset(ctx)
+    full = _decode_run(ctx, rows, n_slots, steps, eos, w, b)
+    B.pr_ctx_reset(ctx)
+    first = _decode_run(ctx, rows, n_slots, steps, eos, w, b, stop=37)
+    state = B.pr_state_export(ctx)
+    other = B.pr_ctx_create(0, max_rows=16, max_requests=1024)
+    try:
+        B.pr_state_import(other, state)
+        score = torch.full((n_slots,), -1.0, device="cuda")
+        ship = torch.zeros(n_slots, dtype=torch.uint8, device="cuda")
+        fl = torch.zeros(n_slots, dtype=torch.int32, device="cuda")
+        agg = torch.zeros(n_slots, 11, device="cuda")
+        slot = torch.arange(n_slots, dtype=torch.int32, device="cuda")
+        dw = torch.from_numpy(w).cuda()
+        for s in range(37, steps):
+            x, ch = rows[s]
+            B.pr_decode_step(other, x, slot, ch, torch.from_numpy(eos[s]).cuda(), dw, b, 0.5, score,
+                             ship, fl, agg_out=agg)
+            for sl in np.nonzero(eos[s])[0]:
+                ref = full[(int(sl), s)]
+                assert score[sl].item() == ref[0] or (np.isnan(ref[0]) and np.isnan(score[sl].item()))
+                assert ship[sl].item() == ref[1] and fl[sl].item() == ref[2]
+                assert np.array_equal(agg[sl].cpu().numpy(), ref[3])
+        for k, v in first.items():
+            assert v[1] == full[k][1]
+    finally:
+        B.pr_ctx_destroy(other)
+    with pytest.raises(B.PRError):
+        B.pr_state_import(ctx, state[:-4])
+    B.pr_ctx_reset(ctx)
+
+
+def test_decode_bad_slot_flagged(ctx):
+    B.pr_ctx_reset(ctx)
+    x, ch = random_rows(2, 300, torch.float32, seed=1)
+    slot = torch.tensor([0, 5000], dtype=torch.int32, device="cuda")
+    eos = torch.ones(2, dtype=torch.uint8, device="cuda")
+    out = torch.zeros(1024, device="cuda")
+    ship = torch.zeros(1024, dtype=torch.uint8, device="cuda")
+    fl = torch.zeros(1024, dtype=torch.int32, device="cuda")
+    B.pr_decode_step(ctx, x, slot, ch, eos, torch.zeros(11, device="cuda"), 0.0, 0.5, out, ship, fl)
+    assert B.pr_ctx_flags(ctx, clear=True) & B.PR_FLAG_BAD_SLOT
+    assert ship[0].item() == 1 and out[0].item() == 0.5
+    B.pr_ctx_reset(ctx)
