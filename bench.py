@@ -225,7 +225,7 @@ def run_gb300(args):
     prbuild.build()
     from paper_2608_28726_gb300 import binding as B
 
-    wl = W.make(WORKLOAD)
+    wl = W.make(WORKLOAD, n_req=args.requests or None)
     x, ch = W.rows(wl, 0, wl.n_rows, device=dev)
     off = torch.from_numpy(wl.offsets).to(dev)
     w = torch.from_numpy(wl.w).to(dev)
@@ -264,6 +264,13 @@ def run_gb300(args):
     total_ms = ev[0].elapsed_time(ev[K])
     total_ms = reduce_max(total_ms, world, dev)
     clocks = sampler.summary(t_wall0, t_wall1)
+    if args.skip_host:
+        sampler.stop()
+        if rank == 0:
+            print(json.dumps({"profiling_case": True, "rows": wl.n_rows, "steps": K,
+                              "ms_per_step": total_ms / K, "gpu_launches": launches}))
+        B.pr_ctx_destroy(ctx)
+        return 0
 
     # end to end from pinned host memory through the public C ABI
     hx = x.cpu().pin_memory()
@@ -360,6 +367,10 @@ def main():
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--requests", type=int, default=0,
+                    help="profiling only: the first N requests of the workload")
+    ap.add_argument("--skip-host", action="store_true",
+                    help="profiling only: skip the host-memory and oracle legs")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)

@@ -11,17 +11,21 @@
 //     S = sum 2^(t_v - m) and U = sum 2^(t_v - m) (t_v - m).  Then
 //     LSE = ln2 (m + log2 S) and H = ln2 (log2 S - U / S).  Partial states
 //     merge as S = sum_i S_i 2^(m_i - M), U = sum_i 2^(m_i - M)(U_i + (m_i - M) S_i).
-//     The per-element work is one packed FMA, one ex2, one packed add and one
-//     packed FMA per two elements (f32x2 instructions of sm_100+).
-//   * exact top-K (and top-2 with the lowest-index tie rule) without touching
-//     elements individually: the row is cut into 16-byte groups (8 bf16 or 4
-//     fp32 elements).  Ordering groups by (group max, lower group index first),
-//     the K largest elements under (value, lower index first) all lie in the K
-//     largest groups.  So the stream only tracks group maxima: a warp keeps the
-//     32 best group keys in a register-resident sorted list and pushes groups
-//     whose maximum reaches its current K-th key into a shared-memory buffer,
-//     merged 32 at a time with warp bitonic networks.  After the stream the K
-//     winning groups (K * 16 bytes) are re-read and their elements sorted.
+//     The row is read in tiles of 4 x 16 bytes per thread; the tile maximum is
+//     a packed max tree, the per-element work one packed FMA, one ex2, one
+//     packed add and one packed FMA per two elements (f32x2 of sm_100+).
+//   * exact top-K (and the first two tokens, lower index first on ties) at
+//     almost no streaming cost: each thread only stores the maximum of each of
+//     its tiles in shared memory.  After the stream, theta1 = the K-th largest
+//     per-thread maximum is a lower bound of the K-th largest element (K
+//     distinct elements reach it); the stored tile maxima >= theta1 are the
+//     candidate "super-groups"; theta = the K-th largest candidate value is a
+//     tighter bound, and every element >= theta lies in a candidate >= theta
+//     (an element below theta has K strictly larger elements, the maxima of K
+//     candidates).  Those few super-groups are re-read and their elements
+//     >= theta sorted by (value, lower index first) with warp bitonic networks.
+//     Ties never lose an element; rows whose ties swamp the buffers fall back
+//     to an exact scan of the whole row.
 //   * rows with -inf (masked tokens), NaN or +inf make the fast accumulators
 //     non-finite; such rows are re-streamed with per-element guards, which
 //     classify them exactly.
@@ -36,8 +40,10 @@ namespace prk {
 constexpr int NT = 256;            // threads per CTA
 constexpr int NWARP = NT / 32;     // warps per CTA
 constexpr int UNR = 4;             // 16-byte groups per thread per tile
-constexpr int LIST = 32;           // group keys kept per warp
-constexpr int BUF = 32 + 32 * UNR; // candidate buffer per warp
+constexpr int TILE = NT * UNR;     // groups per CTA tile
+constexpr int MAX_SLOTS = 24;      // stored tile maxima per thread (tiles are merged beyond)
+constexpr int CCAP = 256;          // candidate super-groups
+constexpr int ECAP = 512;          // candidate elements
 constexpr int MAXC = 8;            // largest cluster (CTAs per row)
 constexpr int NFEAT = 8;
 constexpr int NAGG = 11;
@@ -46,6 +52,7 @@ constexpr float L2E = 1.4426950408889634f;
 constexpr float LN2 = 0.6931471805599453f;
 constexpr float M2_INIT = -1e30f;  // finite "no maximum yet" so that 2^(m - m') is 0, never NaN
 constexpr unsigned FULL = 0xffffffffu;
+constexpr uint32_t TAIL_ID = 0xffffffffu;  // candidate id of the partial last group
 
 constexpr uint32_t FLAG_NONFINITE = 1u;
 constexpr uint32_t FLAG_BAD_CHOSEN = 2u;
@@ -102,6 +109,12 @@ __device__ __forceinline__ uint4 ld_stream(const void* p) {
   return r;
 }
 
+__device__ __forceinline__ uint32_t hmax2(uint32_t a, uint32_t b) {
+  uint32_t d;
+  asm("max.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+  return d;
+}
+
 // order-preserving map float -> uint32 (larger float -> larger integer)
 __device__ __forceinline__ uint32_t ord(float f) {
   uint32_t u = __float_as_uint(f);
@@ -131,14 +144,17 @@ __device__ __forceinline__ uint64_t shfl64(uint64_t v, int src) {
   return ((uint64_t)hi << 32) | lo;
 }
 
-// bitonic sort of one 64-bit key per lane, descending (lane 0 = largest)
-__device__ __forceinline__ uint64_t warp_sort_desc(uint64_t k, int lane) {
+// bitonic sort of one key per lane, descending (lane 0 = largest)
+template <typename K>
+__device__ __forceinline__ K warp_sort_desc(K k, int lane) {
 #pragma unroll
   for (int size = 2; size <= 32; size <<= 1) {
     const bool desc = (lane & size) == 0;
 #pragma unroll
     for (int stride = size >> 1; stride > 0; stride >>= 1) {
-      uint64_t o = shfl_xor64(k, stride);
+      K o;
+      if constexpr (sizeof(K) == 8) o = shfl_xor64(k, stride);
+      else o = __shfl_xor_sync(FULL, k, stride);
       const bool keep_max = (((lane & stride) == 0) == desc);
       k = keep_max ? (k > o ? k : o) : (k < o ? k : o);
     }
@@ -147,29 +163,20 @@ __device__ __forceinline__ uint64_t warp_sort_desc(uint64_t k, int lane) {
 }
 
 // a, b sorted descending across lanes -> the 32 largest of a U b, descending
-__device__ __forceinline__ uint64_t warp_merge_desc(uint64_t a, uint64_t b, int lane) {
-  uint64_t br = shfl64(b, 31 - lane);
-  uint64_t t = a > br ? a : br;
+template <typename K>
+__device__ __forceinline__ K warp_merge_desc(K a, K b, int lane) {
+  K br;
+  if constexpr (sizeof(K) == 8) br = shfl64(b, 31 - lane);
+  else br = __shfl_sync(FULL, b, 31 - lane);
+  K t = a > br ? a : br;
 #pragma unroll
   for (int stride = 16; stride > 0; stride >>= 1) {
-    uint64_t o = shfl_xor64(t, stride);
+    K o;
+    if constexpr (sizeof(K) == 8) o = shfl_xor64(t, stride);
+    else o = __shfl_xor_sync(FULL, t, stride);
     t = ((lane & stride) == 0) ? (t > o ? t : o) : (t < o ? t : o);
   }
   return t;
-}
-
-__device__ __forceinline__ uint32_t warp_sort_desc32(uint32_t k, int lane) {
-#pragma unroll
-  for (int size = 2; size <= 32; size <<= 1) {
-    const bool desc = (lane & size) == 0;
-#pragma unroll
-    for (int stride = size >> 1; stride > 0; stride >>= 1) {
-      uint32_t o = __shfl_xor_sync(FULL, k, stride);
-      const bool keep_max = (((lane & stride) == 0) == desc);
-      k = keep_max ? max(k, o) : min(k, o);
-    }
-  }
-  return k;
 }
 
 // (m, S, U) merge of two partial log-sum-exp / entropy states (base 2)
@@ -224,21 +231,35 @@ struct Traits;
 
 template <>
 struct Traits<__nv_bfloat16> {
-  static constexpr int VEC = 8;  // elements per 16-byte group
+  static constexpr int VEC = 8;                       // elements per 16-byte group
+  static constexpr uint32_t NEG_WORD = 0xff80ff80u;   // two bf16 -inf
   static __device__ __forceinline__ float elem(const void* row, int64_t v) {
     const uint16_t h = reinterpret_cast<const uint16_t*>(row)[v];
     return __uint_as_float((uint32_t)h << 16);
   }
-  // group maximum (NaN ignored unless every element is NaN)
-  static __device__ __forceinline__ float gmax(const uint4& w) {
-    __nv_bfloat162 a = __hmax2(*reinterpret_cast<const __nv_bfloat162*>(&w.x),
-                               *reinterpret_cast<const __nv_bfloat162*>(&w.y));
-    __nv_bfloat162 b = __hmax2(*reinterpret_cast<const __nv_bfloat162*>(&w.z),
-                               *reinterpret_cast<const __nv_bfloat162*>(&w.w));
-    __nv_bfloat162 c = __hmax2(a, b);
-    const uint32_t u = *reinterpret_cast<const uint32_t*>(&c);
+  // a full group by element loads (rows that are not 16-byte aligned)
+  static __device__ __forceinline__ uint4 load_elems(const void* row, int64_t g) {
+    const uint16_t* h = reinterpret_cast<const uint16_t*>(row) + g * VEC;
+    uint4 r;
+    r.x = (uint32_t)h[0] | ((uint32_t)h[1] << 16);
+    r.y = (uint32_t)h[2] | ((uint32_t)h[3] << 16);
+    r.z = (uint32_t)h[4] | ((uint32_t)h[5] << 16);
+    r.w = (uint32_t)h[6] | ((uint32_t)h[7] << 16);
+    return r;
+  }
+  static __device__ __forceinline__ uint32_t wmax(const uint4& w) {
+    return hmax2(hmax2(w.x, w.y), hmax2(w.z, w.w));
+  }
+  static __device__ __forceinline__ float wfinal(uint32_t u) {
     return fmaxf(__uint_as_float(u << 16), __uint_as_float(u & 0xffff0000u));
   }
+  // maximum of the UNR groups of a tile (NaN ignored unless all are NaN)
+  static __device__ __forceinline__ float tile_max(const uint4 (&c)[UNR]) {
+    uint32_t m0 = hmax2(wmax(c[0]), wmax(c[1]));
+    uint32_t m1 = hmax2(wmax(c[2]), wmax(c[3]));
+    return wfinal(hmax2(m0, m1));
+  }
+  static __device__ __forceinline__ float gmax(const uint4& w) { return wfinal(wmax(w)); }
   // accumulate the 8 elements of one group into the packed (S, U) state
   static __device__ __forceinline__ void accum(const uint4& w, float2 nm, float2& S, float2& U) {
     const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
@@ -261,12 +282,20 @@ struct Traits<__nv_bfloat16> {
 template <>
 struct Traits<float> {
   static constexpr int VEC = 4;
+  static constexpr uint32_t NEG_WORD = 0xff800000u;  // fp32 -inf
   static __device__ __forceinline__ float elem(const void* row, int64_t v) {
     return reinterpret_cast<const float*>(row)[v];
+  }
+  static __device__ __forceinline__ uint4 load_elems(const void* row, int64_t g) {
+    const uint32_t* f = reinterpret_cast<const uint32_t*>(row) + g * VEC;
+    return make_uint4(f[0], f[1], f[2], f[3]);
   }
   static __device__ __forceinline__ float gmax(const uint4& w) {
     return fmaxf(fmaxf(__uint_as_float(w.x), __uint_as_float(w.y)),
                  fmaxf(__uint_as_float(w.z), __uint_as_float(w.w)));
+  }
+  static __device__ __forceinline__ float tile_max(const uint4 (&c)[UNR]) {
+    return fmaxf(fmaxf(gmax(c[0]), gmax(c[1])), fmaxf(gmax(c[2]), gmax(c[3])));
   }
   static __device__ __forceinline__ void accum(const uint4& w, float2 nm, float2& S, float2& U) {
     const float2 x0 = make_float2(__uint_as_float(w.x), __uint_as_float(w.y));
@@ -288,37 +317,37 @@ struct Traits<float> {
 // ---- shared state of one CTA ------------------------------------------------------
 
 struct Smem {
-  uint64_t buf[NWARP][BUF];   // candidate group keys per warp
-  uint64_t list[NWARP][LIST]; // per-warp sorted group lists at the end of the stream
+  float tm[MAX_SLOTS][NT];    // per-thread tile (super-group) maxima
+  uint32_t wl[NWARP][32];     // per-warp sorted thread maxima, ord() encoded
+  float cand_v[CCAP];         // candidate super-groups: value
+  uint32_t cand_id[CCAP];     //   and (slot << 8 | thread), or TAIL_ID
+  uint64_t ebuf[ECAP];        // candidate element keys
   float pm[NWARP], pS[NWARP], pU[NWARP];
   int pbad[NWARP];
-  unsigned long long theta;   // CTA-wide group-key threshold (monotone)
-  unsigned int thval;         // CTA-wide value threshold, ord() encoded (monotone)
+  int ncand, nelem, nsel;
+  float theta1, theta;
+  float tail_max;             // maximum of the partial last group (cluster rank 0)
   // the CTA's merged partial state, read by cluster rank 0 through DSMEM
   float fm, fS, fU;
   int fbad;
-  uint64_t flist[LIST];
-  // decisions broadcast by warp 0
-  int careful;
+  uint64_t flist[32];
+  int careful, fallback;
 };
 
-// ---- warp-level candidate buffer ---------------------------------------------------
+// ---- warp-level top-32 of pushed keys ---------------------------------------------
 
 struct WarpTopK {
-  uint64_t* buf;
+  uint64_t* buf;  // at least 64 entries
   int cnt;        // warp-uniform
   uint64_t list;  // this lane's entry of the sorted list (lane 0 = best)
-  uint64_t thk;   // warp-uniform key threshold
-  float thv;      // warp-uniform value threshold
 
   __device__ __forceinline__ void push(bool c, uint64_t key, int lane) {
     const unsigned bal = __ballot_sync(FULL, c);
     if (c) buf[cnt + __popc(bal & ((1u << lane) - 1u))] = key;
     cnt += __popc(bal);
   }
-  // merge every full batch of 32 candidates into the list
-  __device__ __forceinline__ bool drain(int lane) {
-    bool merged = false;
+  // merge every full batch of 32 keys into the list
+  __device__ __forceinline__ void drain(int lane) {
     while (cnt >= 32) {
       __syncwarp();
       uint64_t k = buf[cnt - 32 + lane];
@@ -326,9 +355,7 @@ struct WarpTopK {
       __syncwarp();
       k = warp_sort_desc(k, lane);
       list = warp_merge_desc(list, k, lane);
-      merged = true;
     }
-    return merged;
   }
   // merge whatever is left (fewer than 32)
   __device__ __forceinline__ void drain_all(int lane) {

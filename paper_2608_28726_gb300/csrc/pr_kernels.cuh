@@ -184,7 +184,7 @@ __device__ __forceinline__ void block_reduce_state(Smem& sm, float& m, float& S,
 
 // ---- the row kernel ------------------------------------------------------------------------
 
-template <typename T, int MODE>
+template <typename T, int MODE, bool ALIGNED>
 __global__ void __launch_bounds__(NT) verify_rows(const Args a) {
   __shared__ Smem sm;
   using Tr = Traits<T>;
@@ -211,54 +211,60 @@ __global__ void __launch_bounds__(NT) verify_rows(const Args a) {
   }
 
   const char* rowp = reinterpret_cast<const char*>(a.logits) + row * a.row_stride * (int64_t)sizeof(T);
+  const uint4* vp = reinterpret_cast<const uint4*>(rowp);
   const int64_t V = a.vocab;
-  const int64_t gfull = a.aligned ? V / VEC : 0;  // 16-byte groups on the vector path
-  const int64_t gtot = (V + VEC - 1) / VEC;       // all groups; the last may be partial
-  const int64_t g0 = gfull * rank / C, g1 = gfull * (rank + 1) / C;
+  const int32_t gfull = (int32_t)(V / VEC);  // full 16-byte groups
+  const bool has_tail = (V % VEC) != 0;      // the partial last group, index gfull
+  const int32_t g0 = (int32_t)((int64_t)gfull * rank / C);
+  const int32_t g1 = (int32_t)((int64_t)gfull * (rank + 1) / C);
+  const int32_t ng = g1 - g0;
+  const int32_t nfull = ng / TILE, rem = ng - nfull * TILE;
+  const int32_t ntiles = nfull + (rem > 0 ? 1 : 0);
+  int shift = 0;
+  while (((ntiles + (1 << shift) - 1) >> shift) > MAX_SLOTS) ++shift;
+  const int32_t smask = (1 << shift) - 1;
+  const int32_t nslots = (ntiles + smask) >> shift;
+  const uint4 NEG = make_uint4(Tr::NEG_WORD, Tr::NEG_WORD, Tr::NEG_WORD, Tr::NEG_WORD);
 
   if (tid == 0) {
-    sm.theta = 0ull;
-    sm.thval = 0u;
+    sm.ncand = 0;
+    sm.nelem = 0;
+    sm.tail_max = -INFINITY;
   }
-  __syncthreads();
-
-  WarpTopK tk;
-  tk.buf = sm.buf[warp];
-  tk.cnt = 0;
-  tk.list = 0ull;
-  tk.thk = 0ull;
-  tk.thv = -INFINITY;
 
   float m = M2_INIT;
   float2 S2 = make_float2(0.f, 0.f), U2 = make_float2(0.f, 0.f);
+  float thr_max = -INFINITY, racc = -INFINITY;
   bool bad = false;
 
-  // ---- fast path: stream the groups [g0, g1) -------------------------------------------
+  // ---- stream the groups [g0, g1): tile t holds groups t*TILE + k*NT + tid ------------
   {
-    const uint4* vp = reinterpret_cast<const uint4*>(rowp);
-    const int64_t ng = g1 - g0;
-    const int64_t ntiles = (ng + NT * UNR - 1) / (NT * UNR);
+    auto load = [&](int32_t gi) -> uint4 {
+      return ALIGNED ? ld_stream(vp + g0 + gi) : Tr::load_elems(rowp, (int64_t)(g0 + gi));
+    };
     uint4 cur[UNR], nxt[UNR];
+    if (nfull > 0) {
 #pragma unroll
-    for (int k = 0; k < UNR; ++k) {
-      const int64_t g = g0 + k * NT + tid;
-      cur[k] = g < g1 ? ld_stream(vp + g) : make_uint4(0, 0, 0, 0);
+      for (int k = 0; k < UNR; ++k) cur[k] = load(k * NT + tid);
+    } else {
+#pragma unroll
+      for (int k = 0; k < UNR; ++k) cur[k] = (k * NT + tid < rem) ? load(k * NT + tid) : NEG;
     }
-    for (int64_t t = 0; t < ntiles; ++t) {
-      const int64_t gb = g0 + t * (NT * UNR) + tid;
-      if (t + 1 < ntiles) {
+    for (int32_t t = 0; t < ntiles; ++t) {
+      const int32_t nb = (t + 1) * TILE;
+      if (t + 1 < nfull) {
 #pragma unroll
-        for (int k = 0; k < UNR; ++k) {
-          const int64_t g = gb + NT * UNR + k * NT;
-          nxt[k] = g < g1 ? ld_stream(vp + g) : make_uint4(0, 0, 0, 0);
-        }
+        for (int k = 0; k < UNR; ++k) nxt[k] = load(nb + k * NT + tid);
+      } else if (t + 1 < ntiles) {
+#pragma unroll
+        for (int k = 0; k < UNR; ++k) nxt[k] = (k * NT + tid < rem) ? load(nb + k * NT + tid) : NEG;
       }
-      float vm[UNR];
-      float tmax = -INFINITY;
-#pragma unroll
-      for (int k = 0; k < UNR; ++k) {
-        vm[k] = (gb + k * NT < g1) ? Tr::gmax(cur[k]) : -INFINITY;
-        tmax = fmaxf(tmax, vm[k]);
+      const float tmax = Tr::tile_max(cur);
+      thr_max = fmaxf(thr_max, tmax);
+      racc = fmaxf(racc, tmax);
+      if ((t & smask) == smask || t == ntiles - 1) {
+        sm.tm[t >> shift][tid] = racc;
+        racc = -INFINITY;
       }
       // online rescale, branch-free (a no-op when the maximum did not move)
       const float mn = fmaxf(m, tmax * L2E);
@@ -268,80 +274,169 @@ __global__ void __launch_bounds__(NT) verify_rows(const Args a) {
       S2 = __fmul2_rn(make_float2(f, f), S2);
       m = mn;
       const float2 nm = make_float2(-m, -m);
+      if (t < nfull) {
 #pragma unroll
-      for (int k = 0; k < UNR; ++k)
-        if (gb + k * NT < g1) Tr::accum(cur[k], nm, S2, U2);
-
-      // top-K group candidates
-      if (t == 0) {
-        // the kc-th largest lane maximum is a lower bound of the kc-th group
-        const uint32_t o = warp_sort_desc32(ord(tmax), lane);
-        const uint32_t v0 = __shfl_sync(FULL, o, a.kc - 1);
-        if (lane == 0) atomicMax(&sm.thval, v0);
-        tk.thv = fmaxf(tk.thv, unord(v0));
+        for (int k = 0; k < UNR; ++k) Tr::accum(cur[k], nm, S2, U2);
       } else {
-        const unsigned long long th = *reinterpret_cast<volatile unsigned long long*>(&sm.theta);
-        const uint32_t tv = *reinterpret_cast<volatile unsigned int*>(&sm.thval);
-        if (th > tk.thk) {
-          tk.thk = th;
-          tk.thv = fmaxf(tk.thv, key_val(th));
-        }
-        if (tv) tk.thv = fmaxf(tk.thv, unord(tv));
-      }
-      if (__any_sync(FULL, tmax >= tk.thv)) {
 #pragma unroll
-        for (int k = 0; k < UNR; ++k) {
-          const int64_t g = gb + k * NT;
-          const bool c = (g < g1) && vm[k] >= tk.thv;
-          tk.push(c, c ? make_key(vm[k], (uint32_t)g) : 0ull, lane);
-        }
-        if (tk.drain(lane)) {
-          const uint64_t mine = shfl64(tk.list, a.kc - 1);
-          if (mine > tk.thk) {
-            tk.thk = mine;
-            tk.thv = fmaxf(tk.thv, key_val(mine));
-            if (lane == 0) atomicMax(&sm.theta, (unsigned long long)mine);
-          }
-        }
+        for (int k = 0; k < UNR; ++k)
+          if (k * NT + tid < rem) Tr::accum(cur[k], nm, S2, U2);
       }
 #pragma unroll
       for (int k = 0; k < UNR; ++k) cur[k] = nxt[k];
     }
   }
-
   float S = S2.x + S2.y, U = U2.x + U2.y;
 
-  // ---- generic groups (the partial last group, or every group of an unaligned row)
-  if (rank == 0) {
-    for (int64_t base = gfull; base < gtot; base += NT) {
-      const int64_t g = base + tid;
-      const bool valid = g < gtot;
-      float gm = -INFINITY;
-      if (valid) {
-        for (int j = 0; j < VEC; ++j) {
-          const int64_t v = g * VEC + j;
-          if (v < V) {
-            const float x = Tr::elem(rowp, v);
-            careful_add(x, m, S, U, bad);
-            if (!isnan(x)) gm = fmaxf(gm, x);
-          }
-        }
-      }
-      const bool c = valid && gm >= tk.thv;
-      tk.push(c, c ? make_key(gm, (uint32_t)g) : 0ull, lane);
-      tk.drain(lane);
+  // ---- the partial last group (fewer than VEC elements): cluster rank 0, thread 0
+  if (has_tail && rank == 0 && tid == 0) {
+    float tmx = -INFINITY;
+    for (int64_t v = (int64_t)gfull * VEC; v < V; ++v) {
+      const float x = Tr::elem(rowp, v);
+      careful_add(x, m, S, U, bad);
+      if (!isnan(x)) tmx = fmaxf(tmx, x);
     }
+    sm.tail_max = tmx;
+    thr_max = fmaxf(thr_max, tmx);
   }
 
-  tk.drain_all(lane);
-  sm.list[warp][lane] = tk.list;
+  // ---- theta1: the kc-th largest per-thread maximum (a lower bound of the kc-th element)
+  const int kc = a.kc, K = a.topk;
+  sm.wl[warp][lane] = warp_sort_desc<uint32_t>(ord(thr_max), lane);
   block_reduce_state(sm, m, S, U, bad, warp, lane);  // ends with a __syncthreads
-
-  uint64_t L = 0ull;  // warp 0: the CTA's 32 best group keys
   if (warp == 0) {
-    L = sm.list[0][lane];
+    uint32_t L = sm.wl[0][lane];
 #pragma unroll 1
-    for (int w2 = 1; w2 < NWARP; ++w2) L = warp_merge_desc(L, sm.list[w2][lane], lane);
+    for (int w2 = 1; w2 < NWARP; ++w2) L = warp_merge_desc<uint32_t>(L, sm.wl[w2][lane], lane);
+    const float th1 = unord(__shfl_sync(FULL, L, kc - 1));
+    if (lane == 0) {
+      sm.theta1 = th1;
+      sm.fallback = !(th1 > -INFINITY);
+    }
+  }
+  __syncthreads();
+
+  // ---- candidate super-groups: stored tile maxima >= theta1
+  const float th1 = sm.theta1;
+  if (!sm.fallback) {
+    for (int32_t s = 0; s < nslots; ++s) {
+      const float v = sm.tm[s][tid];
+      if (v >= th1) {
+        const int i = atomicAdd(&sm.ncand, 1);
+        if (i < CCAP) {
+          sm.cand_v[i] = v;
+          sm.cand_id[i] = ((uint32_t)s << 8) | (uint32_t)tid;
+        }
+      }
+    }
+    if (tid == 0 && has_tail && rank == 0 && sm.tail_max >= th1) {
+      const int i = atomicAdd(&sm.ncand, 1);
+      if (i < CCAP) {
+        sm.cand_v[i] = sm.tail_max;
+        sm.cand_id[i] = TAIL_ID;
+      }
+    }
+  }
+  __syncthreads();
+
+  // ---- theta: the exact kc-th largest candidate value (warp 0)
+  if (warp == 0 && !sm.fallback) {
+    const int n = sm.ncand;
+    if (n > CCAP) {
+      if (lane == 0) sm.fallback = 1;
+    } else {
+      uint32_t L = 0u;
+      for (int b0 = 0; b0 < n; b0 += 32) {
+        uint32_t k = b0 + lane < n ? ord(sm.cand_v[b0 + lane]) : 0u;
+        k = warp_sort_desc<uint32_t>(k, lane);
+        L = warp_merge_desc<uint32_t>(L, k, lane);
+      }
+      const float th = unord(__shfl_sync(FULL, L, kc - 1));
+      if (lane == 0) sm.theta = th;
+    }
+  }
+  __syncthreads();
+
+  // ---- re-read the candidates >= theta; elements >= theta become keys
+  if (!sm.fallback) {
+    const float th = sm.theta;
+    const int n = sm.ncand;
+    const int gpc = UNR << shift;  // groups per super-group
+    for (int i = tid; i < n * gpc; i += NT) {
+      const int c = i / gpc, j = i - c * gpc;
+      if (!(sm.cand_v[c] >= th)) continue;
+      const uint32_t id = sm.cand_id[c];
+      if (id == TAIL_ID) {
+        if (j != 0) continue;
+        for (int64_t v = (int64_t)gfull * VEC; v < V; ++v) {
+          const float x = Tr::elem(rowp, v);
+          if (x >= th) {
+            const int e = atomicAdd(&sm.nelem, 1);
+            if (e < ECAP) sm.ebuf[e] = make_key(x, (uint32_t)v);
+          }
+        }
+        continue;
+      }
+      const int32_t t = (int32_t)((id >> 8) << shift) + j / UNR;
+      const int32_t gi = t * TILE + (j % UNR) * NT + (int32_t)(id & 255u);
+      if (t >= ntiles || gi >= ng) continue;
+      const int32_t g = g0 + gi;
+      const uint4 wv = ALIGNED ? ld_stream(vp + g) : Tr::load_elems(rowp, (int64_t)g);
+#pragma unroll
+      for (int e2 = 0; e2 < VEC; ++e2) {
+        const float x = Tr::at(wv, e2);
+        if (x >= th) {
+          const int e = atomicAdd(&sm.nelem, 1);
+          if (e < ECAP) sm.ebuf[e] = make_key(x, (uint32_t)(g * VEC + e2));
+        }
+      }
+    }
+  }
+  __syncthreads();
+
+  // ---- the CTA's exact top-32 elements (warp 0)
+  uint64_t E = 0ull;
+  if (warp == 0) {
+    const int n = sm.nelem;
+    if (!sm.fallback && n <= ECAP) {
+      for (int b0 = 0; b0 < n; b0 += 32) {
+        uint64_t k = b0 + lane < n ? sm.ebuf[b0 + lane] : 0ull;
+        k = warp_sort_desc<uint64_t>(k, lane);
+        E = warp_merge_desc<uint64_t>(E, k, lane);
+      }
+    } else {
+      // exact scan of the whole range (rows whose ties overflow the buffers)
+      const float thr = th1;
+      WarpTopK ek;
+      ek.buf = sm.ebuf;
+      ek.cnt = 0;
+      ek.list = 0ull;
+      for (int32_t gb = 0; gb < ng; gb += 32) {
+        const int32_t gi = gb + lane;
+        const bool in = gi < ng;
+        uint4 wv = NEG;
+        if (in) wv = ALIGNED ? ld_stream(vp + g0 + gi) : Tr::load_elems(rowp, (int64_t)(g0 + gi));
+#pragma unroll 1
+        for (int e2 = 0; e2 < VEC; ++e2) {
+          const float x = Tr::at(wv, e2);
+          const bool c = in && x >= thr;
+          ek.push(c, c ? make_key(x, (uint32_t)((g0 + gi) * VEC + e2)) : 0ull, lane);
+          ek.drain(lane);
+        }
+      }
+      if (has_tail && rank == 0) {
+        for (int64_t v0 = (int64_t)gfull * VEC; v0 < V; v0 += 32) {
+          const int64_t v = v0 + lane;
+          const bool in = v < V;
+          const float x = in ? Tr::elem(rowp, v) : -INFINITY;
+          const bool c = in && x >= thr;
+          ek.push(c, c ? make_key(x, (uint32_t)v) : 0ull, lane);
+          ek.drain(lane);
+        }
+      }
+      ek.drain_all(lane);
+      E = ek.list;
+    }
   }
 
   // ---- split-vocab merge across the cluster (distributed shared memory)
@@ -353,7 +448,7 @@ __global__ void __launch_bounds__(NT) verify_rows(const Args a) {
         sm.fU = U;
         sm.fbad = bad;
       }
-      sm.flist[lane] = L;
+      sm.flist[lane] = E;
     }
     cluster_sync_all();
     if (rank == 0 && warp == 0) {
@@ -365,7 +460,7 @@ __global__ void __launch_bounds__(NT) verify_rows(const Args a) {
         lse_merge(m, S, U, mo, So, Uo);
         bad = bad || bo;
         const uint64_t peer = dsmem_ld_u64(dsmem_addr(&sm.flist[lane], r));
-        L = warp_merge_desc(L, peer, lane);
+        E = warp_merge_desc<uint64_t>(E, peer, lane);
       }
     }
     cluster_sync_all();
@@ -386,34 +481,6 @@ __global__ void __launch_bounds__(NT) verify_rows(const Args a) {
     bad = cbad;
   }
   if (warp != 0) return;
-
-  // ---- exact top-kc elements from the kc best groups (warp 0)
-  const int kc = a.kc, K = a.topk;
-  const uint64_t lastg = shfl64(L, kc - 1);
-  const float thg = lastg ? key_val(lastg) : -INFINITY;
-  WarpTopK ek;
-  ek.buf = sm.buf[0];
-  ek.cnt = 0;
-  ek.list = 0ull;
-  {
-    const bool has = lane < kc && L != 0ull;
-    const uint32_t g = key_idx(L);
-    uint4 wv = make_uint4(0, 0, 0, 0);
-    const bool vec = has && (int64_t)g < gfull;
-    if (vec) wv = ld_stream(reinterpret_cast<const uint4*>(rowp) + g);
-#pragma unroll 1
-    for (int j = 0; j < VEC; ++j) {
-      const int64_t v = (int64_t)g * VEC + j;
-      const bool in = has && v < V;
-      float x = -INFINITY;
-      if (in) x = vec ? Tr::at(wv, j) : Tr::elem(rowp, v);
-      const bool c = in && x >= thg;
-      ek.push(c, c ? make_key(x, (uint32_t)v) : 0ull, lane);
-      ek.drain(lane);
-    }
-    ek.drain_all(lane);
-  }
-  const uint64_t E = ek.list;
 
   // ---- finalize the row's record
   const int32_t y = a.chosen[row];

@@ -66,26 +66,27 @@ struct pr_ctx {
 namespace {
 
 template <typename T, int MODE>
-void* kernel_ptr() {
-  return reinterpret_cast<void*>(&prk::verify_rows<T, MODE>);
+void* kernel_ptr(bool aligned) {
+  return aligned ? reinterpret_cast<void*>(&prk::verify_rows<T, MODE, true>)
+                 : reinterpret_cast<void*>(&prk::verify_rows<T, MODE, false>);
 }
 
-void* row_kernel(pr_dtype dt, int mode) {
+void* row_kernel(pr_dtype dt, int mode, bool aligned) {
   if (dt == PR_DTYPE_BF16) {
-    if (mode == prk::MODE_FEATURES) return kernel_ptr<__nv_bfloat16, prk::MODE_FEATURES>();
-    if (mode == prk::MODE_ROUTE) return kernel_ptr<__nv_bfloat16, prk::MODE_ROUTE>();
-    return kernel_ptr<__nv_bfloat16, prk::MODE_DECODE>();
+    if (mode == prk::MODE_FEATURES) return kernel_ptr<__nv_bfloat16, prk::MODE_FEATURES>(aligned);
+    if (mode == prk::MODE_ROUTE) return kernel_ptr<__nv_bfloat16, prk::MODE_ROUTE>(aligned);
+    return kernel_ptr<__nv_bfloat16, prk::MODE_DECODE>(aligned);
   }
-  if (mode == prk::MODE_FEATURES) return kernel_ptr<float, prk::MODE_FEATURES>();
-  if (mode == prk::MODE_ROUTE) return kernel_ptr<float, prk::MODE_ROUTE>();
-  return kernel_ptr<float, prk::MODE_DECODE>();
+  if (mode == prk::MODE_FEATURES) return kernel_ptr<float, prk::MODE_FEATURES>(aligned);
+  if (mode == prk::MODE_ROUTE) return kernel_ptr<float, prk::MODE_ROUTE>(aligned);
+  return kernel_ptr<float, prk::MODE_DECODE>(aligned);
 }
 
 int blocks_per_sm(pr_ctx* c, pr_dtype dt, int mode) {
   int& v = c->bps[dt == PR_DTYPE_BF16 ? 1 : 0][mode];
   if (v == 0) {
     int n = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, row_kernel(dt, mode), prk::NT, 0) !=
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, row_kernel(dt, mode, true), prk::NT, 0) !=
             cudaSuccess ||
         n <= 0)
       n = 1;
@@ -121,7 +122,7 @@ pr_status launch_rows(pr_ctx* c, pr_dtype dt, int mode, const prk::Args& a, cuda
   cfg.attrs = attr;
   cfg.numAttrs = C > 1 ? 1 : 0;
   void* args[] = {const_cast<prk::Args*>(&a)};
-  PR_CUDA(cudaLaunchKernelExC(&cfg, row_kernel(dt, mode), args));
+  PR_CUDA(cudaLaunchKernelExC(&cfg, row_kernel(dt, mode, a.aligned != 0), args));
   g_launches.fetch_add(1, std::memory_order_relaxed);
   return PR_OK;
 }
