@@ -1,0 +1,56 @@
+"""Multi-rank host logic of bench.py on CPU (gloo, world size 2): every rank
+verifies its own batch, the job time is the slowest rank's, and the job value
+sums the rows of all ranks."""
+import os
+import socket
+
+import pytest
+import torch
+import torch.distributed as dist
+import torch.multiprocessing as mp
+
+
+def _free_port():
+    s = socket.socket()
+    s.bind(("127.0.0.1", 0))
+    port = s.getsockname()[1]
+    s.close()
+    return port
+
+
+def _worker(rank, world, port, out):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank),
+                      WORLD_SIZE=str(world), LOCAL_RANK=str(rank))
+    import bench
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    r, w, local = bench.dist_env()
+    assert (r, w, local) == (rank, world, rank)
+    bench.barrier(w)
+    t = bench.reduce_max(10.0 + 5.0 * rank, w, torch.device("cpu"))
+    out[rank] = t
+    dist.destroy_process_group()
+
+
+def test_max_over_ranks_with_gloo():
+    world = 2
+    port = _free_port()
+    mgr = mp.Manager()
+    out = mgr.dict()
+    mp.spawn(_worker, args=(world, port, out), nprocs=world, join=True)
+    assert out[0] == out[1] == 15.0
+
+
+def test_single_rank_needs_no_process_group():
+    import bench
+    assert bench.reduce_max(3.5, 1, torch.device("cpu")) == 3.5
+    bench.barrier(1)
+
+
+def test_reference_arm_on_nonzero_rank_does_no_work(monkeypatch):
+    import argparse
+
+    import bench
+    monkeypatch.setenv("RANK", "1")
+    monkeypatch.setenv("WORLD_SIZE", "2")
+    args = argparse.Namespace(gpus=2, steps=1, warmup=0)
+    assert bench.run_reference(args) == 0
