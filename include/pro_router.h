@@ -238,6 +238,44 @@ pr_status pr_decode_step(pr_ctx* ctx, const void* logits, pr_dtype dt, int32_t n
 pr_status pr_state_export(pr_ctx* ctx, void* host_buf, size_t* bytes);
 pr_status pr_state_import(pr_ctx* ctx, const void* host_buf, size_t bytes);
 
+/* ---- verification without allocation ------------------------------------------------- */
+
+#define PR_NOALLOC_MAX_ROWS 16384    /* largest n_rows pr_route_noalloc accepts */
+#define PR_NOALLOC_MAX_REQUESTS 1024 /* largest n_req pr_route_noalloc accepts */
+
+/*
+ * pr_route without a context and without allocating anything.  The paper has
+ * no counterpart: this call exists for hosts that cannot let a library call
+ * cudaMalloc -- an inference engine that reserves the GPU's memory for its own
+ * pool at start-up (so a later cudaMalloc fails or fragments that pool), or a
+ * serving loop that must not take the device-wide synchronisation a cudaMalloc
+ * or cudaFree can imply while other streams are running.
+ *
+ * It does what pr_route does for a whole batch in one call (row_base 0, no
+ * chunking), with K = 20 and the raw top-K entropy, on the current CUDA
+ * device.  The caller still passes every input and output buffer (device
+ * memory, the same layouts as pr_route).  The per-row records and request
+ * counters live in a fixed scratch array compiled into the library: each
+ * device that loads it keeps that array (about 580 KB) until the process
+ * exits.  Limits: 1 <= n_rows <= PR_NOALLOC_MAX_ROWS and
+ * 1 <= n_req <= PR_NOALLOC_MAX_REQUESTS; larger batches are rejected with
+ * PR_ERR_INVALID_ARG before anything is queued (use pr_route with a context
+ * instead).  offsets[n_req] must not exceed n_rows (requests reaching past it
+ * get PR_FLAG_BAD_OFFSETS).
+ *
+ * The first call on a device looks up the scratch array's device address and
+ * the launch shape, once, with that device current; make that first call
+ * before any stream capture.  Every call clears the counters it needs on
+ * `stream` and then reuses the same array, which keeps the previous call's
+ * contents: two calls whose work overlaps on the GPU (different streams, no
+ * ordering between them) race on the scratch and give undefined results.
+ * Calls issued on one stream, or otherwise ordered, are safe.
+ */
+pr_status pr_route_noalloc(const void* logits, pr_dtype dt, int64_t n_rows, int64_t vocab,
+                           int64_t row_stride, const int32_t* chosen, const int64_t* offsets,
+                           int32_t n_req, const float* w, float b, float tau, float* score,
+                           uint8_t* ship, uint32_t* req_flags, float* agg, void* stream);
+
 /* ---- diagnostics ------------------------------------------------------------------ */
 
 /* Static description of a status code. */

@@ -21,13 +21,14 @@ PR_FLAG_NONFINITE, PR_FLAG_BAD_CHOSEN, PR_FLAG_EMPTY_REQ = 1, 2, 4
 PR_FLAG_BAD_OFFSETS, PR_FLAG_BAD_SLOT = 8, 16
 PR_NFEAT, PR_NAGG, PR_MAX_TOPK = 8, 11, 32
 PR_OPT_TOPK, PR_OPT_TOPK_RENORM, PR_OPT_SPLIT = 0, 1, 2
+PR_NOALLOC_MAX_ROWS, PR_NOALLOC_MAX_REQUESTS = 16384, 1024
 
 # every symbol include/pro_router.h declares
 EXPORTS = (
     "pr_ctx_create", "pr_ctx_destroy", "pr_ctx_reset", "pr_ctx_set_option", "pr_ctx_flags",
     "pr_token_features", "pr_aggregate_score", "pr_route", "pr_route_host", "pr_decode_step",
     "pr_state_export", "pr_state_import", "pr_status_string", "pr_last_cuda_error",
-    "pr_launch_count",
+    "pr_launch_count", "pr_route_noalloc",
 )
 
 if not os.path.exists(LIB):
@@ -51,6 +52,8 @@ _SIGS = {
                       _P, _P, _P, _P, _P],
     "pr_decode_step": [_P, _P, ctypes.c_int, _I32, _I64, _I64, _P, _P, _P, _P, _F32, _F32, _P, _P,
                        _P, _P, _P],
+    "pr_route_noalloc": [_P, ctypes.c_int, _I64, _I64, _I64, _P, _P, _I32, _P, _F32, _F32, _P, _P,
+                         _P, _P, _P],
     "pr_state_export": [_P, _P, ctypes.POINTER(_SZ)],
     "pr_state_import": [_P, _P, _SZ],
 }
@@ -213,6 +216,22 @@ def pr_route_host(ctx, logits, chosen, offsets, w, b: float, tau: float, chunk_r
                               _ptr(offsets), n_req, _ptr(w), float(b), float(tau), int(chunk_rows),
                               _ptr(score), _ptr(ship), _ptr(req_flags), _ptr(agg),
                               _stream(stream)), "pr_route_host")
+    return score, ship, req_flags, agg
+
+
+def pr_route_noalloc(logits, chosen, offsets, w, b: float, tau: float, score, ship, req_flags,
+                     agg=None, vocab=None, stream=None):
+    """pr_route for callers that cannot allocate: no context, the library's
+    fixed scratch, every output buffer supplied by the caller (device tensors on
+    the current device).  Batches above PR_NOALLOC_MAX_ROWS rows or
+    PR_NOALLOC_MAX_REQUESTS requests raise PRError (invalid argument)."""
+    n = logits.size(0)
+    V, stride = _rows(logits, vocab)
+    n_req = offsets.numel() - 1
+    _check(_lib.pr_route_noalloc(_ptr(logits), _dtype(logits), n, V, stride, _ptr(chosen),
+                                 _ptr(offsets), n_req, _ptr(w), float(b), float(tau), _ptr(score),
+                                 _ptr(ship), _ptr(req_flags), _ptr(agg), _stream(stream)),
+           "pr_route_noalloc")
     return score, ship, req_flags, agg
 
 

@@ -3,6 +3,7 @@
 #include <cuda_runtime.h>
 
 #include <atomic>
+#include <mutex>
 #include <cmath>
 #include <cstdio>
 #include <cstring>
@@ -563,6 +564,126 @@ pr_status pr_route_host(pr_ctx* c, const void* logits, pr_dtype dt, int64_t n_ro
     PR_CUDA(cudaMemcpyAsync(agg, d_agg, (size_t)n_req * prk::NAGG * sizeof(float),
                             cudaMemcpyDeviceToHost, s));
   PR_CUDA(cudaStreamSynchronize(s));
+  return PR_OK;
+}
+
+}  // extern "C"
+
+// ---- verification without any allocation ---------------------------------------------
+//
+// Scratch of pr_route_noalloc: per-row records, per-request completion counters
+// and a flag word, in one file-scope device array.  Every device that loads
+// this library holds it (about 580 KB) until the process exits.
+
+namespace {
+
+constexpr size_t NA_REC_BYTES = (size_t)PR_NOALLOC_MAX_ROWS * prk::NFEAT * sizeof(float);
+constexpr size_t NA_RFL_BYTES = (size_t)PR_NOALLOC_MAX_ROWS * sizeof(uint32_t);
+constexpr size_t NA_CNT_BYTES = (size_t)PR_NOALLOC_MAX_REQUESTS * sizeof(int32_t);
+constexpr size_t NA_OFF_RFL = NA_REC_BYTES;
+constexpr size_t NA_OFF_CNT = NA_OFF_RFL + NA_RFL_BYTES;
+constexpr size_t NA_OFF_FLAGS = NA_OFF_CNT + NA_CNT_BYTES;
+constexpr size_t NA_BYTES = NA_OFF_FLAGS + 256;
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[NA_BYTES];
+
+constexpr int NA_MAX_DEVICES = 64;
+
+struct NoAllocDevice {
+  bool ready = false;
+  unsigned char* scratch = nullptr;  // device address of g_noalloc_scratch on this device
+  int num_sms = 0;
+  int bps[2] = {0, 0};               // CTAs per SM of the route kernel, fp32 / bf16
+};
+
+std::mutex g_noalloc_mu;
+NoAllocDevice g_noalloc_dev[NA_MAX_DEVICES];
+
+// Once per device, with that device current: the scratch's device address
+// (host code may not use the symbol itself) and the launch shape.
+pr_status noalloc_setup(int dev, NoAllocDevice** out) {
+  if (dev < 0 || dev >= NA_MAX_DEVICES) return PR_ERR_UNSUPPORTED;
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  NoAllocDevice& d = g_noalloc_dev[dev];
+  if (!d.ready) {
+    void* p = nullptr;
+    PR_CUDA(cudaGetSymbolAddress(&p, g_noalloc_scratch));
+    PR_CUDA(cudaDeviceGetAttribute(&d.num_sms, cudaDevAttrMultiProcessorCount, dev));
+    for (int i = 0; i < 2; ++i) {
+      const pr_dtype dt = i ? PR_DTYPE_BF16 : PR_DTYPE_F32;
+      int n = 0;
+      PR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(
+          &n, row_kernel(dt, prk::MODE_ROUTE, true), prk::NT, 0));
+      d.bps[i] = n > 0 ? n : 1;
+    }
+    d.scratch = static_cast<unsigned char*>(p);
+    d.ready = true;
+  }
+  *out = &d;
+  return PR_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+pr_status pr_route_noalloc(const void* logits, pr_dtype dt, int64_t n_rows, int64_t vocab,
+                           int64_t row_stride, const int32_t* chosen, const int64_t* offsets,
+                           int32_t n_req, const float* w, float b, float tau, float* score,
+                           uint8_t* ship, uint32_t* req_flags, float* agg, void* stream) {
+  pr_status st = check_rows(dt, logits, n_rows, vocab, row_stride);
+  if (st != PR_OK) return st;
+  if (n_rows > PR_NOALLOC_MAX_ROWS || n_req > PR_NOALLOC_MAX_REQUESTS) return PR_ERR_INVALID_ARG;
+  if (n_rows < 1 || n_req < 1 || !offsets || !w || !score || !ship || !req_flags || !chosen)
+    return PR_ERR_INVALID_ARG;
+  int dev = 0;
+  PR_CUDA(cudaGetDevice(&dev));
+  NoAllocDevice* d = nullptr;
+  if ((st = noalloc_setup(dev, &d)) != PR_OK) return st;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+
+  // the counters and the flag word start every call at zero
+  PR_CUDA(cudaMemsetAsync(d->scratch + NA_OFF_CNT, 0, (size_t)n_req * sizeof(int32_t), s));
+  PR_CUDA(cudaMemsetAsync(d->scratch + NA_OFF_FLAGS, 0, sizeof(uint32_t), s));
+
+  prk::Args a;
+  fill_row_args(a, logits, dt, n_rows, vocab, row_stride, chosen, 20, 0);
+  a.offsets = offsets;
+  a.n_req = n_req;
+  a.row_base = 0;
+  a.rec = reinterpret_cast<float*>(d->scratch);
+  a.rec_flags = reinterpret_cast<uint32_t*>(d->scratch + NA_OFF_RFL);
+  a.req_cnt = reinterpret_cast<int32_t*>(d->scratch + NA_OFF_CNT);
+  a.max_rows = n_rows;
+  a.w = w;
+  a.b = b;
+  a.zthr = zthreshold(tau);
+  a.score = score;
+  a.ship = ship;
+  a.req_flags = req_flags;
+  a.agg = agg;
+  a.ctx_flags = reinterpret_cast<uint32_t*>(d->scratch + NA_OFF_FLAGS);
+
+  // CTAs per row as in pr_route's automatic choice
+  const int64_t slots = (int64_t)d->num_sms * d->bps[dt == PR_DTYPE_BF16 ? 1 : 0];
+  int C = 1;
+  while (C < prk::MAXC && n_rows * C < 2 * slots) C <<= 1;
+  if (n_rows * C > 0x7fffffffLL) return PR_ERR_INVALID_ARG;
+  cudaLaunchConfig_t cfg;
+  memset(&cfg, 0, sizeof cfg);
+  cfg.gridDim = dim3((unsigned)(n_rows * C), 1, 1);
+  cfg.blockDim = dim3(prk::NT, 1, 1);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = (unsigned)C;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = C > 1 ? 1 : 0;
+  void* args[] = {&a};
+  PR_CUDA(cudaLaunchKernelExC(&cfg, row_kernel(dt, prk::MODE_ROUTE, a.aligned != 0), args));
+  g_launches.fetch_add(1, std::memory_order_relaxed);
   return PR_OK;
 }
 
