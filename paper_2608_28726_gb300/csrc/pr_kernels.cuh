@@ -1,6 +1,10 @@
-// Kernels of the verifier data path: the row kernel (Eq. 3 features, with a
+// Kernels of the verifier data path: the row kernels (Eq. 3 features, with a
 // fused pooling / scoring / ship-rule epilogue in route and decode modes) and
 // the standalone pooling kernel.  Algorithm notes are in pr_device.cuh.
+//   verify_rows_ws  persistent, warp-specialised: one CTA streams one row at a
+//                   time (used whenever a row needs no split)
+//   verify_rows     one thread-block cluster of C CTAs per row (C = 2, 4, 8:
+//                   batches too small to fill the GPU, e.g. decode steps)
 #pragma once
 
 #include "pr_device.cuh"
@@ -25,6 +29,7 @@ __device__ __forceinline__ Pooled pool_rows(const float* feat, const uint32_t* f
   float s[5] = {0.f, 0.f, 0.f, 0.f, 0.f};
   float mn[5] = {INFINITY, INFINITY, INFINITY, INFINITY, INFINITY};
   uint32_t fl = 0;
+#pragma unroll 4
   for (int64_t i = lo + lane; i < hi; i += 32) {
     const float4 a = __ldcg(reinterpret_cast<const float4*>(feat + i * NFEAT));
     const float4 c = __ldcg(reinterpret_cast<const float4*>(feat + i * NFEAT + 4));
@@ -182,7 +187,210 @@ __device__ __forceinline__ void block_reduce_state(Smem& sm, float& m, float& S,
   }
 }
 
-// ---- the row kernel ------------------------------------------------------------------------
+// ---- one row's features and the mode's epilogue (one warp) ------------------------------
+
+// What a row's epilogue needs that does not depend on the reduction: the
+// emitted token and its logit, and the row's request (rows, from the CSR
+// offsets) or decode slot.  The persistent kernel loads it for the next row
+// while it waits for that row's stream, off the critical path.
+struct RowPre {
+  int32_t y;       // emitted token id
+  float xy;        // its logit (NaN when y is outside [0, V))
+  int32_t r;       // request (features with offsets, route) or decode slot; -1 if none
+  int64_t lo, hi;  // rows of the request
+  int eos;         // decode: the request ends with this row
+};
+
+// Whole warp (the request search is warp-collective).
+template <typename T, int MODE>
+__device__ __forceinline__ RowPre load_pre(const Args& a, int64_t row, const char* rowp, int lane) {
+  using Tr = Traits<T>;
+  RowPre p;
+  p.y = a.chosen[row];
+  p.xy = (p.y >= 0 && (int64_t)p.y < a.vocab) ? Tr::elem(rowp, p.y) : NAN;
+  p.r = -1;
+  p.lo = p.hi = 0;
+  p.eos = 0;
+  if (MODE == MODE_FEATURES && a.offsets) {
+    p.r = find_request(a.offsets, a.n_req, row, lane);
+  } else if (MODE == MODE_ROUTE) {
+    p.r = find_request(a.offsets, a.n_req, a.row_base + row, lane);
+  } else if (MODE == MODE_DECODE) {
+    p.r = a.slot[row];
+    p.eos = a.eos[row];
+  }
+  if (MODE != MODE_DECODE && p.r >= 0) {
+    p.lo = __ldg(a.offsets + p.r);
+    p.hi = __ldg(a.offsets + p.r + 1);
+  }
+  return p;
+}
+
+__device__ __forceinline__ int atom_add_acq_rel(int* p, int v) {
+  int old;
+  asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+  return old;
+}
+
+// Eq. 3 features of the row from its (m, S, U) state and its top-32 element keys
+// E (lane 0 = largest), then, by mode: write the record; or fold it into the
+// request and, for the request's last row, pool / score / threshold; or fold it
+// into its decode slot.  Whole warp.
+template <typename T, int MODE>
+__device__ __forceinline__ void row_finish(const Args& a, int64_t row, float m, float S, float U,
+                                           bool bad, uint64_t E, const RowPre& pre, int lane) {
+  const int64_t V = a.vocab;
+  const int kc = a.kc, K = a.topk;
+  const int32_t y = pre.y;
+  uint32_t flags = 0;
+  if (y < 0 || (int64_t)y >= V) flags |= FLAG_BAD_CHOSEN;
+  const bool nonfinite = bad || !(S > 0.f) || !isfinite(S) || !isfinite(U);
+  if (nonfinite) flags |= FLAG_NONFINITE;
+
+  const float log2S = log2f(S);
+  const bool hasE = lane < kc && E != 0ull;
+  const float xk = hasE ? key_val(E) : -INFINITY;
+  const float lp2 = fmaf(xk, L2E, -m) - log2S;  // log2 p of this lane's token
+  const float pk = hasE ? exp2f(lp2) : 0.f;
+  float term = (lane < K && pk > 0.f) ? pk * lp2 : 0.f;
+  float pmass = lane < K ? pk : 0.f;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    term += __shfl_xor_sync(FULL, term, o);
+    pmass += __shfl_xor_sync(FULL, pmass, o);
+  }
+  const float hraw = term * LN2;  // sum over top-K of p ln p = -H^K
+  const float h = a.renorm ? (pmass > 0.f ? hraw / pmass - logf(pmass) : 0.f) : hraw;
+  const float x1 = __shfl_sync(FULL, xk, 0);
+  const float p1 = __shfl_sync(FULL, pk, 0);
+  const float p2 = V >= 2 ? __shfl_sync(FULL, pk, 1) : 0.f;
+  const uint64_t e1 = shfl64(E, 0), e2 = shfl64(E, 1);
+  float logp = NAN;
+  if (!(flags & FLAG_BAD_CHOSEN)) logp = (fmaf(pre.xy, L2E, -m) - log2S) * LN2;
+  float fv[NFEAT];
+  fv[0] = logp;
+  fv[1] = p1;
+  fv[2] = p1 - p2;
+  fv[3] = (log2S - U / S) * LN2;
+  fv[4] = h;
+  fv[5] = 0.f;
+  fv[6] = (m + log2S) * LN2;
+  fv[7] = x1;
+  int32_t i1 = (int32_t)key_idx(e1), i2 = V >= 2 ? (int32_t)key_idx(e2) : -1;
+  if (nonfinite) {
+#pragma unroll
+    for (int j = 0; j < NFEAT; ++j) fv[j] = NAN;
+    i1 = i2 = -1;
+  }
+
+  if (MODE == MODE_FEATURES) {
+    if (a.offsets && !nonfinite && pre.r >= 0)
+      fv[5] = (float)(row - pre.lo + 1) / (float)(pre.hi - pre.lo);
+    if (lane < NFEAT) {
+      float v = fv[0];
+#pragma unroll
+      for (int j = 1; j < NFEAT; ++j)
+        if (lane == j) v = fv[j];
+      a.feat[row * NFEAT + lane] = v;
+    }
+    if (lane == 0) {
+      a.top2[2 * row] = i1;
+      a.top2[2 * row + 1] = i2;
+      a.row_flags[row] = flags;
+    }
+    return;
+  }
+
+  if (MODE == MODE_ROUTE) {
+    const int64_t gr = a.row_base + row;
+    const int32_t r = pre.r;
+    const int64_t lo = pre.lo, hi = pre.hi;
+    if (r < 0 || lo < 0 || hi > a.max_rows) {
+      if (lane == 0) atomicOr(a.ctx_flags, FLAG_BAD_OFFSETS);
+      return;
+    }
+    if (!nonfinite) fv[5] = (float)(gr - lo + 1) / (float)(hi - lo);
+    int last = 0;
+    if (lane == 0) {
+      // the record, then one acquire-release increment: the request's last row
+      // sees every other row's record
+      float4* rp = reinterpret_cast<float4*>(a.rec + gr * NFEAT);
+      rp[0] = make_float4(fv[0], fv[1], fv[2], fv[3]);
+      rp[1] = make_float4(fv[4], fv[5], fv[6], fv[7]);
+      a.rec_flags[gr] = flags;
+      last = (atom_add_acq_rel(a.req_cnt + r, 1) == (int)(hi - lo) - 1);
+    }
+    last = __shfl_sync(FULL, last, 0);
+    if (last) {
+      const Pooled p = pool_rows(a.rec, a.rec_flags, lo, hi, a.w, a.b, a.zthr, lane);
+      write_pooled(p, r, a.agg, a.score, a.ship, a.req_flags, lane);
+      if (lane == 0) a.req_cnt[r] = 0;
+    }
+    return;
+  }
+
+  if (MODE == MODE_DECODE) {
+    if (lane != 0) return;
+    const int32_t s = pre.r;
+    if (s < 0 || s >= a.n_slots) {
+      atomicOr(a.ctx_flags, FLAG_BAD_SLOT);
+      return;
+    }
+    float* A = a.acc + (int64_t)s * ACC_WORDS;
+    const int32_t n = __float_as_int(A[0]) + 1;
+    const uint32_t fl = __float_as_uint(A[1]) | flags;
+    const float v[5] = {fv[0], fv[1], fv[2], -fv[3], fv[4]};
+#pragma unroll
+    for (int f = 0; f < 5; ++f) {
+      if (n == 1) {
+        A[2 + f] = v[f];
+        A[7 + f] = 0.f;
+        A[12 + f] = v[f];
+      } else {
+        // compensated (Kahan) running sum in step order
+        const float sum = A[2 + f], comp = A[7 + f];
+        const float yv = v[f] - comp;
+        const float tsum = sum + yv;
+        A[7 + f] = (tsum - sum) - yv;
+        A[2 + f] = tsum;
+        A[12 + f] = fminf(A[12 + f], v[f]);
+      }
+    }
+    if (!pre.eos) {
+      A[0] = __int_as_float(n);
+      A[1] = __uint_as_float(fl);
+      return;
+    }
+    // the request ends with this row: pool, score, ship rule, clear the slot
+    float ag[NAGG];
+    float sc;
+    uint8_t sh;
+    if (fl & (FLAG_NONFINITE | FLAG_BAD_CHOSEN)) {
+      for (int j = 0; j < NAGG; ++j) ag[j] = NAN;
+      sc = NAN;
+      sh = 0;
+    } else {
+      const float Tf = (float)n;
+      for (int f = 0; f < 5; ++f) {
+        ag[2 * f] = A[2 + f] / Tf;
+        ag[2 * f + 1] = A[12 + f];
+      }
+      ag[10] = (float)(n + 1) / (float)(2 * n);
+      float z = a.b;
+      for (int j = 0; j < NAGG; ++j) z = fmaf(__ldg(a.w + j), ag[j], z);
+      sc = 1.f / (1.f + expf(-z));
+      sh = (z >= a.zthr) ? 1 : 0;
+    }
+    if (a.agg)
+      for (int j = 0; j < NAGG; ++j) a.agg[(int64_t)s * NAGG + j] = ag[j];
+    a.score[s] = sc;
+    a.ship[s] = sh;
+    a.req_flags[s] = fl;
+    for (int j = 0; j < ACC_WORDS; ++j) A[j] = 0.f;
+  }
+}
+
+// ---- the row kernel for split rows: one thread-block cluster of C CTAs per row ----------------
 
 template <typename T, int MODE, bool ALIGNED>
 __global__ void __launch_bounds__(NT) verify_rows(const Args a) {
@@ -482,166 +690,418 @@ __global__ void __launch_bounds__(NT) verify_rows(const Args a) {
   }
   if (warp != 0) return;
 
-  // ---- finalize the row's record
-  const int32_t y = a.chosen[row];
-  uint32_t flags = 0;
-  if (y < 0 || (int64_t)y >= V) flags |= FLAG_BAD_CHOSEN;
-  const bool nonfinite = bad || !(S > 0.f) || !isfinite(S) || !isfinite(U);
-  if (nonfinite) flags |= FLAG_NONFINITE;
+  const RowPre pre = load_pre<T, MODE>(a, row, rowp, lane);
+  row_finish<T, MODE>(a, row, m, S, U, bad, E, pre, lane);
+}
 
-  const float log2S = log2f(S);
-  const bool hasE = lane < kc && E != 0ull;
-  const float xk = hasE ? key_val(E) : -INFINITY;
-  const float lp2 = fmaf(xk, L2E, -m) - log2S;  // log2 p of this lane's token
-  const float pk = hasE ? exp2f(lp2) : 0.f;
-  float term = (lane < K && pk > 0.f) ? pk * lp2 : 0.f;
-  float pmass = lane < K ? pk : 0.f;
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    term += __shfl_xor_sync(FULL, term, o);
-    pmass += __shfl_xor_sync(FULL, pmass, o);
-  }
-  const float hraw = term * LN2;  // sum over top-K of p ln p = -H^K
-  const float h = a.renorm ? (pmass > 0.f ? hraw / pmass - logf(pmass) : 0.f) : hraw;
-  const float x1 = __shfl_sync(FULL, xk, 0);
-  const float p1 = __shfl_sync(FULL, pk, 0);
-  const float p2 = V >= 2 ? __shfl_sync(FULL, pk, 1) : 0.f;
-  const uint64_t e1 = shfl64(E, 0), e2 = shfl64(E, 1);
-  float logp = NAN;
-  if (!(flags & FLAG_BAD_CHOSEN)) {
-    const float xy = Tr::elem(rowp, y);
-    logp = (fmaf(xy, L2E, -m) - log2S) * LN2;
-  }
-  float fv[NFEAT];
-  fv[0] = logp;
-  fv[1] = p1;
-  fv[2] = p1 - p2;
-  fv[3] = (log2S - U / S) * LN2;
-  fv[4] = h;
-  fv[5] = 0.f;
-  fv[6] = (m + log2S) * LN2;
-  fv[7] = x1;
-  int32_t i1 = (int32_t)key_idx(e1), i2 = V >= 2 ? (int32_t)key_idx(e2) : -1;
-  if (nonfinite) {
-#pragma unroll
-    for (int j = 0; j < NFEAT; ++j) fv[j] = NAN;
-    i1 = i2 = -1;
-  }
+// ---- the persistent, warp-specialised row kernel (one CTA per row at a time) -----------------
+//
+// NWARP streaming warps read rows blockIdx.x, blockIdx.x + gridDim.x, ...; they
+// never wait on the per-row selection: at the end of a row they leave its tile
+// maxima, per-warp (m, S, U) and sorted per-thread maxima in one of two shared
+// buffers, signal the finaliser warp with a named barrier and go on (the next
+// row's first tile is already in flight).  The finaliser warp turns a buffer
+// into the row's exact top-K, features and epilogue, then hands the buffer
+// back.  Named barriers (bar.arrive / bar.sync with NT + 32 threads) are the
+// only synchronisation; every thread reaches each of them a known number of
+// times, so no wait depends on data.
 
-  if (MODE == MODE_FEATURES) {
-    if (a.offsets && !nonfinite) {
-      const int32_t r = find_request(a.offsets, a.n_req, row, lane);
-      if (r >= 0) {
-        const int64_t lo = __ldg(a.offsets + r), hi = __ldg(a.offsets + r + 1);
-        fv[5] = (float)(row - lo + 1) / (float)(hi - lo);
+constexpr int NT_WS = NT + 32;
+constexpr int BAR_FULL = 1;   // ids 1, 2: buffer b holds a streamed row
+constexpr int BAR_EMPTY = 3;  // ids 3, 4: buffer b may be overwritten
+
+__device__ __forceinline__ void named_bar_sync(int id, int n) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
+}
+__device__ __forceinline__ void named_bar_arrive(int id, int n) {
+  asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(n) : "memory");
+}
+
+struct SmemWS {
+  float tm[2][MAX_SLOTS][NT];   // per-thread tile (super-group) maxima, two row buffers
+  uint32_t wl[2][NWARP][32];    // per-warp sorted per-thread maxima, ord() encoded
+  float thmax[2][NT];           // per-thread maxima
+  float pm[2][NWARP], pS[2][NWARP], pU[2][NWARP];
+  uint32_t thl[NT];             // finaliser: threads whose maximum reaches theta1
+  float cand_v[CCAP];           // finaliser: candidate super-groups
+  uint32_t cand_id[CCAP];
+  uint64_t ebuf[ECAP];          // finaliser: candidate element keys
+};
+
+// Row geometry shared by the streaming warps and the finaliser (C = 1).
+struct RowGeom {
+  int32_t gfull, nfull, rem, ntiles, shift, smask, nslots;
+  bool has_tail;
+  __device__ __forceinline__ RowGeom(int64_t V, int vec) {
+    gfull = (int32_t)(V / vec);
+    has_tail = (V % vec) != 0;
+    nfull = gfull / TILE;
+    rem = gfull - nfull * TILE;
+    ntiles = nfull + (rem > 0 ? 1 : 0);
+    shift = 0;
+    while (((ntiles + (1 << shift) - 1) >> shift) > MAX_SLOTS) ++shift;
+    smask = (1 << shift) - 1;
+    nslots = (ntiles + smask) >> shift;
+  }
+};
+
+// The finaliser warp's work for one streamed row held in buffer b.
+template <typename T, int MODE, bool ALIGNED>
+__device__ __noinline__ void finalize_ws(const Args& a, SmemWS& sm, int b, int64_t row,
+                                         const RowGeom& geo, const RowPre& pre, int lane) {
+  using Tr = Traits<T>;
+  constexpr int VEC = Tr::VEC;
+  const int64_t V = a.vocab;
+  const int kc = a.kc;
+  const char* rowp = reinterpret_cast<const char*>(a.logits) + row * a.row_stride * (int64_t)sizeof(T);
+  const uint4* vp = reinterpret_cast<const uint4*>(rowp);
+  const uint4 NEG = make_uint4(Tr::NEG_WORD, Tr::NEG_WORD, Tr::NEG_WORD, Tr::NEG_WORD);
+  const unsigned lt = (1u << lane) - 1u;
+
+  // ---- the row's (m, S, U) from the streaming warps' partials
+  float m = lane < NWARP ? sm.pm[b][lane] : M2_INIT;
+  float S = lane < NWARP ? sm.pS[b][lane] : 0.f;
+  float U = lane < NWARP ? sm.pU[b][lane] : 0.f;
+#pragma unroll
+  for (int o = NWARP / 2; o > 0; o >>= 1) {
+    const float mo = __shfl_xor_sync(FULL, m, o);
+    const float So = __shfl_xor_sync(FULL, S, o);
+    const float Uo = __shfl_xor_sync(FULL, U, o);
+    lse_merge(m, S, U, mo, So, Uo);
+  }
+  m = __shfl_sync(FULL, m, 0);
+  S = __shfl_sync(FULL, S, 0);
+  U = __shfl_sync(FULL, U, 0);
+  bool bad = false;
+
+  // ---- the partial last group (fewer than VEC elements)
+  float tail_max = -INFINITY;
+  if (geo.has_tail) {
+    if (lane == 0) {
+      for (int64_t v = (int64_t)geo.gfull * VEC; v < V; ++v) {
+        const float x = Tr::elem(rowp, v);
+        careful_add(x, m, S, U, bad);
+        if (!isnan(x)) tail_max = fmaxf(tail_max, x);
       }
     }
-    if (lane < NFEAT) {
-      float v = fv[0];
+    m = __shfl_sync(FULL, m, 0);
+    S = __shfl_sync(FULL, S, 0);
+    U = __shfl_sync(FULL, U, 0);
+    bad = __shfl_sync(FULL, (int)bad, 0) != 0;
+    tail_max = __shfl_sync(FULL, tail_max, 0);
+  }
+
+  // ---- theta1: the kc-th largest per-thread maximum
+  uint32_t L = sm.wl[b][0][lane];
+#pragma unroll 1
+  for (int w = 1; w < NWARP; ++w) L = warp_merge_desc<uint32_t>(L, sm.wl[b][w][lane], lane);
+  if (geo.has_tail) L = warp_merge_desc<uint32_t>(L, lane == 0 ? ord(tail_max) : 0u, lane);
+  const float th1 = unord(__shfl_sync(FULL, L, kc - 1));
+  bool fb = !(th1 > -INFINITY);
+
+  // ---- candidate super-groups: stored maxima >= theta1.  Only threads whose
+  // own maximum reaches theta1 can hold one (typically a few more than kc).
+  int n = 0;
+  if (!fb) {
+    int nth = 0;
 #pragma unroll
-      for (int j = 1; j < NFEAT; ++j)
-        if (lane == j) v = fv[j];
-      a.feat[row * NFEAT + lane] = v;
+    for (int j = 0; j < NT / 32; ++j) {
+      const int t = j * 32 + lane;
+      const bool c = sm.thmax[b][t] >= th1;
+      const unsigned bal = __ballot_sync(FULL, c);
+      if (c) sm.thl[nth + __popc(bal & lt)] = (uint32_t)t;
+      nth += __popc(bal);
+    }
+    __syncwarp();
+    const int total = nth * geo.nslots;
+#pragma unroll 1
+    for (int i0 = 0; i0 < total; i0 += 32) {
+      const int it = i0 + lane;
+      bool c = false;
+      float v = -INFINITY;
+      uint32_t id = 0;
+      if (it < total) {
+        const int q = it / geo.nslots, s2 = it - q * geo.nslots;
+        const uint32_t t = sm.thl[q];
+        v = sm.tm[b][s2][t];
+        c = v >= th1;
+        id = ((uint32_t)s2 << 8) | t;
+      }
+      const unsigned bal = __ballot_sync(FULL, c);
+      const int pos = n + __popc(bal & lt);
+      if (c && pos < CCAP) {
+        sm.cand_v[pos] = v;
+        sm.cand_id[pos] = id;
+      }
+      n += __popc(bal);
+    }
+    if (geo.has_tail && tail_max >= th1) {
+      if (lane == 0 && n < CCAP) {
+        sm.cand_v[n] = tail_max;
+        sm.cand_id[n] = TAIL_ID;
+      }
+      ++n;
+    }
+    if (n > CCAP) fb = true;
+  }
+  __syncwarp();
+
+  // ---- theta: the exact kc-th largest candidate value
+  float th = th1;
+  if (!fb) {
+    uint32_t L2 = 0u;
+#pragma unroll 1
+    for (int b0 = 0; b0 < n; b0 += 32) {
+      uint32_t k = b0 + lane < n ? ord(sm.cand_v[b0 + lane]) : 0u;
+      k = warp_sort_desc<uint32_t>(k, lane);
+      L2 = warp_merge_desc<uint32_t>(L2, k, lane);
+    }
+    th = unord(__shfl_sync(FULL, L2, kc - 1));
+  }
+
+  // ---- re-read the candidates >= theta (4 group loads in flight per lane)
+  int ne = 0;
+  if (!fb) {
+    const int gpc = UNR << geo.shift;
+    const int total = n * gpc;
+#pragma unroll 1
+    for (int i0 = 0; i0 < total; i0 += 128) {
+      uint4 wv[4];
+      int32_t gsel[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int it = i0 + q * 32 + lane;
+        gsel[q] = -1;
+        if (it < total) {
+          const int c = it / gpc, j = it - c * gpc;
+          const uint32_t id = sm.cand_id[c];
+          if (id != TAIL_ID && sm.cand_v[c] >= th) {
+            const int32_t t = (int32_t)((id >> 8) << geo.shift) + j / UNR;
+            const int32_t gi = t * TILE + (j % UNR) * NT + (int32_t)(id & 255u);
+            if (t < geo.ntiles && gi < geo.gfull) gsel[q] = gi;
+          }
+        }
+        wv[q] = NEG;
+        if (gsel[q] >= 0) wv[q] = ALIGNED ? ld_stream(vp + gsel[q]) : Tr::load_elems(rowp, gsel[q]);
+      }
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+#pragma unroll
+        for (int e2 = 0; e2 < VEC; ++e2) {
+          const float x = Tr::at(wv[q], e2);
+          const bool c = gsel[q] >= 0 && x >= th;
+          const unsigned bal = __ballot_sync(FULL, c);
+          const int pos = ne + __popc(bal & lt);
+          if (c && pos < ECAP) sm.ebuf[pos] = make_key(x, (uint32_t)(gsel[q] * VEC + e2));
+          ne += __popc(bal);
+        }
+      }
+    }
+    if (geo.has_tail && tail_max >= th) {
+      const int64_t v = (int64_t)geo.gfull * VEC + lane;
+      const float x = v < V ? Tr::elem(rowp, v) : -INFINITY;
+      const bool c = v < V && x >= th;
+      const unsigned bal = __ballot_sync(FULL, c);
+      const int pos = ne + __popc(bal & lt);
+      if (c && pos < ECAP) sm.ebuf[pos] = make_key(x, (uint32_t)v);
+      ne += __popc(bal);
+    }
+    if (ne > ECAP) fb = true;
+  }
+  __syncwarp();
+
+  // ---- the row's exact top-32 elements
+  uint64_t E = 0ull;
+  if (!fb) {
+#pragma unroll 1
+    for (int b0 = 0; b0 < ne; b0 += 32) {
+      uint64_t k = b0 + lane < ne ? sm.ebuf[b0 + lane] : 0ull;
+      k = warp_sort_desc<uint64_t>(k, lane);
+      E = warp_merge_desc<uint64_t>(E, k, lane);
+    }
+  } else {
+    // exact scan of the whole row (rows whose ties overflow the buffers)
+    WarpTopK ek;
+    ek.buf = sm.ebuf;
+    ek.cnt = 0;
+    ek.list = 0ull;
+#pragma unroll 1
+    for (int32_t g0 = 0; g0 < geo.gfull; g0 += 32) {
+      const int32_t g = g0 + lane;
+      const bool in = g < geo.gfull;
+      uint4 wv = NEG;
+      if (in) wv = ALIGNED ? ld_stream(vp + g) : Tr::load_elems(rowp, g);
+#pragma unroll 1
+      for (int e2 = 0; e2 < VEC; ++e2) {
+        const float x = Tr::at(wv, e2);
+        const bool c = in && x >= th1;
+        ek.push(c, c ? make_key(x, (uint32_t)(g * VEC + e2)) : 0ull, lane);
+        ek.drain(lane);
+      }
+    }
+    if (geo.has_tail) {
+      const int64_t v = (int64_t)geo.gfull * VEC + lane;
+      const bool in = v < V;
+      const float x = in ? Tr::elem(rowp, v) : -INFINITY;
+      const bool c = in && x >= th1;
+      ek.push(c, c ? make_key(x, (uint32_t)v) : 0ull, lane);
+      ek.drain(lane);
+    }
+    ek.drain_all(lane);
+    E = ek.list;
+  }
+
+  // ---- rows that made the fast accumulators non-finite: re-stream with guards
+  if (!bad && !(isfinite(S) && isfinite(U))) {
+    float cm = M2_INIT, cS = 0.f, cU = 0.f;
+    bool cbad = false;
+#pragma unroll 1
+    for (int64_t v = lane; v < V; v += 32) careful_add(Tr::elem(rowp, v), cm, cS, cU, cbad);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float mo = __shfl_xor_sync(FULL, cm, o);
+      const float So = __shfl_xor_sync(FULL, cS, o);
+      const float Uo = __shfl_xor_sync(FULL, cU, o);
+      lse_merge(cm, cS, cU, mo, So, Uo);
+    }
+    m = __shfl_sync(FULL, cm, 0);
+    S = __shfl_sync(FULL, cS, 0);
+    U = __shfl_sync(FULL, cU, 0);
+    bad = __any_sync(FULL, cbad);
+  }
+
+  row_finish<T, MODE>(a, row, m, S, U, bad, E, pre, lane);
+}
+
+template <typename T, int MODE, bool ALIGNED>
+__global__ void __launch_bounds__(NT_WS) verify_rows_ws(const Args a) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  SmemWS& sm = *reinterpret_cast<SmemWS*>(smem_raw);
+  using Tr = Traits<T>;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int64_t G = gridDim.x;
+
+  // Route mode: results of empty requests touching this launch's row range and
+  // of requests whose offsets are inconsistent.
+  if (MODE == MODE_ROUTE) {
+    for (int64_t r = (int64_t)blockIdx.x * NT_WS + tid; r < a.n_req; r += G * NT_WS) {
+      const int64_t lo = a.offsets[r], hi = a.offsets[r + 1];
+      if (lo < 0 || hi < lo || hi > a.max_rows) {
+        write_special(r, NAN, FLAG_BAD_OFFSETS, a.agg, a.score, a.ship, a.req_flags);
+        atomicOr(a.ctx_flags, FLAG_BAD_OFFSETS);
+      } else if (lo == hi && lo >= a.row_base && lo <= a.row_base + a.n_rows) {
+        write_special(r, 0.f, FLAG_EMPTY_REQ, a.agg, a.score, a.ship, a.req_flags);
+      }
+    }
+  }
+
+  const RowGeom geo(a.vocab, Tr::VEC);
+
+  if (warp == NWARP) {
+    // ---- the finaliser warp: the next row's inputs are fetched while its
+    // stream is still running
+    auto rowp_of = [&](int64_t r) {
+      return reinterpret_cast<const char*>(a.logits) + r * a.row_stride * (int64_t)sizeof(T);
+    };
+    int i = 0;
+    int64_t row = blockIdx.x;
+    RowPre pre = load_pre<T, MODE>(a, row, rowp_of(row), lane);
+    for (; row < a.n_rows; row += G, ++i) {
+      const int b = i & 1;
+      named_bar_sync(BAR_FULL + b, NT_WS);
+      finalize_ws<T, MODE, ALIGNED>(a, sm, b, row, geo, pre, lane);
+      if (row + 2 * G < a.n_rows) {
+        __syncwarp();
+        __threadfence_block();
+        named_bar_arrive(BAR_EMPTY + b, NT_WS);
+      }
+      if (row + G < a.n_rows) pre = load_pre<T, MODE>(a, row + G, rowp_of(row + G), lane);
+    }
+    return;
+  }
+
+  // ---- the streaming warps
+  const uint4 NEG = make_uint4(Tr::NEG_WORD, Tr::NEG_WORD, Tr::NEG_WORD, Tr::NEG_WORD);
+  auto load_tile = [&](uint4 (&dst)[UNR], int64_t r, int32_t t) {
+    const char* rp = reinterpret_cast<const char*>(a.logits) + r * a.row_stride * (int64_t)sizeof(T);
+    const uint4* vp = reinterpret_cast<const uint4*>(rp);
+    const int32_t base = t * TILE + tid;
+    if (t < geo.nfull) {
+#pragma unroll
+      for (int k = 0; k < UNR; ++k)
+        dst[k] = ALIGNED ? ld_stream(vp + base + k * NT) : Tr::load_elems(rp, base + k * NT);
+    } else {
+#pragma unroll
+      for (int k = 0; k < UNR; ++k)
+        dst[k] = (k * NT + tid < geo.rem)
+                     ? (ALIGNED ? ld_stream(vp + base + k * NT) : Tr::load_elems(rp, base + k * NT))
+                     : NEG;
+    }
+  };
+
+  uint4 cur[UNR], nxt[UNR];
+  int64_t row = blockIdx.x;
+  if (row < a.n_rows && geo.ntiles > 0) load_tile(cur, row, 0);
+  int i = 0;
+  while (row < a.n_rows) {
+    const int b = i & 1;
+    if (i >= 2) named_bar_sync(BAR_EMPTY + b, NT_WS);
+    const int64_t next = row + G;
+    float m = M2_INIT;
+    float2 S2 = make_float2(0.f, 0.f), U2 = make_float2(0.f, 0.f);
+    float thr_max = -INFINITY, racc = -INFINITY;
+    for (int32_t t = 0; t < geo.ntiles; ++t) {
+      if (t + 1 < geo.ntiles) load_tile(nxt, row, t + 1);
+      else if (next < a.n_rows) load_tile(nxt, next, 0);
+      const float tmax = Tr::tile_max(cur);
+      thr_max = fmaxf(thr_max, tmax);
+      racc = fmaxf(racc, tmax);
+      if ((t & geo.smask) == geo.smask || t == geo.ntiles - 1) {
+        sm.tm[b][t >> geo.shift][tid] = racc;
+        racc = -INFINITY;
+      }
+      const float mn = fmaxf(m, tmax * L2E);
+      const float dl = m - mn;
+      const float f = ex2(dl);
+      U2 = __fmul2_rn(make_float2(f, f), __ffma2_rn(make_float2(dl, dl), S2, U2));
+      S2 = __fmul2_rn(make_float2(f, f), S2);
+      m = mn;
+      const float2 nm = make_float2(-m, -m);
+      if (t < geo.nfull) {
+#pragma unroll
+        for (int k = 0; k < UNR; ++k) Tr::accum(cur[k], nm, S2, U2);
+      } else {
+#pragma unroll
+        for (int k = 0; k < UNR; ++k)
+          if (k * NT + tid < geo.rem) Tr::accum(cur[k], nm, S2, U2);
+      }
+#pragma unroll
+      for (int k = 0; k < UNR; ++k) cur[k] = nxt[k];
+    }
+    // the warp's partial state and its sorted per-thread maxima
+    float S = S2.x + S2.y, U = U2.x + U2.y;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float mo = __shfl_xor_sync(FULL, m, o);
+      const float So = __shfl_xor_sync(FULL, S, o);
+      const float Uo = __shfl_xor_sync(FULL, U, o);
+      lse_merge(m, S, U, mo, So, Uo);
     }
     if (lane == 0) {
-      a.top2[2 * row] = i1;
-      a.top2[2 * row + 1] = i2;
-      a.row_flags[row] = flags;
+      sm.pm[b][warp] = m;
+      sm.pS[b][warp] = S;
+      sm.pU[b][warp] = U;
     }
-    return;
-  }
-
-  if (MODE == MODE_ROUTE) {
-    const int64_t gr = a.row_base + row;
-    const int32_t r = find_request(a.offsets, a.n_req, gr, lane);
-    const int64_t lo = r >= 0 ? __ldg(a.offsets + r) : 0, hi = r >= 0 ? __ldg(a.offsets + r + 1) : 0;
-    if (r < 0 || lo < 0 || hi > a.max_rows) {
-      if (lane == 0) atomicOr(a.ctx_flags, FLAG_BAD_OFFSETS);
-      return;
-    }
-    if (!nonfinite) fv[5] = (float)(gr - lo + 1) / (float)(hi - lo);
-    if (lane < NFEAT) {
-      float v = fv[0];
-#pragma unroll
-      for (int j = 1; j < NFEAT; ++j)
-        if (lane == j) v = fv[j];
-      a.rec[gr * NFEAT + lane] = v;
-    }
-    if (lane == 0) a.rec_flags[gr] = flags;
-    __threadfence();
+    sm.wl[b][warp][lane] = warp_sort_desc<uint32_t>(ord(thr_max), lane);
+    sm.thmax[b][tid] = thr_max;
     __syncwarp();
-    int last = 0;
-    if (lane == 0) last = (atomicAdd(a.req_cnt + r, 1) == (int)(hi - lo) - 1);
-    last = __shfl_sync(FULL, last, 0);
-    if (last) {
-      __threadfence();
-      const Pooled p = pool_rows(a.rec, a.rec_flags, lo, hi, a.w, a.b, a.zthr, lane);
-      write_pooled(p, r, a.agg, a.score, a.ship, a.req_flags, lane);
-      if (lane == 0) a.req_cnt[r] = 0;
-    }
-    return;
-  }
-
-  if (MODE == MODE_DECODE) {
-    if (lane != 0) return;
-    const int32_t s = a.slot[row];
-    if (s < 0 || s >= a.n_slots) {
-      atomicOr(a.ctx_flags, FLAG_BAD_SLOT);
-      return;
-    }
-    float* A = a.acc + (int64_t)s * ACC_WORDS;
-    const int32_t n = __float_as_int(A[0]) + 1;
-    const uint32_t fl = __float_as_uint(A[1]) | flags;
-    const float v[5] = {fv[0], fv[1], fv[2], -fv[3], fv[4]};
-#pragma unroll
-    for (int f = 0; f < 5; ++f) {
-      if (n == 1) {
-        A[2 + f] = v[f];
-        A[7 + f] = 0.f;
-        A[12 + f] = v[f];
-      } else {
-        // compensated (Kahan) running sum in step order
-        const float sum = A[2 + f], comp = A[7 + f];
-        const float yv = v[f] - comp;
-        const float tsum = sum + yv;
-        A[7 + f] = (tsum - sum) - yv;
-        A[2 + f] = tsum;
-        A[12 + f] = fminf(A[12 + f], v[f]);
-      }
-    }
-    if (!a.eos[row]) {
-      A[0] = __int_as_float(n);
-      A[1] = __uint_as_float(fl);
-      return;
-    }
-    // the request ends with this row: pool, score, ship rule, clear the slot
-    float ag[NAGG];
-    float sc;
-    uint8_t sh;
-    if (fl & (FLAG_NONFINITE | FLAG_BAD_CHOSEN)) {
-      for (int j = 0; j < NAGG; ++j) ag[j] = NAN;
-      sc = NAN;
-      sh = 0;
-    } else {
-      const float Tf = (float)n;
-      for (int f = 0; f < 5; ++f) {
-        ag[2 * f] = A[2 + f] / Tf;
-        ag[2 * f + 1] = A[12 + f];
-      }
-      ag[10] = (float)(n + 1) / (float)(2 * n);
-      float z = a.b;
-      for (int j = 0; j < NAGG; ++j) z = fmaf(__ldg(a.w + j), ag[j], z);
-      sc = 1.f / (1.f + expf(-z));
-      sh = (z >= a.zthr) ? 1 : 0;
-    }
-    if (a.agg)
-      for (int j = 0; j < NAGG; ++j) a.agg[(int64_t)s * NAGG + j] = ag[j];
-    a.score[s] = sc;
-    a.ship[s] = sh;
-    a.req_flags[s] = fl;
-    for (int j = 0; j < ACC_WORDS; ++j) A[j] = 0.f;
+    __threadfence_block();
+    named_bar_arrive(BAR_FULL + b, NT_WS);
+    row = next;
+    ++i;
   }
 }
+
 
 // ---- standalone pooling kernel: one warp per request ----------------------------------
 

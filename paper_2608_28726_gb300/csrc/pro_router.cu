@@ -6,6 +6,7 @@
 #include <mutex>
 #include <cmath>
 #include <cstdio>
+#include <algorithm>
 #include <cstring>
 #include <new>
 
@@ -62,6 +63,8 @@ struct pr_ctx {
   cudaEvent_t ev_free[2] = {nullptr, nullptr};
   // occupancy cache per (dtype, mode)
   int bps[2][3] = {{0, 0, 0}, {0, 0, 0}};
+  // persistent kernel: CTAs per SM per (dtype, mode, aligned); 0 = not set up yet
+  int ws_bps[2][3][2] = {};
 };
 
 namespace {
@@ -96,6 +99,38 @@ int blocks_per_sm(pr_ctx* c, pr_dtype dt, int mode) {
   return v;
 }
 
+template <typename T, int MODE>
+void* ws_kernel_ptr(bool aligned) {
+  return aligned ? reinterpret_cast<void*>(&prk::verify_rows_ws<T, MODE, true>)
+                 : reinterpret_cast<void*>(&prk::verify_rows_ws<T, MODE, false>);
+}
+
+void* ws_kernel(pr_dtype dt, int mode, bool aligned) {
+  if (dt == PR_DTYPE_BF16) {
+    if (mode == prk::MODE_FEATURES) return ws_kernel_ptr<__nv_bfloat16, prk::MODE_FEATURES>(aligned);
+    if (mode == prk::MODE_ROUTE) return ws_kernel_ptr<__nv_bfloat16, prk::MODE_ROUTE>(aligned);
+    return ws_kernel_ptr<__nv_bfloat16, prk::MODE_DECODE>(aligned);
+  }
+  if (mode == prk::MODE_FEATURES) return ws_kernel_ptr<float, prk::MODE_FEATURES>(aligned);
+  if (mode == prk::MODE_ROUTE) return ws_kernel_ptr<float, prk::MODE_ROUTE>(aligned);
+  return ws_kernel_ptr<float, prk::MODE_DECODE>(aligned);
+}
+
+// shared memory opt-in and residency of the persistent kernel, once per instantiation
+pr_status ws_setup(pr_ctx* c, pr_dtype dt, int mode, bool aligned, int* bps) {
+  int& v = c->ws_bps[dt == PR_DTYPE_BF16 ? 1 : 0][mode][aligned ? 1 : 0];
+  if (v == 0) {
+    void* f = ws_kernel(dt, mode, aligned);
+    PR_CUDA(cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)sizeof(prk::SmemWS)));
+    int n = 0;
+    PR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, f, prk::NT_WS, sizeof(prk::SmemWS)));
+    v = n > 0 ? n : 1;
+  }
+  *bps = v;
+  return PR_OK;
+}
+
 // CTAs per row: the forced option, or enough to put two waves of CTAs on the GPU
 int choose_split(pr_ctx* c, pr_dtype dt, int mode, int64_t n_rows) {
   if (c->split == 1 || c->split == 2 || c->split == 4 || c->split == 8) return c->split;
@@ -108,6 +143,18 @@ int choose_split(pr_ctx* c, pr_dtype dt, int mode, int64_t n_rows) {
 pr_status launch_rows(pr_ctx* c, pr_dtype dt, int mode, const prk::Args& a, cudaStream_t st) {
   if (a.n_rows == 0) return PR_OK;
   const int C = choose_split(c, dt, mode, a.n_rows);
+  if (C == 1) {
+    // persistent warp-specialised kernel: every SM gets its resident CTAs
+    int bps = 0;
+    const pr_status s = ws_setup(c, dt, mode, a.aligned != 0, &bps);
+    if (s != PR_OK) return s;
+    const int64_t grid = std::min<int64_t>(a.n_rows, (int64_t)c->num_sms * bps);
+    void* args[] = {const_cast<prk::Args*>(&a)};
+    PR_CUDA(cudaLaunchKernel(ws_kernel(dt, mode, a.aligned != 0), dim3((unsigned)grid),
+                             dim3(prk::NT_WS), args, sizeof(prk::SmemWS), st));
+    g_launches.fetch_add(1, std::memory_order_relaxed);
+    return PR_OK;
+  }
   if (a.n_rows * C > 0x7fffffffLL) return PR_ERR_INVALID_ARG;
   cudaLaunchConfig_t cfg;
   memset(&cfg, 0, sizeof cfg);

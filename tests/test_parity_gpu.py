@@ -62,20 +62,24 @@ def _check_features(feat, top2, rflags, of, oi, ofl, what):
 
 # ---- per-token features ----------------------------------------------------------------
 
+# split 0 lets the library choose (a cluster per row for these small batches);
+# split 1 forces the persistent warp-specialised kernel
+@pytest.mark.parametrize("split", [0, 1])
 @pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
 @pytest.mark.parametrize("V", [1, 2, 7, 8, 9, 31, 160, 1000, 4097, 32000, 70001])
-def test_features_vocab_sizes(ctx, dtype, V):
-    _set(ctx)
+def test_features_vocab_sizes(ctx, dtype, V, split):
+    _set(ctx, split=split)
     x, ch = random_rows(24, V, dtype, seed=V)
     feat, top2, rf = B.pr_token_features(ctx, x, ch, topk=20)
     of, oi, ofl = _oracle_rows(x, ch)
     _check_features(feat, top2, rf, of, oi, ofl, "V=%d" % V)
 
 
+@pytest.mark.parametrize("split", [0, 1])
 @pytest.mark.parametrize("K", [1, 2, 3, 19, 20, 21, 32])
 @pytest.mark.parametrize("renorm", [0, 1])
-def test_features_topk(ctx, K, renorm):
-    _set(ctx, renorm=renorm)
+def test_features_topk(ctx, K, renorm, split):
+    _set(ctx, renorm=renorm, split=split)
     x, ch = random_rows(16, 3001, torch.bfloat16, seed=100 + K)
     feat, top2, rf = B.pr_token_features(ctx, x, ch, topk=K)
     of, oi, ofl = _oracle_rows(x, ch, K=K, renorm=bool(renorm))
@@ -83,10 +87,12 @@ def test_features_topk(ctx, K, renorm):
     _set(ctx)
 
 
+@pytest.mark.parametrize("split", [0, 1])
 @pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
 @pytest.mark.parametrize("shift", [1, 3])
-def test_features_unaligned_rows(ctx, dtype, shift):
-    """Row starts off the 16-byte grid take the guarded element path."""
+def test_features_unaligned_rows(ctx, dtype, shift, split):
+    """Row starts off the 16-byte grid take the element-load path."""
+    _set(ctx, split=split)
     V = 2053
     base, ch = random_rows(12, V + shift + 5, dtype, seed=7 + shift)
     x = base[:, shift:shift + V]  # row stride V + shift + 5, start offset `shift` elements
@@ -94,6 +100,7 @@ def test_features_unaligned_rows(ctx, dtype, shift):
     feat, top2, rf = B.pr_token_features(ctx, x, ch % V, topk=20)
     of, oi, ofl = _oracle_rows(x.contiguous(), ch % V)
     _check_features(feat, top2, rf, of, oi, ofl, "unaligned")
+    _set(ctx)
 
 
 def test_features_vocab_narrower_than_stride(ctx):
@@ -133,10 +140,11 @@ def _special_rows(V, dtype):
     return x.cuda(), torch.tensor(chosen, dtype=torch.int32).cuda()
 
 
+@pytest.mark.parametrize("split", [0, 1])
 @pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
 @pytest.mark.parametrize("V", [257, 4096])
-def test_features_special_rows(ctx, dtype, V):
-    _set(ctx)
+def test_features_special_rows(ctx, dtype, V, split):
+    _set(ctx, split=split)
     x, ch = _special_rows(V, dtype)
     feat, top2, rf = B.pr_token_features(ctx, x, ch, topk=20)
     of, oi, ofl = _oracle_rows(x, ch)
@@ -152,6 +160,23 @@ def test_split_factor_invariance(ctx, dtype):
         _set(ctx, split=split)
         feat, top2, rf = B.pr_token_features(ctx, x, ch, topk=20)
         _check_features(feat, top2, rf, of, oi, ofl, "split=%d" % split)
+    _set(ctx)
+
+
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+def test_persistent_many_rows_per_cta(ctx, dtype):
+    """3,000 rows: each persistent CTA carries several rows through both shared
+    buffers; special rows (masked, NaN, ties, constant) sit among them."""
+    _set(ctx, split=1)
+    V = 4097
+    x, ch = random_rows(3000, V, dtype, seed=77)
+    sx, sch = _special_rows(V, dtype)
+    for j in range(sx.size(0)):
+        x[97 * j + 5] = sx[j]
+        ch[97 * j + 5] = sch[j]
+    feat, top2, rf = B.pr_token_features(ctx, x, ch, topk=20)
+    of, oi, ofl = _oracle_rows(x, ch)
+    _check_features(feat, top2, rf, of, oi, ofl, "persistent")
     _set(ctx)
 
 
@@ -185,9 +210,10 @@ def _check_requests(score, ship, rflags, agg, o, tau, what):
     assert_ship(ship.cpu().numpy(), o["ship"], o["score"], tau)
 
 
+@pytest.mark.parametrize("split", [0, 1])
 @pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
-def test_route_matches_oracle(ctx, dtype):
-    _set(ctx)
+def test_route_matches_oracle(ctx, dtype, split):
+    _set(ctx, split=split)
     lengths = [3, 0, 40, 1, 77, 0, 12, 130, 2]
     x, ch, off, w, b = _batch(lengths, 3001, dtype, seed=21)
     o = oracle.route(as_oracle(x), ch.cpu().numpy(), off, w.astype(np.float64), b, 0.5)
