@@ -718,19 +718,18 @@ __device__ __forceinline__ void named_bar_arrive(int id, int n) {
 }
 
 struct SmemWS {
-  float tm[2][MAX_SLOTS][NT];   // per-thread tile (super-group) maxima, two row buffers
+  float4 tinfo[2][NT];          // per thread: best, second and third tile maxima, and
+                                //   (best tile | second tile << 16); two row buffers
   uint32_t wl[2][NWARP][32];    // per-warp sorted per-thread maxima, ord() encoded
-  float thmax[2][NT];           // per-thread maxima
   float pm[2][NWARP], pS[2][NWARP], pU[2][NWARP];
-  uint32_t thl[NT];             // finaliser: threads whose maximum reaches theta1
-  float cand_v[CCAP];           // finaliser: candidate super-groups
-  uint32_t cand_id[CCAP];
+  float cand_v[CCAP];           // finaliser: candidate tiles (value,
+  uint32_t cand_id[CCAP];       //   tile << 8 | thread)
   uint64_t ebuf[ECAP];          // finaliser: candidate element keys
 };
 
 // Row geometry shared by the streaming warps and the finaliser (C = 1).
 struct RowGeom {
-  int32_t gfull, nfull, rem, ntiles, shift, smask, nslots;
+  int32_t gfull, nfull, rem, ntiles;
   bool has_tail;
   __device__ __forceinline__ RowGeom(int64_t V, int vec) {
     gfull = (int32_t)(V / vec);
@@ -738,14 +737,18 @@ struct RowGeom {
     nfull = gfull / TILE;
     rem = gfull - nfull * TILE;
     ntiles = nfull + (rem > 0 ? 1 : 0);
-    shift = 0;
-    while (((ntiles + (1 << shift) - 1) >> shift) > MAX_SLOTS) ++shift;
-    smask = (1 << shift) - 1;
-    nslots = (ntiles + smask) >> shift;
   }
 };
 
 // The finaliser warp's work for one streamed row held in buffer b.
+//
+// Every streaming thread reports its best and second-best tile (value and
+// index) and its third-best tile value.  theta1 = the kc-th largest thread
+// maximum.  Candidate tiles are the best / second-best tiles >= theta1; a
+// thread whose third-best value also reaches theta1 contributes all its
+// tiles, and then theta stays theta1 (exact, if slower).  Otherwise theta =
+// the kc-th largest candidate value.  Elements >= theta of the candidate
+// tiles are the only ones that can be among the top kc.
 template <typename T, int MODE, bool ALIGNED>
 __device__ __noinline__ void finalize_ws(const Args& a, SmemWS& sm, int b, int64_t row,
                                          const RowGeom& geo, const RowPre& pre, int lane) {
@@ -791,50 +794,67 @@ __device__ __noinline__ void finalize_ws(const Args& a, SmemWS& sm, int b, int64
     tail_max = __shfl_sync(FULL, tail_max, 0);
   }
 
-  // ---- theta1: the kc-th largest per-thread maximum
-  uint32_t L = sm.wl[b][0][lane];
-#pragma unroll 1
-  for (int w = 1; w < NWARP; ++w) L = warp_merge_desc<uint32_t>(L, sm.wl[b][w][lane], lane);
+  // ---- theta1: the kc-th largest per-thread maximum (a merge tree over the
+  // eight per-warp sorted lists; independent merges interleave)
+  uint32_t L0 = warp_merge_desc<uint32_t>(sm.wl[b][0][lane], sm.wl[b][1][lane], lane);
+  uint32_t L1 = warp_merge_desc<uint32_t>(sm.wl[b][2][lane], sm.wl[b][3][lane], lane);
+  uint32_t L2 = warp_merge_desc<uint32_t>(sm.wl[b][4][lane], sm.wl[b][5][lane], lane);
+  uint32_t L3 = warp_merge_desc<uint32_t>(sm.wl[b][6][lane], sm.wl[b][7][lane], lane);
+  L0 = warp_merge_desc<uint32_t>(L0, L1, lane);
+  L2 = warp_merge_desc<uint32_t>(L2, L3, lane);
+  uint32_t L = warp_merge_desc<uint32_t>(L0, L2, lane);
   if (geo.has_tail) L = warp_merge_desc<uint32_t>(L, lane == 0 ? ord(tail_max) : 0u, lane);
   const float th1 = unord(__shfl_sync(FULL, L, kc - 1));
   bool fb = !(th1 > -INFINITY);
 
-  // ---- candidate super-groups: stored maxima >= theta1.  Only threads whose
-  // own maximum reaches theta1 can hold one (typically a few more than kc).
-  int n = 0;
+  // ---- candidate tiles
+  int n = 0;            // candidate tiles
+  bool all3 = false;    // some thread has three tiles >= theta1
   if (!fb) {
-    int nth = 0;
-#pragma unroll
+#pragma unroll 2
     for (int j = 0; j < NT / 32; ++j) {
-      const int t = j * 32 + lane;
-      const bool c = sm.thmax[b][t] >= th1;
-      const unsigned bal = __ballot_sync(FULL, c);
-      if (c) sm.thl[nth + __popc(bal & lt)] = (uint32_t)t;
-      nth += __popc(bal);
-    }
-    __syncwarp();
-    const int total = nth * geo.nslots;
-#pragma unroll 1
-    for (int i0 = 0; i0 < total; i0 += 32) {
-      const int it = i0 + lane;
-      bool c = false;
-      float v = -INFINITY;
-      uint32_t id = 0;
-      if (it < total) {
-        const int q = it / geo.nslots, s2 = it - q * geo.nslots;
-        const uint32_t t = sm.thl[q];
-        v = sm.tm[b][s2][t];
-        c = v >= th1;
-        id = ((uint32_t)s2 << 8) | t;
+      const uint32_t t = (uint32_t)(j * 32 + lane);
+      const float4 inf = sm.tinfo[b][t];
+      const uint32_t ids = __float_as_uint(inf.w);
+      const bool c1 = inf.x >= th1, c2 = inf.y >= th1, c3 = inf.z >= th1;
+      all3 = all3 || c3;
+      // the best and second-best tiles
+      const unsigned b1 = __ballot_sync(FULL, c1);
+      const unsigned b2 = __ballot_sync(FULL, c2 && !c3);
+      const int p1 = n + __popc(b1 & lt);
+      const int p2 = n + __popc(b1) + __popc(b2 & lt);
+      if (c1 && p1 < CCAP) {
+        sm.cand_v[p1] = inf.x;
+        sm.cand_id[p1] = ((ids & 0xffffu) << 8) | t;
       }
-      const unsigned bal = __ballot_sync(FULL, c);
-      const int pos = n + __popc(bal & lt);
-      if (c && pos < CCAP) {
-        sm.cand_v[pos] = v;
-        sm.cand_id[pos] = id;
+      if (c2 && !c3 && p2 < CCAP) {
+        sm.cand_v[p2] = inf.y;
+        sm.cand_id[p2] = ((ids >> 16) << 8) | t;
       }
-      n += __popc(bal);
+      n += __popc(b1) + __popc(b2);
+      // a thread with a third tile >= theta1: every other tile of it
+      unsigned b3 = __ballot_sync(FULL, c3);
+      while (b3) {
+        const int src = __ffs(b3) - 1;
+        b3 &= b3 - 1;
+        const uint32_t ts = (uint32_t)(j * 32 + src);
+        const uint32_t ids_s = __shfl_sync(FULL, ids, src);
+        const uint32_t ti1 = ids_s & 0xffffu;
+        for (int t0 = 0; t0 < geo.ntiles; t0 += 32) {
+          const int tt = t0 + lane;
+          const bool c = tt < geo.ntiles && (uint32_t)tt != ti1;
+          const unsigned bb = __ballot_sync(FULL, c);
+          const int pos = n + __popc(bb & lt);
+          if (c && pos < CCAP) {
+            sm.cand_v[pos] = th1;
+            sm.cand_id[pos] = ((uint32_t)tt << 8) | ts;
+          }
+          n += __popc(bb);
+        }
+      }
     }
+    all3 = __any_sync(FULL, all3);
+    // the partial last group is a candidate too (its elements are read below)
     if (geo.has_tail && tail_max >= th1) {
       if (lane == 0 && n < CCAP) {
         sm.cand_v[n] = tail_max;
@@ -846,43 +866,56 @@ __device__ __noinline__ void finalize_ws(const Args& a, SmemWS& sm, int b, int64
   }
   __syncwarp();
 
-  // ---- theta: the exact kc-th largest candidate value
+  // ---- re-read the candidate tiles (issued first, so that sorting the
+  // candidates for theta overlaps the loads), then keep elements >= theta
+  const int total = fb ? 0 : n * UNR;
+  uint4 wv[4];
+  int32_t gsel[4];
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const int it = q * 32 + lane;
+    gsel[q] = -1;
+    if (it < total) {
+      const uint32_t id = sm.cand_id[it >> 2];
+      const int32_t gi = (int32_t)(id >> 8) * TILE + (it & (UNR - 1)) * NT + (int32_t)(id & 255u);
+      if (id != TAIL_ID && gi < geo.gfull) gsel[q] = gi;
+    }
+    wv[q] = NEG;
+    if (gsel[q] >= 0) wv[q] = ALIGNED ? ld_stream(vp + gsel[q]) : Tr::load_elems(rowp, gsel[q]);
+  }
+
+  // ---- theta: the exact kc-th largest candidate value (theta1 if a thread
+  // contributed all its tiles)
   float th = th1;
-  if (!fb) {
-    uint32_t L2 = 0u;
+  if (!fb && !all3) {
+    uint32_t Lc = 0u;
 #pragma unroll 1
     for (int b0 = 0; b0 < n; b0 += 32) {
       uint32_t k = b0 + lane < n ? ord(sm.cand_v[b0 + lane]) : 0u;
       k = warp_sort_desc<uint32_t>(k, lane);
-      L2 = warp_merge_desc<uint32_t>(L2, k, lane);
+      Lc = warp_merge_desc<uint32_t>(Lc, k, lane);
     }
-    th = unord(__shfl_sync(FULL, L2, kc - 1));
+    const uint32_t kth = __shfl_sync(FULL, Lc, kc - 1);
+    if (kth != 0u) th = unord(kth);  // (there are always kc candidates; kept as a guard)
   }
 
-  // ---- re-read the candidates >= theta (4 group loads in flight per lane)
   int ne = 0;
   if (!fb) {
-    const int gpc = UNR << geo.shift;
-    const int total = n * gpc;
-#pragma unroll 1
     for (int i0 = 0; i0 < total; i0 += 128) {
-      uint4 wv[4];
-      int32_t gsel[4];
+      if (i0 > 0) {
+        // more than 128 candidate groups: the next batch of loads
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const int it = i0 + q * 32 + lane;
-        gsel[q] = -1;
-        if (it < total) {
-          const int c = it / gpc, j = it - c * gpc;
-          const uint32_t id = sm.cand_id[c];
-          if (id != TAIL_ID && sm.cand_v[c] >= th) {
-            const int32_t t = (int32_t)((id >> 8) << geo.shift) + j / UNR;
-            const int32_t gi = t * TILE + (j % UNR) * NT + (int32_t)(id & 255u);
-            if (t < geo.ntiles && gi < geo.gfull) gsel[q] = gi;
+        for (int q = 0; q < 4; ++q) {
+          const int it = i0 + q * 32 + lane;
+          gsel[q] = -1;
+          if (it < total && sm.cand_v[it >> 2] >= th) {
+            const uint32_t id = sm.cand_id[it >> 2];
+            const int32_t gi = (int32_t)(id >> 8) * TILE + (it & (UNR - 1)) * NT + (int32_t)(id & 255u);
+            if (id != TAIL_ID && gi < geo.gfull) gsel[q] = gi;
           }
+          wv[q] = NEG;
+          if (gsel[q] >= 0) wv[q] = ALIGNED ? ld_stream(vp + gsel[q]) : Tr::load_elems(rowp, gsel[q]);
         }
-        wv[q] = NEG;
-        if (gsel[q] >= 0) wv[q] = ALIGNED ? ld_stream(vp + gsel[q]) : Tr::load_elems(rowp, gsel[q]);
       }
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
@@ -929,11 +962,11 @@ __device__ __noinline__ void finalize_ws(const Args& a, SmemWS& sm, int b, int64
     for (int32_t g0 = 0; g0 < geo.gfull; g0 += 32) {
       const int32_t g = g0 + lane;
       const bool in = g < geo.gfull;
-      uint4 wv = NEG;
-      if (in) wv = ALIGNED ? ld_stream(vp + g) : Tr::load_elems(rowp, g);
+      uint4 w4 = NEG;
+      if (in) w4 = ALIGNED ? ld_stream(vp + g) : Tr::load_elems(rowp, g);
 #pragma unroll 1
       for (int e2 = 0; e2 < VEC; ++e2) {
-        const float x = Tr::at(wv, e2);
+        const float x = Tr::at(w4, e2);
         const bool c = in && x >= th1;
         ek.push(c, c ? make_key(x, (uint32_t)(g * VEC + e2)) : 0ull, lane);
         ek.drain(lane);
@@ -974,7 +1007,7 @@ __device__ __noinline__ void finalize_ws(const Args& a, SmemWS& sm, int b, int64
 }
 
 template <typename T, int MODE, bool ALIGNED>
-__global__ void __launch_bounds__(NT_WS) verify_rows_ws(const Args a) {
+__global__ void __launch_bounds__(NT_WS, 3) verify_rows_ws(const Args a) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   SmemWS& sm = *reinterpret_cast<SmemWS*>(smem_raw);
   using Tr = Traits<T>;
@@ -1049,16 +1082,22 @@ __global__ void __launch_bounds__(NT_WS) verify_rows_ws(const Args a) {
     const int64_t next = row + G;
     float m = M2_INIT;
     float2 S2 = make_float2(0.f, 0.f), U2 = make_float2(0.f, 0.f);
-    float thr_max = -INFINITY, racc = -INFINITY;
+    // this thread's best, second and third tile maxima and the first two tiles
+    float v1 = -INFINITY, v2 = -INFINITY, v3 = -INFINITY;
+    uint32_t i1 = 0, i2 = 0;
     for (int32_t t = 0; t < geo.ntiles; ++t) {
       if (t + 1 < geo.ntiles) load_tile(nxt, row, t + 1);
       else if (next < a.n_rows) load_tile(nxt, next, 0);
       const float tmax = Tr::tile_max(cur);
-      thr_max = fmaxf(thr_max, tmax);
-      racc = fmaxf(racc, tmax);
-      if ((t & geo.smask) == geo.smask || t == geo.ntiles - 1) {
-        sm.tm[b][t >> geo.shift][tid] = racc;
-        racc = -INFINITY;
+      {
+        const bool c1 = tmax > v1, c2 = tmax > v2;
+        v3 = fmaxf(v3, fminf(tmax, v2));
+        const float nv2 = c1 ? v1 : (c2 ? tmax : v2);
+        const uint32_t ni2 = c1 ? i1 : (c2 ? (uint32_t)t : i2);
+        v1 = c1 ? tmax : v1;
+        i1 = c1 ? (uint32_t)t : i1;
+        v2 = nv2;
+        i2 = ni2;
       }
       const float mn = fmaxf(m, tmax * L2E);
       const float dl = m - mn;
@@ -1078,7 +1117,7 @@ __global__ void __launch_bounds__(NT_WS) verify_rows_ws(const Args a) {
 #pragma unroll
       for (int k = 0; k < UNR; ++k) cur[k] = nxt[k];
     }
-    // the warp's partial state and its sorted per-thread maxima
+    // the warp's partial state, its sorted per-thread maxima, the tile report
     float S = S2.x + S2.y, U = U2.x + U2.y;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
@@ -1092,8 +1131,8 @@ __global__ void __launch_bounds__(NT_WS) verify_rows_ws(const Args a) {
       sm.pS[b][warp] = S;
       sm.pU[b][warp] = U;
     }
-    sm.wl[b][warp][lane] = warp_sort_desc<uint32_t>(ord(thr_max), lane);
-    sm.thmax[b][tid] = thr_max;
+    sm.wl[b][warp][lane] = warp_sort_desc<uint32_t>(ord(v1), lane);
+    sm.tinfo[b][tid] = make_float4(v1, v2, v3, __uint_as_float(i1 | (i2 << 16)));
     __syncwarp();
     __threadfence_block();
     named_bar_arrive(BAR_FULL + b, NT_WS);
@@ -1101,7 +1140,6 @@ __global__ void __launch_bounds__(NT_WS) verify_rows_ws(const Args a) {
     ++i;
   }
 }
-
 
 // ---- standalone pooling kernel: one warp per request ----------------------------------
 
