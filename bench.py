@@ -275,8 +275,8 @@ def run_gb300(args):
     # end to end from pinned host memory through the public C ABI
     hx = x.cpu().pin_memory()
     hc = ch.cpu().pin_memory()
-    hoff = torch.from_numpy(wl.offsets)
-    hw = torch.from_numpy(wl.w)
+    hoff = torch.from_numpy(wl.offsets).pin_memory()
+    hw = torch.from_numpy(wl.w).pin_memory()
     hs = torch.empty(wl.n_req).pin_memory()
     hsh = torch.empty(wl.n_req, dtype=torch.uint8).pin_memory()
     hf = torch.empty(wl.n_req, dtype=torch.int32).pin_memory()
@@ -360,13 +360,133 @@ def run_gb300(args):
         dist.destroy_process_group()
     return 0
 
+def run_other_workload(args):
+    """The four other workloads, timed the same way (CUDA events on the stream,
+    max over ranks); inputs resident in HBM.  Batches smaller than L2 are
+    rotated over distinct copies so every step reads from DRAM."""
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", init_method="env://")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    from paper_2608_28726_gb300 import build as prbuild
+    prbuild.build()
+    from paper_2608_28726_gb300 import binding as B
+    stream = torch.cuda.current_stream(dev)
+    name = args.workload
+    launches0 = None
+
+    if name == "decode":
+        tr = W.decode_trace()
+        wl = tr.as_workload()
+        S, T = tr.n_slots, tr.n_steps
+        x_all = torch.empty(T * S, wl.vocab, dtype=wl.torch_dtype, device=dev)
+        ch_all = torch.empty(T * S, dtype=torch.int32, device=dev)
+        W.rows(wl, 0, T * S, device=dev, out=x_all, chosen_out=ch_all)
+        eos = torch.from_numpy(tr.eos).to(dev)
+        slot = torch.arange(S, dtype=torch.int32, device=dev)
+        w = torch.from_numpy(tr.w).to(dev)
+        ctx = B.pr_ctx_create(local, max_rows=S, max_requests=S)
+        outs = (torch.empty(S, device=dev), torch.empty(S, dtype=torch.uint8, device=dev),
+                torch.empty(S, dtype=torch.int32, device=dev))
+        state = {"t": 0}
+
+        def step():
+            t = state["t"]
+            if t == T:
+                B.pr_ctx_reset(ctx, stream=stream)
+                t = 0
+            B.pr_decode_step(ctx, x_all[t * S:(t + 1) * S], slot, ch_all[t * S:(t + 1) * S], eos[t],
+                             w, tr.b, tr.tau, *outs, stream=stream)
+            state["t"] = t + 1
+
+        rows_per_step = S
+        bytes_per_step = S * (wl.vocab * 2 + 4 + 1 + 4) + S * 4
+        desc = ("decode steps: 256 live slots x 1,000 steps (%d rows resident), V=%d bf16, "
+                "lengths U{64..1000}, one pr_decode_step per step" % (T * S, wl.vocab))
+        dtype = "bf16"
+    else:
+        wl = W.make(name)
+        copies = 1
+        if name == "tiny":
+            copies = 8  # 8 x 45 MB rotated: more than L2 between reuses
+        xs, chs = [], []
+        for c in range(copies):
+            x = torch.empty(wl.n_rows, wl.vocab, dtype=wl.torch_dtype, device=dev)
+            ch = torch.empty(wl.n_rows, dtype=torch.int32, device=dev)
+            W.rows(wl, 0, wl.n_rows, device=dev, out=x, chosen_out=ch)
+            xs.append(x)
+            chs.append(ch)
+        off = torch.from_numpy(wl.offsets).to(dev)
+        w = torch.from_numpy(wl.w).to(dev)
+        ctx = B.pr_ctx_create(local, max_rows=wl.n_rows, max_requests=wl.n_req)
+        outs = (torch.empty(wl.n_req, device=dev), torch.empty(wl.n_req, dtype=torch.uint8, device=dev),
+                torch.empty(wl.n_req, dtype=torch.int32, device=dev))
+        chunk = wl.chunk_rows or wl.n_rows
+        state = {"c": 0}
+
+        def step():
+            c = state["c"] % copies
+            state["c"] += 1
+            for lo in range(0, wl.n_rows, chunk):
+                hi = min(wl.n_rows, lo + chunk)
+                B.pr_route(ctx, xs[c][lo:hi], chs[c][lo:hi], off, w, wl.b, wl.tau, row_base=lo,
+                           score=outs[0], ship=outs[1], req_flags=outs[2], agg=None,
+                           stream=stream, want_agg=False)
+
+        rows_per_step = wl.n_rows
+        bytes_per_step = algorithmic_bytes(wl)
+        desc = {"tiny": "tiny: 8 requests, T~U{16..64} (%d rows), V=%d fp32, 8 rotated copies",
+                "ragged": "ragged: 1,024 requests, lognormal lengths (%d rows), V=%d bf16, "
+                          "8,192-row chunks",
+                "wide": "wide vocabulary: 512 requests, T~U{64..512} (%d rows), V=%d fp32 "
+                        "Student-t(3), one launch"}[name] % (wl.n_rows, wl.vocab)
+        dtype = "f32" if wl.dtype == "f32" else "bf16"
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    torch.cuda.synchronize(dev)
+    K = args.steps
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    launches0 = B.launch_count()
+    ev0.record(stream)
+    for _ in range(K):
+        step()
+    ev1.record(stream)
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    launches = B.launch_count() - launches0
+    ms = reduce_max(ev0.elapsed_time(ev1), world, dev) / K
+    peaks_file = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    peak = float(json.load(open(peaks_file))["hbm_gbs"]) if os.path.exists(peaks_file) else 6800.0
+    achieved = bytes_per_step / (ms / 1e3) / 1e9
+    if rank == 0:
+        print(json.dumps({
+            "metric": "verified tokens/sec (%s workload)" % name,
+            "value": rows_per_step * world / (ms / 1e3), "unit": UNIT, "n_gpus": world, "steps": K,
+            "warmup": max(3, args.warmup), "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": dtype, "data": "synthetic",
+            "config": {"workload": desc, "rows_per_step_per_gpu": rows_per_step},
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                         "frac": achieved / peak, "traffic": None,
+                         "algorithmic_bytes_per_step": bytes_per_step},
+            "gpu_launches": launches}))
+    B.pr_ctx_destroy(ctx)
+    return 0
+
 
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=200)
-    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--workload", default=WORKLOAD,
+                    choices=["full", "tiny", "ragged", "wide", "decode"],
+                    help="full (default, the headline line) or one of the other workloads")
     ap.add_argument("--requests", type=int, default=0,
                     help="profiling only: the first N requests of the workload")
     ap.add_argument("--skip-host", action="store_true",
@@ -374,6 +494,8 @@ def main():
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)
+    if args.workload != WORKLOAD:
+        return run_other_workload(args)
     return run_gb300(args)
 
 

@@ -131,12 +131,14 @@ pr_status ws_setup(pr_ctx* c, pr_dtype dt, int mode, bool aligned, int* bps) {
   return PR_OK;
 }
 
-// CTAs per row: the forced option, or enough to put two waves of CTAs on the GPU
+// CTAs per row: the forced option, or the largest split (<= 8) whose CTAs
+// still fit in one wave of the cluster kernel; batches too large for that
+// (more rows than half a wave) go to the persistent kernel (split 1).
 int choose_split(pr_ctx* c, pr_dtype dt, int mode, int64_t n_rows) {
   if (c->split == 1 || c->split == 2 || c->split == 4 || c->split == 8) return c->split;
   const int64_t slots = (int64_t)c->num_sms * blocks_per_sm(c, dt, mode);
   int s = 1;
-  while (s < prk::MAXC && n_rows * s < 2 * slots) s <<= 1;
+  while (s < prk::MAXC && n_rows * (s * 2) <= slots) s <<= 1;
   return s;
 }
 
