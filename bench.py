@@ -35,7 +35,7 @@ WORKLOAD = "full"
 METRIC = "verified tokens/sec at V=151,936 bf16 and achieved HBM GB/s vs peak (1xGB300)"
 UNIT = "tokens/s"
 KERNEL_FILES = ("pr_device.cuh", "pr_kernels.cuh", "pro_router.cu")
-PROFILE = os.path.join(ROOT, "profiles", "verify_rows_bf16_full_response.md")
+PROFILE = os.path.join(ROOT, "profiles", "verify_rows_ws_bf16_full_response.md")
 
 
 def dist_env():
@@ -264,8 +264,8 @@ def run_gb300(args):
     total_ms = ev[0].elapsed_time(ev[K])
     total_ms = reduce_max(total_ms, world, dev)
     clocks = sampler.summary(t_wall0, t_wall1)
+    sampler.stop()  # nvidia-smi polling is not part of the host-memory leg
     if args.skip_host:
-        sampler.stop()
         if rank == 0:
             print(json.dumps({"profiling_case": True, "rows": wl.n_rows, "steps": K,
                               "ms_per_step": total_ms / K, "gpu_launches": launches}))
@@ -294,7 +294,6 @@ def run_gb300(args):
         e2e_step()
     barrier(world)
     e2e_s = reduce_max(time.perf_counter() - t0, world, dev)
-    sampler.stop()
 
     h2d = hx.numel() * hx.element_size() + hc.numel() * 4 + hoff.numel() * 8 + hw.numel() * 4
     d2h = hs.numel() * 4 + hsh.numel() + hf.numel() * 4
@@ -340,7 +339,7 @@ def run_gb300(args):
                        "parallelism": "dp%d (independent batches)" % world},
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak, "traffic": profiled_traffic(),
-                         "kernel": "verify_rows<bf16, route>", "peak_source": peak_src,
+                         "kernel": "verify_rows_ws<bf16, route>", "peak_source": peak_src,
                          "algorithmic_bytes_per_launch": abytes,
                          "avg_launch_ms": avg_launch_ms},
             "cpu_baseline": {"value": rows / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
