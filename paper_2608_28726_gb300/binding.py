@@ -20,7 +20,7 @@ PR_DTYPE_F32, PR_DTYPE_BF16 = 0, 1
 PR_FLAG_NONFINITE, PR_FLAG_BAD_CHOSEN, PR_FLAG_EMPTY_REQ = 1, 2, 4
 PR_FLAG_BAD_OFFSETS, PR_FLAG_BAD_SLOT = 8, 16
 PR_NFEAT, PR_NAGG, PR_MAX_TOPK = 8, 11, 32
-PR_OPT_TOPK, PR_OPT_TOPK_RENORM, PR_OPT_SPLIT = 0, 1, 2
+PR_OPT_TOPK, PR_OPT_TOPK_RENORM, PR_OPT_SPLIT, PR_OPT_OVERLAP = 0, 1, 2, 3
 PR_NOALLOC_MAX_ROWS, PR_NOALLOC_MAX_REQUESTS = 16384, 1024
 
 # every symbol include/pro_router.h declares

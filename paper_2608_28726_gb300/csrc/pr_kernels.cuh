@@ -121,6 +121,33 @@ __device__ __forceinline__ int32_t find_request(const int64_t* off, int32_t n_re
   return (a <= gr && gr < c) ? (int32_t)lo : -1;
 }
 
+// Route mode: the results of empty requests touching this launch's row range
+// and of requests whose offsets are inconsistent (requests start, start +
+// stride, ...).  Written by every launch; idempotent.
+__device__ __forceinline__ void route_special_requests(const Args& a, int64_t start,
+                                                       int64_t stride) {
+  for (int64_t r = start; r < a.n_req; r += stride) {
+    const int64_t lo = a.offsets[r], hi = a.offsets[r + 1];
+    if (lo < 0 || hi < lo || hi > a.max_rows) {
+      write_special(r, NAN, FLAG_BAD_OFFSETS, a.agg, a.score, a.ship, a.req_flags);
+      atomicOr(a.ctx_flags, FLAG_BAD_OFFSETS);
+    } else if (lo == hi && lo >= a.row_base && lo <= a.row_base + a.n_rows) {
+      write_special(r, 0.f, FLAG_EMPTY_REQ, a.agg, a.score, a.ship, a.req_flags);
+    }
+  }
+}
+
+// Programmatic dependent launch.  A launch made with the overlap option may
+// start while the previous kernel on its stream is still running: every CTA
+// allows its own dependents at once, reads only its inputs before
+// pdl_wait(), and waits there before its first global write and before any
+// read of context state (counters, decode slots) the previous launch may
+// still update.  Without the option both are no-ops.
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // ---- cluster helpers ------------------------------------------------------------------
 
 __device__ __forceinline__ void cluster_sync_all() {
@@ -404,19 +431,7 @@ __global__ void __launch_bounds__(NT) verify_rows(const Args a) {
   asm("mov.u32 %0, %%clusterid.x;" : "=r"(cid));
   const int64_t row = cid;
 
-  // Route mode: every launch writes the results of empty requests touching its
-  // row range and of requests whose offsets are inconsistent.
-  if (MODE == MODE_ROUTE) {
-    for (int64_t r = (int64_t)blockIdx.x * NT + tid; r < a.n_req; r += (int64_t)gridDim.x * NT) {
-      const int64_t lo = a.offsets[r], hi = a.offsets[r + 1];
-      if (lo < 0 || hi < lo || hi > a.max_rows) {
-        write_special(r, NAN, FLAG_BAD_OFFSETS, a.agg, a.score, a.ship, a.req_flags);
-        atomicOr(a.ctx_flags, FLAG_BAD_OFFSETS);
-      } else if (lo == hi && lo >= a.row_base && lo <= a.row_base + a.n_rows) {
-        write_special(r, 0.f, FLAG_EMPTY_REQ, a.agg, a.score, a.ship, a.req_flags);
-      }
-    }
-  }
+  pdl_trigger();  // a dependent launch may start streaming while this one finishes
 
   const char* rowp = reinterpret_cast<const char*>(a.logits) + row * a.row_stride * (int64_t)sizeof(T);
   const uint4* vp = reinterpret_cast<const uint4*>(rowp);
@@ -691,6 +706,11 @@ __global__ void __launch_bounds__(NT) verify_rows(const Args a) {
   if (warp != 0) return;
 
   const RowPre pre = load_pre<T, MODE>(a, row, rowp, lane);
+  pdl_wait();
+  if (MODE == MODE_ROUTE) {
+    const int64_t nclusters = gridDim.x / C;
+    route_special_requests(a, (int64_t)cid * 32 + lane, nclusters * 32);
+  }
   row_finish<T, MODE>(a, row, m, S, U, bad, E, pre, lane);
 }
 
@@ -1014,19 +1034,7 @@ __global__ void __launch_bounds__(NT_WS, 3) verify_rows_ws(const Args a) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int64_t G = gridDim.x;
 
-  // Route mode: results of empty requests touching this launch's row range and
-  // of requests whose offsets are inconsistent.
-  if (MODE == MODE_ROUTE) {
-    for (int64_t r = (int64_t)blockIdx.x * NT_WS + tid; r < a.n_req; r += G * NT_WS) {
-      const int64_t lo = a.offsets[r], hi = a.offsets[r + 1];
-      if (lo < 0 || hi < lo || hi > a.max_rows) {
-        write_special(r, NAN, FLAG_BAD_OFFSETS, a.agg, a.score, a.ship, a.req_flags);
-        atomicOr(a.ctx_flags, FLAG_BAD_OFFSETS);
-      } else if (lo == hi && lo >= a.row_base && lo <= a.row_base + a.n_rows) {
-        write_special(r, 0.f, FLAG_EMPTY_REQ, a.agg, a.score, a.ship, a.req_flags);
-      }
-    }
-  }
+  pdl_trigger();  // a dependent launch may start streaming while this one finishes
 
   const RowGeom geo(a.vocab, Tr::VEC);
 
@@ -1039,6 +1047,8 @@ __global__ void __launch_bounds__(NT_WS, 3) verify_rows_ws(const Args a) {
     int i = 0;
     int64_t row = blockIdx.x;
     RowPre pre = load_pre<T, MODE>(a, row, rowp_of(row), lane);
+    pdl_wait();
+    if (MODE == MODE_ROUTE) route_special_requests(a, (int64_t)blockIdx.x * 32 + lane, G * 32);
     for (; row < a.n_rows; row += G, ++i) {
       const int b = i & 1;
       named_bar_sync(BAR_FULL + b, NT_WS);

@@ -40,7 +40,7 @@ struct pr_ctx {
   int64_t max_rows = 0;
   int32_t max_requests = 0;
   // options
-  int32_t topk = 20, renorm = 0, split = 0;
+  int32_t topk = 20, renorm = 0, split = 0, overlap = 0;
   // workspace
   float* rec = nullptr;          // [max_rows][8] per-row records of pr_route
   uint32_t* rec_flags = nullptr; // [max_rows]
@@ -151,9 +151,19 @@ pr_status launch_rows(pr_ctx* c, pr_dtype dt, int mode, const prk::Args& a, cuda
     const pr_status s = ws_setup(c, dt, mode, a.aligned != 0, &bps);
     if (s != PR_OK) return s;
     const int64_t grid = std::min<int64_t>(a.n_rows, (int64_t)c->num_sms * bps);
+    cudaLaunchConfig_t cfg;
+    memset(&cfg, 0, sizeof cfg);
+    cfg.gridDim = dim3((unsigned)grid, 1, 1);
+    cfg.blockDim = dim3(prk::NT_WS, 1, 1);
+    cfg.dynamicSmemBytes = sizeof(prk::SmemWS);
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = c->overlap ? 1 : 0;
     void* args[] = {const_cast<prk::Args*>(&a)};
-    PR_CUDA(cudaLaunchKernel(ws_kernel(dt, mode, a.aligned != 0), dim3((unsigned)grid),
-                             dim3(prk::NT_WS), args, sizeof(prk::SmemWS), st));
+    PR_CUDA(cudaLaunchKernelExC(&cfg, ws_kernel(dt, mode, a.aligned != 0), args));
     g_launches.fetch_add(1, std::memory_order_relaxed);
     return PR_OK;
   }
@@ -164,13 +174,22 @@ pr_status launch_rows(pr_ctx* c, pr_dtype dt, int mode, const prk::Args& a, cuda
   cfg.blockDim = dim3(prk::NT, 1, 1);
   cfg.dynamicSmemBytes = 0;
   cfg.stream = st;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = (unsigned)C;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
+  cudaLaunchAttribute attr[2];
+  int na = 0;
+  if (C > 1) {
+    attr[na].id = cudaLaunchAttributeClusterDimension;
+    attr[na].val.clusterDim.x = (unsigned)C;
+    attr[na].val.clusterDim.y = 1;
+    attr[na].val.clusterDim.z = 1;
+    ++na;
+  }
+  if (c->overlap) {
+    attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[na].val.programmaticStreamSerializationAllowed = 1;
+    ++na;
+  }
   cfg.attrs = attr;
-  cfg.numAttrs = C > 1 ? 1 : 0;
+  cfg.numAttrs = na;
   void* args[] = {const_cast<prk::Args*>(&a)};
   PR_CUDA(cudaLaunchKernelExC(&cfg, row_kernel(dt, mode, a.aligned != 0), args));
   g_launches.fetch_add(1, std::memory_order_relaxed);
@@ -338,6 +357,10 @@ pr_status pr_ctx_set_option(pr_ctx* c, int32_t option, int32_t value) {
       if (value != 0 && value != 1 && value != 2 && value != 4 && value != 8)
         return PR_ERR_INVALID_ARG;
       c->split = value;
+      return PR_OK;
+    case PR_OPT_OVERLAP:
+      if (value != 0 && value != 1) return PR_ERR_INVALID_ARG;
+      c->overlap = value;
       return PR_OK;
   }
   return PR_ERR_INVALID_ARG;

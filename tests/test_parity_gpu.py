@@ -462,3 +462,39 @@ def test_decode_bad_slot_flagged(ctx):
     assert B.pr_ctx_flags(ctx, clear=True) & B.PR_FLAG_BAD_SLOT
     assert ship[0].item() == 1 and out[0].item() == 0.5
     B.pr_ctx_reset(ctx)
+
+
+def test_overlap_option_changes_nothing_but_timing(ctx):
+    """With PR_OPT_OVERLAP a call may start while the previous one finishes;
+    back-to-back route calls and decode steps give bit-identical results."""
+    lengths = [40, 0, 75, 3, 150]
+    x, ch, off, w, b = _batch(lengths, 5000, torch.bfloat16, seed=91)
+    dw, doff = torch.from_numpy(w).cuda(), torch.from_numpy(off).cuda()
+    results = {}
+    for overlap in (0, 1):
+        B.pr_ctx_set_option(ctx, B.PR_OPT_OVERLAP, overlap)
+        outs = []
+        for split in (1, 2):  # the persistent kernel and the cluster kernel
+            _set(ctx, split=split)
+            for rep in range(4):
+                outs.append(B.pr_route(ctx, x, ch, doff, dw, b, 0.5))
+        torch.cuda.synchronize()
+        results[overlap] = outs
+    for (a0, a1) in zip(results[0], results[1]):
+        for t0, t1 in zip(a0, a1):
+            assert torch.equal(t0.nan_to_num(5.0), t1.nan_to_num(5.0))
+    # decode: the same trace with and without overlap
+    n_slots, steps = 6, 60
+    rows, eos, reqs, w2, b2 = _small_trace(n_slots, steps, seed=5)
+    ends = {}
+    for overlap in (0, 1):
+        B.pr_ctx_set_option(ctx, B.PR_OPT_OVERLAP, overlap)
+        B.pr_ctx_reset(ctx)
+        ends[overlap] = _decode_run(ctx, rows, n_slots, steps, eos, w2, b2)
+    for k, v in ends[0].items():
+        v1 = ends[1][k]
+        assert v[1:3] == v1[1:3] and np.array_equal(v[3], v1[3], equal_nan=True)
+        assert v[0] == v1[0] or (np.isnan(v[0]) and np.isnan(v1[0]))
+    B.pr_ctx_set_option(ctx, B.PR_OPT_OVERLAP, 0)
+    _set(ctx)
+    B.pr_ctx_reset(ctx)
