@@ -236,3 +236,50 @@ def decode_trace(n_slots: int = 256, n_steps: int = 1000, lo: int = 64, hi: int 
             t += L
     w, b = scorer(seed_host)
     return DecodeTrace(n_slots, n_steps, vocab, "bf16", seed_dev, "full", reqs, eos, w, b)
+
+
+# ---- scorer head weights ---------------------------------------------------------
+
+HEAD_D, HEAD_HEADS, HEAD_DFF, HEAD_DIN = 64, 4, 128, 4
+
+
+def head_param_count(n_layers: int) -> int:
+    per_layer = (3 * HEAD_D * HEAD_D + 3 * HEAD_D + HEAD_D * HEAD_D + HEAD_D + 2 * HEAD_D
+                 + HEAD_DFF * HEAD_D + HEAD_DFF + HEAD_D * HEAD_DFF + HEAD_D + 2 * HEAD_D)
+    return HEAD_D * HEAD_DIN + HEAD_D + n_layers * per_layer + HEAD_D + 1
+
+
+def head_weights(n_layers: int = 2, seed: int = 3001) -> np.ndarray:
+    """Seeded stand-in for the head's trained weights (flat float32, the layout
+    the library documents): matrices N(0, 1/fan_in), biases N(0, 0.02^2),
+    LayerNorm gains 1 + N(0, 0.1^2) and shifts N(0, 0.1^2)."""
+    g = np.random.Generator(np.random.PCG64(seed))
+    D, F, I = HEAD_D, HEAD_DFF, HEAD_DIN
+    parts = []
+
+    def mat(rows, cols):
+        parts.append(g.normal(0.0, 1.0 / np.sqrt(cols), size=rows * cols))
+
+    def vec(n, scale=0.02, base=0.0):
+        parts.append(base + g.normal(0.0, scale, size=n))
+
+    mat(D, I)
+    vec(D)
+    for _ in range(n_layers):
+        mat(3 * D, D)
+        vec(3 * D)
+        mat(D, D)
+        vec(D)
+        vec(D, 0.1, 1.0)
+        vec(D, 0.1)
+        mat(F, D)
+        vec(F)
+        mat(D, F)
+        vec(D)
+        vec(D, 0.1, 1.0)
+        vec(D, 0.1)
+    mat(1, D)
+    vec(1)
+    w = np.concatenate(parts).astype(np.float32)
+    assert w.size == head_param_count(n_layers)
+    return w
