@@ -244,6 +244,51 @@ pr_status pr_decode_step(pr_ctx* ctx, const void* logits, pr_dtype dt, int32_t n
 pr_status pr_state_export(pr_ctx* ctx, void* host_buf, size_t* bytes);
 pr_status pr_state_import(pr_ctx* ctx, const void* host_buf, size_t bytes);
 
+/* ---- transformer scorer head ------------------------------------------------------ */
+
+#define PR_HEAD_D 64          /* model width */
+#define PR_HEAD_HEADS 4       /* attention heads (width 16 each) */
+#define PR_HEAD_FF 128        /* feed-forward width */
+#define PR_HEAD_MAX_LAYERS 8  /* largest number of encoder layers accepted */
+
+/* Number of floats of the head's weights for n_layers encoder layers
+ * (67,329 for 2 layers); -1 if n_layers is outside [1, PR_HEAD_MAX_LAYERS]. */
+int64_t pr_head_param_count(int32_t n_layers);
+
+/*
+ * The paper's learned scorer (Section 3.1) over per-request feature
+ * sequences: for request r the T = offsets[r+1] - offsets[r] rows give
+ * x_t = (l_t, m_t, h_t, rho_t) (record slots LOGP, MAXP, TOPK, RHO of Eq. 3);
+ * h_0 = W_in x_t + b_in + PE(t) with the sinusoidal encoding PE(t)[2i] =
+ * sin(t / 10000^(2i/64)), PE(t)[2i+1] = cos(same), t = 0 .. T-1; n_layers
+ * post-norm transformer encoder layers (4-head self-attention, residual,
+ * LayerNorm; ReLU feed-forward of width 128, residual, LayerNorm; eps 1e-5);
+ * z = w_out . mean_t(h_L) + b_out; score = sigmoid(z); ship = (z >= logit(tau)).
+ *   feat       device float [n_rows][PR_NFEAT], e.g. from pr_token_features
+ *              with offsets (so that rho is filled in)
+ *   row_flags  device uint32 [n_rows] or NULL; a request with a row flagged
+ *              PR_FLAG_NONFINITE or PR_FLAG_BAD_CHOSEN escalates with score NaN
+ *   offsets    device int64 [n_req + 1], non-decreasing for valid requests; a
+ *              request with offsets[r] < 0, offsets[r+1] < offsets[r] or
+ *              offsets[r+1] > n_rows gets score NaN and PR_FLAG_BAD_OFFSETS;
+ *              an empty request gets score 0 and PR_FLAG_EMPTY_REQ
+ *   w          device float [pr_head_param_count(n_layers)], 16-byte aligned,
+ *              in this order (matrices row-major, y = W x + b):
+ *                W_in[64][4] b_in[64]
+ *                per layer: W_qkv[192][64] (rows q, k, v) b_qkv[192]
+ *                  W_o[64][64] b_o[64] g1[64] be1[64] W_1[128][64] b_1[128]
+ *                  W_2[64][128] b_2[64] g2[64] be2[64]
+ *                w_out[64] b_out
+ *   score, ship, req_flags   device [n_req]            (outputs)
+ * One CTA per request; all arithmetic is fp32 in a fixed order.  The context
+ * holds a device scratch of 1 KB per row, allocated (or grown) by the first
+ * call with more rows than before -- that call synchronises the device.
+ */
+pr_status pr_head_score(pr_ctx* ctx, const float* feat, const uint32_t* row_flags,
+                        int64_t n_rows, const int64_t* offsets, int32_t n_req, const float* w,
+                        int32_t n_layers, float tau, float* score, uint8_t* ship,
+                        uint32_t* req_flags, void* stream);
+
 /* ---- verification without allocation ------------------------------------------------- */
 
 #define PR_NOALLOC_MAX_ROWS 16384    /* largest n_rows pr_route_noalloc accepts */

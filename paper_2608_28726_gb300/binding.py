@@ -22,13 +22,14 @@ PR_FLAG_BAD_OFFSETS, PR_FLAG_BAD_SLOT = 8, 16
 PR_NFEAT, PR_NAGG, PR_MAX_TOPK = 8, 11, 32
 PR_OPT_TOPK, PR_OPT_TOPK_RENORM, PR_OPT_SPLIT, PR_OPT_OVERLAP = 0, 1, 2, 3
 PR_NOALLOC_MAX_ROWS, PR_NOALLOC_MAX_REQUESTS = 16384, 1024
+PR_HEAD_D, PR_HEAD_HEADS, PR_HEAD_FF, PR_HEAD_MAX_LAYERS = 64, 4, 128, 8
 
 # every symbol include/pro_router.h declares
 EXPORTS = (
     "pr_ctx_create", "pr_ctx_destroy", "pr_ctx_reset", "pr_ctx_set_option", "pr_ctx_flags",
     "pr_token_features", "pr_aggregate_score", "pr_route", "pr_route_host", "pr_decode_step",
     "pr_state_export", "pr_state_import", "pr_status_string", "pr_last_cuda_error",
-    "pr_launch_count", "pr_route_noalloc",
+    "pr_launch_count", "pr_route_noalloc", "pr_head_param_count", "pr_head_score",
 )
 
 if not os.path.exists(LIB):
@@ -54,6 +55,7 @@ _SIGS = {
                        _P, _P, _P],
     "pr_route_noalloc": [_P, ctypes.c_int, _I64, _I64, _I64, _P, _P, _I32, _P, _F32, _F32, _P, _P,
                          _P, _P, _P],
+    "pr_head_score": [_P, _P, _P, _I64, _P, _I32, _P, _I32, _F32, _P, _P, _P, _P],
     "pr_state_export": [_P, _P, ctypes.POINTER(_SZ)],
     "pr_state_import": [_P, _P, _SZ],
 }
@@ -67,6 +69,8 @@ _lib.pr_last_cuda_error.argtypes = []
 _lib.pr_last_cuda_error.restype = ctypes.c_char_p
 _lib.pr_launch_count.argtypes = []
 _lib.pr_launch_count.restype = ctypes.c_uint64
+_lib.pr_head_param_count.argtypes = [_I32]
+_lib.pr_head_param_count.restype = _I64
 
 
 class PRError(RuntimeError):
@@ -256,3 +260,22 @@ def pr_state_export(ctx) -> bytes:
 def pr_state_import(ctx, state: bytes):
     buf = ctypes.create_string_buffer(state, len(state))
     _check(_lib.pr_state_import(ctx, buf, len(state)), "pr_state_import")
+
+
+# ---- transformer scorer head ------------------------------------------------------------
+
+def pr_head_param_count(n_layers: int) -> int:
+    return int(_lib.pr_head_param_count(int(n_layers)))
+
+
+def pr_head_score(ctx, feat, offsets, w, n_layers: int, tau: float, row_flags=None, score=None,
+                  ship=None, req_flags=None, stream=None):
+    n_req = offsets.numel() - 1
+    dev = feat.device
+    score = torch.empty(n_req, dtype=torch.float32, device=dev) if score is None else score
+    ship = torch.empty(n_req, dtype=torch.uint8, device=dev) if ship is None else ship
+    req_flags = torch.empty(n_req, dtype=torch.int32, device=dev) if req_flags is None else req_flags
+    _check(_lib.pr_head_score(ctx, _ptr(feat), _ptr(row_flags), feat.size(0), _ptr(offsets), n_req,
+                              _ptr(w), int(n_layers), float(tau), _ptr(score), _ptr(ship),
+                              _ptr(req_flags), _stream(stream)), "pr_head_score")
+    return score, ship, req_flags

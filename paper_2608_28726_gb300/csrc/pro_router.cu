@@ -11,6 +11,7 @@
 #include <new>
 
 #include "pr_kernels.cuh"
+#include "pr_head.cuh"
 #include "pro_router.h"
 
 namespace {
@@ -65,6 +66,10 @@ struct pr_ctx {
   int bps[2][3] = {{0, 0, 0}, {0, 0, 0}};
   // persistent kernel: CTAs per SM per (dtype, mode, aligned); 0 = not set up yet
   int ws_bps[2][3][2] = {};
+  // scorer head: activation scratch (rows x prk::HSCR floats), grown on demand
+  float* head_scr = nullptr;
+  int64_t head_scr_rows = 0;
+  bool head_ready = false;
 };
 
 namespace {
@@ -326,6 +331,7 @@ pr_status pr_ctx_destroy(pr_ctx* c) {
   cudaFree(c->h_out);
   cudaFree(c->h_ship_dev);
   cudaFree(c->h_flags_dev);
+  cudaFree(c->head_scr);
   if (c->copy_stream) cudaStreamDestroy(c->copy_stream);
   delete c;
   return PR_OK;
@@ -530,6 +536,64 @@ pr_status pr_state_import(pr_ctx* c, const void* host_buf, size_t bytes) {
   PR_CUDA(cudaDeviceSynchronize());
   if (body) PR_CUDA(cudaMemcpy(c->acc, static_cast<const char*>(host_buf) + sizeof hdr, body,
                                cudaMemcpyHostToDevice));
+  return PR_OK;
+}
+
+int64_t pr_head_param_count(int32_t n_layers) {
+  if (n_layers < 1 || n_layers > prk::HMAXL) return -1;
+  return prk::head_param_count(n_layers);
+}
+
+pr_status pr_head_score(pr_ctx* c, const float* feat, const uint32_t* row_flags, int64_t n_rows,
+                        const int64_t* offsets, int32_t n_req, const float* w, int32_t n_layers,
+                        float tau, float* score, uint8_t* ship, uint32_t* req_flags,
+                        void* stream) {
+  if (!c || n_req < 0 || n_rows < 0) return PR_ERR_INVALID_ARG;
+  if (n_layers < 1 || n_layers > prk::HMAXL) return PR_ERR_INVALID_ARG;
+  if (n_rows > ((int64_t)1 << 23)) return PR_ERR_INVALID_ARG;  // int row arithmetic per request
+  if (n_req == 0) return PR_OK;
+  if (!offsets || !w || !score || !ship || !req_flags) return PR_ERR_INVALID_ARG;
+  if (n_rows > 0 && !feat) return PR_ERR_INVALID_ARG;
+  if (!aligned16(w)) return PR_ERR_INVALID_ARG;
+  pr_status st = set_device(c);
+  if (st != PR_OK) return st;
+  if (!c->head_ready) {
+    PR_CUDA(cudaFuncSetAttribute(prk::head_requests, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)sizeof(prk::HeadSmem)));
+    c->head_ready = true;
+  }
+  if (n_rows > c->head_scr_rows) {
+    // grow: wait for the kernels that may still use the old scratch
+    PR_CUDA(cudaDeviceSynchronize());
+    cudaFree(c->head_scr);
+    c->head_scr = nullptr;
+    c->head_scr_rows = 0;
+    if (cudaMalloc(&c->head_scr, (size_t)n_rows * prk::HSCR * sizeof(float)) != cudaSuccess) {
+      cudaGetLastError();
+      c->head_scr = nullptr;
+      return PR_ERR_NO_MEMORY;
+    }
+    c->head_scr_rows = n_rows;
+  }
+  prk::HeadArgs a;
+  memset(&a, 0, sizeof a);
+  a.feat = feat;
+  a.row_flags = row_flags;
+  a.n_rows = n_rows;
+  a.offsets = offsets;
+  a.n_req = n_req;
+  a.w = w;
+  a.n_layers = n_layers;
+  a.zthr = zthreshold(tau);
+  a.scratch = c->head_scr;
+  a.score = score;
+  a.ship = ship;
+  a.req_flags = req_flags;
+  a.ctx_flags = c->flags;
+  prk::head_requests<<<(unsigned)n_req, prk::NT, sizeof(prk::HeadSmem),
+                       reinterpret_cast<cudaStream_t>(stream)>>>(a);
+  PR_CUDA(cudaGetLastError());
+  g_launches.fetch_add(1, std::memory_order_relaxed);
   return PR_OK;
 }
 

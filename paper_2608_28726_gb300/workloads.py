@@ -283,3 +283,28 @@ def head_weights(n_layers: int = 2, seed: int = 3001) -> np.ndarray:
     w = np.concatenate(parts).astype(np.float32)
     assert w.size == head_param_count(n_layers)
     return w
+
+
+def head_features(lengths, seed: int = 4001) -> tuple[np.ndarray, np.ndarray]:
+    """Seeded row records for the scorer head: (feat float32 [n_rows][8], offsets).
+
+    Slot values follow the verifier's record layout: m ~ U(0.02, 1); the
+    emitted token is the top one on half of the rows (l = log m), otherwise
+    l = log m - Exp(mean 2); h ~ -U(0, ln 20); rho = t / T with t 1-based.  The
+    slots the head does not read (margin, entropy, LSE, x1) hold N(0, 5^2)
+    noise so that reading a wrong slot shows up.
+    """
+    lengths = np.asarray(lengths, np.int64)
+    offsets = np.concatenate([[0], np.cumsum(lengths)]).astype(np.int64)
+    n = int(offsets[-1])
+    g = np.random.Generator(np.random.PCG64(seed))
+    feat = g.normal(0.0, 5.0, size=(n, 8))
+    m = g.uniform(0.02, 1.0, size=n)
+    top = g.random(n) < 0.5
+    feat[:, 0] = np.log(m) - np.where(top, 0.0, g.exponential(2.0, size=n))
+    feat[:, 1] = m
+    feat[:, 4] = -g.uniform(0.0, np.log(20.0), size=n)
+    for r in range(lengths.size):
+        T = int(lengths[r])
+        feat[offsets[r]:offsets[r + 1], 5] = np.arange(1, T + 1) / max(T, 1)
+    return feat.astype(np.float32), offsets

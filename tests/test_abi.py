@@ -80,3 +80,20 @@ def test_no_gpu_means_no_context(lib):
     h = P()
     assert lib.pr_ctx_create(ctypes.byref(h), 0, 16, 4) == -1
     assert not h.value
+
+
+def test_head_parameter_count_matches_the_oracle_layout(lib):
+    """The library's weight count for the scorer head is the oracle's layout size."""
+    from oracle import head
+    lib.pr_head_param_count.argtypes = [ctypes.c_int32]
+    lib.pr_head_param_count.restype = ctypes.c_int64
+    assert lib.pr_head_param_count(2) == 67329 == head.n_params(2)
+    for n in (1, 4, 8):
+        assert lib.pr_head_param_count(n) == head.n_params(n)
+    assert lib.pr_head_param_count(0) == -1
+    assert lib.pr_head_param_count(9) == -1
+    P = ctypes.c_void_p
+    lib.pr_head_score.argtypes = [P, P, P, ctypes.c_int64, P, ctypes.c_int32, P, ctypes.c_int32,
+                                  ctypes.c_float, P, P, P, P]
+    assert lib.pr_head_score(None, None, None, 0, None, 1, None, 2, 0.5, None, None, None,
+                             None) == -1
