@@ -510,6 +510,220 @@ def run_other_workload(args):
     return 0
 
 
+HEAD_FILES = ("pr_device.cuh", "pr_head.cuh", "pr_head_api.cu")
+HEAD_PROFILE = os.path.join(ROOT, "profiles", "head_attn_f32_full_response.md")
+# fp32 CUDA-core peak: 152 SMs x 128 FMA lanes x 2 flop x 2,070 MHz (maximum SM clock)
+FP32_PEAK_TFLOPS = 152 * 128 * 2 * 2.070e9 / 1e12
+
+
+def head_flops(lengths, n_layers: int):
+    """Algorithmic flops of the scorer head: per layer and token the QKV,
+    output, and two feed-forward projections (2 x 64 x (192 + 64 + 128 + 128)),
+    per layer, request and head the scores and the weighted values
+    (2 x 2 x 16 x T^2, four heads); the embedding and pooling are left out.
+    Returns (whole step, one attention launch)."""
+    T = np.asarray(lengths, np.float64)
+    attn = float(4 * 2 * 2 * 16 * np.sum(T * T))
+    rows = float(2 * 64 * (3 * 64 + 64 + 2 * 128) * np.sum(T))
+    return n_layers * (rows + attn), attn
+
+
+def head_oracle_sample(req_hi: int, n_layers: int):
+    """The float64 head oracle on requests 0 .. req_hi - 1 of the head workload,
+    in a child process with one BLAS / OpenMP thread.  Returns (seconds,
+    scores, ship)."""
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1")
+    out = subprocess.run([sys.executable, os.path.abspath(__file__), "--head-oracle-sample",
+                          str(req_hi), "--head-layers", str(n_layers)],
+                         env=env, capture_output=True, text=True, check=True)
+    d = json.loads(out.stdout.strip().splitlines()[-1])
+    return d["seconds"], np.asarray(d["score"], np.float64), np.asarray(d["ship"], np.uint8)
+
+
+def head_oracle_child(req_hi: int, n_layers: int):
+    from oracle import head as ohead
+    wl = W.make(WORKLOAD)
+    feat_h, offsets = W.head_features(wl.lengths, seed=4001)
+    w_h = W.head_weights(n_layers)
+    hi = int(offsets[req_hi])
+    t0 = time.perf_counter()
+    so, po, _ = ohead.head_score(feat_h[:hi].astype(np.float64), np.zeros(hi, np.uint32),
+                                 offsets[:req_hi + 1], w_h.astype(np.float64), n_layers, wl.tau)
+    dt = time.perf_counter() - t0
+    print(json.dumps({"seconds": dt, "score": so.tolist(), "ship": po.tolist()}))
+    return 0
+
+
+def run_head_workload(args):
+    """The transformer scorer head (2 layers) on the full-response request
+    layout: 64 requests, T ~ U{32..256}, seeded feature records resident in HBM;
+    the activations fit in L2, so L2 is flushed between timed steps."""
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", init_method="env://")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    from paper_2608_28726_gb300 import build as prbuild
+    prbuild.build()
+    from paper_2608_28726_gb300 import binding as B
+    n_layers = 2
+    wl = W.make(WORKLOAD)
+    lengths = wl.lengths
+    feat_h, offsets = W.head_features(lengths, seed=4001)
+    w_h = W.head_weights(n_layers)
+    feat = torch.from_numpy(feat_h).to(dev)
+    off = torch.from_numpy(offsets).to(dev)
+    w = torch.from_numpy(w_h).to(dev)
+    n_req, n_rows = len(lengths), int(offsets[-1])
+    ctx = B.pr_ctx_create(local, max_rows=0, max_requests=1)
+    stream = torch.cuda.current_stream(dev)
+    score = torch.empty(n_req, device=dev)
+    ship = torch.empty(n_req, dtype=torch.uint8, device=dev)
+    rflags = torch.empty(n_req, dtype=torch.int32, device=dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)  # 256 MB > L2
+
+    def step():
+        B.pr_head_score(ctx, feat, off, w, n_layers, wl.tau, score=score, ship=ship,
+                        req_flags=rflags, stream=stream)
+
+    K = args.steps
+    sampler = ClockSampler(local)
+    sampler.start()
+
+    def timed(timing: int):
+        B.pr_ctx_set_option(ctx, B.PR_OPT_TIMING, timing)
+        for _ in range(max(3, args.warmup)):
+            step()
+        torch.cuda.synchronize(dev)
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(K)]
+        kernel_ms = []
+        barrier(world)
+        torch.cuda.synchronize(dev)
+        n0 = B.launch_count()
+        for i in range(K):
+            flush.zero_()
+            ev[i][0].record(stream)
+            step()
+            ev[i][1].record(stream)
+            if timing:
+                kernel_ms.append(B.pr_ctx_kernel_times(ctx))
+        torch.cuda.synchronize(dev)
+        barrier(world)
+        total = sum(a.elapsed_time(b) for a, b in ev)
+        return reduce_max(total, world, dev) / K, B.launch_count() - n0, kernel_ms
+
+    t_wall0 = time.time()
+    ms, launches, _ = timed(0)
+    t_wall1 = time.time()
+    iso_ms, _, kernel_ms = timed(1)
+    B.pr_ctx_set_option(ctx, B.PR_OPT_TIMING, 0)
+    clocks = sampler.summary(t_wall0, t_wall1)
+    sampler.stop()
+    attn_idx = [2 + 2 * l for l in range(n_layers)]
+    attn_ms = float(np.mean([k[i] for k in kernel_ms for i in attn_idx]))
+    per_kernel = np.mean(np.asarray(kernel_ms), axis=0).tolist()
+
+    # end to end through the public API: features and offsets from pinned host
+    # memory, scores, ship bits and flags back to pinned host memory
+    hf, ho = torch.from_numpy(feat_h).pin_memory(), torch.from_numpy(offsets).pin_memory()
+    hs = torch.empty(n_req).pin_memory()
+    hsh = torch.empty(n_req, dtype=torch.uint8).pin_memory()
+    hfl = torch.empty(n_req, dtype=torch.int32).pin_memory()
+    dfeat, doff = torch.empty_like(feat), torch.empty_like(off)
+
+    def e2e_step():
+        dfeat.copy_(hf, non_blocking=True)
+        doff.copy_(ho, non_blocking=True)
+        B.pr_head_score(ctx, dfeat, doff, w, n_layers, wl.tau, score=score, ship=ship,
+                        req_flags=rflags, stream=stream)
+        hs.copy_(score, non_blocking=True)
+        hsh.copy_(ship, non_blocking=True)
+        hfl.copy_(rflags, non_blocking=True)
+        torch.cuda.synchronize(dev)
+
+    e2e_step()
+    e2e_steps = max(3, min(K, 50))
+    barrier(world)
+    t0 = time.perf_counter()
+    for _ in range(e2e_steps):
+        e2e_step()
+    barrier(world)
+    e2e_s = reduce_max(time.perf_counter() - t0, world, dev)
+    h2d = hf.numel() * 4 + ho.numel() * 8
+    d2h = n_req * (4 + 1 + 4)
+
+    step_flops, attn_flops = head_flops(lengths, n_layers)
+    achieved = attn_flops / (attn_ms / 1e3) / 1e12
+    if rank == 0:
+        req_hi = n_req  # the whole workload: under a second of oracle time
+        lo, hi = 0, int(offsets[req_hi])
+        dt, so, po = head_oracle_sample(req_hi, n_layers)
+        cores = 1
+        g = score[:req_hi].cpu().numpy().astype(np.float64)
+        ok = bool(np.all(np.abs(g - so) <= 1e-5) and
+                  np.all((ship[:req_hi].cpu().numpy() == po) | (np.abs(so - wl.tau) < 1e-6)))
+        print(json.dumps({
+            "metric": "scored tokens/sec (transformer scorer head, %d layers, 64-request "
+                      "full-response layout)" % n_layers,
+            "value": n_rows * world / (ms / 1e3), "unit": UNIT, "n_gpus": world, "steps": K,
+            "warmup": max(3, args.warmup), "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": {"workload": "scorer head: %d requests, T~U{32..256} (%d rows), seeded "
+                                   "feature records, seeded weights (67,329 floats)" % (
+                                       n_req, n_rows),
+                       "l2": "256 MB written between timed steps (flush)",
+                       "n_layers": n_layers},
+            "roofline": {"bound": "alu", "achieved": achieved, "peak": FP32_PEAK_TFLOPS,
+                         "unit": "TFLOP/s", "frac": achieved / FP32_PEAK_TFLOPS,
+                         "traffic": profiled_head_traffic(), "kernel": "head_attn",
+                         "peak_source": "derived: 152 SMs x 128 fp32 FMA lanes x 2 x 2.07 GHz",
+                         "algorithmic_flops_per_launch": attn_flops,
+                         "avg_launch_ms": attn_ms,
+                         "step_flops": step_flops,
+                         "step_tflops": step_flops / (ms / 1e3) / 1e12,
+                         "isolated_kernel_ms": per_kernel,
+                         "isolated_step_ms": iso_ms},
+            "cpu_baseline": {"value": (hi - lo) / dt, "unit": UNIT, "cores": cores,
+                             "kind": "oracle",
+                             "sample": "requests 0..%d (%d rows), float64 numpy head oracle" % (
+                                 req_hi - 1, hi - lo)},
+            "e2e": {"value": n_rows * world * e2e_steps / e2e_s, "unit": UNIT,
+                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                    "api": "pr_head_score with host copies of features, offsets and results"},
+            "gpu_launches": launches,
+            "clocks": clocks,
+            "parity": {"requests_checked": req_hi, "ok": ok},
+        }))
+    B.pr_ctx_destroy(ctx)
+    return 0
+
+
+def profiled_head_traffic():
+    """DRAM bytes per head_attn launch from the committed ncu summary, if taken on
+    the current head source (else None)."""
+    try:
+        text = open(HEAD_PROFILE).read()
+    except OSError:
+        return None
+    vals = {}
+    for line in text.splitlines():
+        if ":" in line and line.strip().startswith("- "):
+            k, v = line.strip()[2:].split(":", 1)
+            vals[k.strip()] = v.strip().strip("`")
+    h = hashlib.sha256()
+    for f in HEAD_FILES:
+        with open(os.path.join(ROOT, "paper_2608_28726_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    if vals.get("kernel_source_sha") != h.hexdigest()[:16]:
+        return None
+    try:
+        return int(vals["dram_bytes_per_launch"])
+    except (KeyError, ValueError):
+        return None
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -517,15 +731,22 @@ def main():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--workload", default=WORKLOAD,
-                    choices=["full", "tiny", "ragged", "wide", "decode"],
-                    help="full (default, the headline line) or one of the other workloads")
+                    choices=["full", "tiny", "ragged", "wide", "decode", "head"],
+                    help="full (default, the headline line), one of the other verifier "
+                         "workloads, or head (the transformer scorer head)")
     ap.add_argument("--requests", type=int, default=0,
                     help="profiling only: the first N requests of the workload")
     ap.add_argument("--skip-host", action="store_true",
                     help="profiling only: skip the host-memory and oracle legs")
+    ap.add_argument("--head-oracle-sample", type=int, default=0, help=argparse.SUPPRESS)
+    ap.add_argument("--head-layers", type=int, default=2, help=argparse.SUPPRESS)
     args = ap.parse_args()
+    if args.head_oracle_sample:
+        return head_oracle_child(args.head_oracle_sample, args.head_layers)
     if args.impl == "reference":
         return run_reference(args)
+    if args.workload == "head":
+        return run_head_workload(args)
     if args.workload != WORKLOAD:
         return run_other_workload(args)
     return run_gb300(args)

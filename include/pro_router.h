@@ -107,6 +107,9 @@ typedef enum { PR_DTYPE_F32 = 0, PR_DTYPE_BF16 = 1 } pr_dtype;
                                 anything.  Only for callers whose inputs are complete before
                                 the preceding kernel starts (e.g. back-to-back verifier calls
                                 on resident logits).  Default 0. */
+#define PR_OPT_TIMING 4      /* 1: calls that launch several kernels (pr_head_score) record a CUDA
+                                event after each kernel, for pr_ctx_kernel_times; the kernels
+                                then no longer overlap one another.  Default 0. */
 
 typedef struct pr_ctx pr_ctx;
 
@@ -138,6 +141,15 @@ pr_status pr_ctx_set_option(pr_ctx* ctx, int32_t option, int32_t value);
  * clear.  Synchronises `stream`.  With `clear` != 0 the word is zeroed.
  */
 pr_status pr_ctx_flags(pr_ctx* ctx, void* stream, int32_t clear, uint32_t* flags);
+
+/*
+ * Per-kernel device times (milliseconds, launch order) of the last call made
+ * with PR_OPT_TIMING = 1: for pr_head_score the embedding, the first QKV
+ * projection, then per layer the attention and the row-local block, then the
+ * pool.  Waits for the call's last event.  Writes min(count, cap) values to
+ * `ms` and the count to *n (0 if no timed call was made).
+ */
+pr_status pr_ctx_kernel_times(pr_ctx* ctx, float* ms, int32_t cap, int32_t* n);
 
 /* ---- the three verifier calls ----------------------------------------------- */
 
@@ -264,8 +276,8 @@ int64_t pr_head_param_count(int32_t n_layers);
  * post-norm transformer encoder layers (4-head self-attention, residual,
  * LayerNorm; ReLU feed-forward of width 128, residual, LayerNorm; eps 1e-5);
  * z = w_out . mean_t(h_L) + b_out; score = sigmoid(z); ship = (z >= logit(tau)).
- *   feat       device float [n_rows][PR_NFEAT], e.g. from pr_token_features
- *              with offsets (so that rho is filled in)
+ *   feat       device float [n_rows][PR_NFEAT], 16-byte aligned, e.g. from
+ *              pr_token_features with offsets (so that rho is filled in)
  *   row_flags  device uint32 [n_rows] or NULL; a request with a row flagged
  *              PR_FLAG_NONFINITE or PR_FLAG_BAD_CHOSEN escalates with score NaN
  *   offsets    device int64 [n_req + 1], non-decreasing for valid requests; a
@@ -280,9 +292,11 @@ int64_t pr_head_param_count(int32_t n_layers);
  *                  W_2[64][128] b_2[64] g2[64] be2[64]
  *                w_out[64] b_out
  *   score, ship, req_flags   device [n_req]            (outputs)
- * One CTA per request; all arithmetic is fp32 in a fixed order.  The context
- * holds a device scratch of 1 KB per row, allocated (or grown) by the first
- * call with more rows than before -- that call synchronises the device.
+ * The batch runs layer by layer in 2 n_layers + 3 launches on `stream`; all
+ * arithmetic is fp32 in a fixed order, so results are bit-reproducible.  The
+ * context holds a device scratch of 1 KB per row, allocated (or grown) by the
+ * first call with more rows than before -- that call synchronises the device;
+ * calls on different streams must not overlap (they share that scratch).
  */
 pr_status pr_head_score(pr_ctx* ctx, const float* feat, const uint32_t* row_flags,
                         int64_t n_rows, const int64_t* offsets, int32_t n_req, const float* w,

@@ -20,7 +20,7 @@ PR_DTYPE_F32, PR_DTYPE_BF16 = 0, 1
 PR_FLAG_NONFINITE, PR_FLAG_BAD_CHOSEN, PR_FLAG_EMPTY_REQ = 1, 2, 4
 PR_FLAG_BAD_OFFSETS, PR_FLAG_BAD_SLOT = 8, 16
 PR_NFEAT, PR_NAGG, PR_MAX_TOPK = 8, 11, 32
-PR_OPT_TOPK, PR_OPT_TOPK_RENORM, PR_OPT_SPLIT, PR_OPT_OVERLAP = 0, 1, 2, 3
+PR_OPT_TOPK, PR_OPT_TOPK_RENORM, PR_OPT_SPLIT, PR_OPT_OVERLAP, PR_OPT_TIMING = 0, 1, 2, 3, 4
 PR_NOALLOC_MAX_ROWS, PR_NOALLOC_MAX_REQUESTS = 16384, 1024
 PR_HEAD_D, PR_HEAD_HEADS, PR_HEAD_FF, PR_HEAD_MAX_LAYERS = 64, 4, 128, 8
 
@@ -30,6 +30,7 @@ EXPORTS = (
     "pr_token_features", "pr_aggregate_score", "pr_route", "pr_route_host", "pr_decode_step",
     "pr_state_export", "pr_state_import", "pr_status_string", "pr_last_cuda_error",
     "pr_launch_count", "pr_route_noalloc", "pr_head_param_count", "pr_head_score",
+    "pr_ctx_kernel_times",
 )
 
 if not os.path.exists(LIB):
@@ -55,6 +56,7 @@ _SIGS = {
                        _P, _P, _P],
     "pr_route_noalloc": [_P, ctypes.c_int, _I64, _I64, _I64, _P, _P, _I32, _P, _F32, _F32, _P, _P,
                          _P, _P, _P],
+    "pr_ctx_kernel_times": [_P, _P, _I32, ctypes.POINTER(_I32)],
     "pr_head_score": [_P, _P, _P, _I64, _P, _I32, _P, _I32, _F32, _P, _P, _P, _P],
     "pr_state_export": [_P, _P, ctypes.POINTER(_SZ)],
     "pr_state_import": [_P, _P, _SZ],
@@ -148,6 +150,14 @@ def pr_ctx_reset(ctx, stream=None):
 
 def pr_ctx_set_option(ctx, option: int, value: int):
     _check(_lib.pr_ctx_set_option(ctx, int(option), int(value)), "pr_ctx_set_option")
+
+
+def pr_ctx_kernel_times(ctx, cap: int = 32) -> list:
+    """Per-kernel times (ms) of the last call made with PR_OPT_TIMING = 1."""
+    buf = (ctypes.c_float * cap)()
+    n = _I32(0)
+    _check(_lib.pr_ctx_kernel_times(ctx, buf, cap, ctypes.byref(n)), "pr_ctx_kernel_times")
+    return [float(buf[i]) for i in range(min(n.value, cap))]
 
 
 def pr_ctx_flags(ctx, stream=None, clear: bool = False) -> int:

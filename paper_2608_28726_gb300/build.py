@@ -3,8 +3,9 @@
     python -m paper_2608_28726_gb300.build          # build if sources changed
     python -m paper_2608_28726_gb300.build --force  # rebuild
 
-nvcc cross-compiles without a GPU.  The library links the CUDA runtime
-statically, so it depends only on the driver at run time.
+nvcc cross-compiles without a GPU.  The translation units under csrc/ are
+compiled in parallel and linked into one shared library; it links the CUDA
+runtime statically, so it depends only on the driver at run time.
 """
 from __future__ import annotations
 
@@ -42,16 +43,36 @@ def stale() -> bool:
     return any(os.path.getmtime(s) > t for s in sources())
 
 
+def units() -> list[str]:
+    """Translation units of the library (compiled in parallel, then linked)."""
+    return sorted(os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith(".cu"))
+
+
 def build(force: bool = False, verbose: bool = False) -> str:
     if not force and not stale():
         return LIB
     os.makedirs(OUT_DIR, exist_ok=True)
-    tmp = LIB + ".tmp%d" % os.getpid()
-    cmd = [nvcc(), *ARCH, "-O3", "-lineinfo", "-std=c++17", "-shared", "-Xcompiler", "-fPIC",
-           "-I", INCLUDE, os.path.join(CSRC, "pro_router.cu"), "-o", tmp]
+    tag = ".tmp%d" % os.getpid()
+    flags = [*ARCH, "-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I", INCLUDE]
     if verbose:
-        cmd.insert(1, "-Xptxas=-v")
-    subprocess.check_call(cmd)
+        flags.insert(0, "-Xptxas=-v")
+    objs, procs = [], []
+    for src in units():
+        obj = os.path.join(OUT_DIR, os.path.basename(src)[:-3] + tag + ".o")
+        objs.append(obj)
+        procs.append((src, subprocess.Popen([nvcc(), *flags, "-c", src, "-o", obj])))
+    failed = [src for src, p in procs if p.wait() != 0]
+    if failed:
+        for obj in objs:
+            if os.path.exists(obj):
+                os.remove(obj)
+        raise subprocess.CalledProcessError(1, "nvcc -c " + " ".join(failed))
+    tmp = LIB + tag
+    try:
+        subprocess.check_call([nvcc(), *ARCH, "-shared", *objs, "-o", tmp])
+    finally:
+        for obj in objs:
+            os.remove(obj)
     os.replace(tmp, LIB)
     return LIB
 

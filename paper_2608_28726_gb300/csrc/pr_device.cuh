@@ -371,4 +371,15 @@ struct WarpTopK {
   }
 };
 
+// Programmatic dependent launch.  A launch made with programmatic stream serialization may
+// start while the previous kernel on its stream is still running: every CTA
+// allows its own dependents at once, reads only its inputs before
+// pdl_wait(), and waits there before its first global write and before any
+// read of context state (counters, decode slots) the previous launch may
+// still update.  Without the option both are no-ops.
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 }  // namespace prk

@@ -137,16 +137,6 @@ __device__ __forceinline__ void route_special_requests(const Args& a, int64_t st
   }
 }
 
-// Programmatic dependent launch.  A launch made with the overlap option may
-// start while the previous kernel on its stream is still running: every CTA
-// allows its own dependents at once, reads only its inputs before
-// pdl_wait(), and waits there before its first global write and before any
-// read of context state (counters, decode slots) the previous launch may
-// still update.  Without the option both are no-ops.
-__device__ __forceinline__ void pdl_trigger() {
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-}
-__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
 // ---- cluster helpers ------------------------------------------------------------------
 
@@ -524,7 +514,7 @@ __global__ void __launch_bounds__(NT) verify_rows(const Args a) {
   }
 
   // ---- theta1: the kc-th largest per-thread maximum (a lower bound of the kc-th element)
-  const int kc = a.kc, K = a.topk;
+  const int kc = a.kc;
   sm.wl[warp][lane] = warp_sort_desc<uint32_t>(ord(thr_max), lane);
   block_reduce_state(sm, m, S, U, bad, warp, lane);  // ends with a __syncthreads
   if (warp == 0) {

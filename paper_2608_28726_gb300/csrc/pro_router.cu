@@ -10,11 +10,10 @@
 #include <cstring>
 #include <new>
 
+#include "pr_ctx.h"
 #include "pr_kernels.cuh"
-#include "pr_head.cuh"
-#include "pro_router.h"
 
-namespace {
+namespace prh {
 
 thread_local char g_cuda_err[256] = "";
 std::atomic<uint64_t> g_launches{0};
@@ -24,53 +23,46 @@ pr_status cuda_fail(cudaError_t e, const char* what) {
   return PR_ERR_CUDA;
 }
 
-#define PR_CUDA(call)                                   \
-  do {                                                  \
-    cudaError_t e_ = (call);                            \
-    if (e_ != cudaSuccess) return cuda_fail(e_, #call); \
-  } while (0)
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+float zthreshold(float tau) {
+  const double t = (double)tau;
+  if (!(t > 0.0)) return -INFINITY;
+  if (!(t < 1.0)) return INFINITY;
+  return (float)std::log(t / (1.0 - t));
+}
+
+pr_status set_device(pr_ctx* c) {
+  PR_CUDA(cudaSetDevice(c->device));
+  return PR_OK;
+}
+
+pr_status timing_begin(pr_ctx* c, cudaStream_t s) {
+  c->tev_n = 0;
+  if (!c->timing) return PR_OK;
+  return timing_mark(c, s);
+}
+
+pr_status timing_mark(pr_ctx* c, cudaStream_t s) {
+  if (!c->timing || c->tev_n > PR_MAX_TIMED) return PR_OK;
+  cudaEvent_t& e = c->tev[c->tev_n];
+  if (!e) PR_CUDA(cudaEventCreate(&e));
+  PR_CUDA(cudaEventRecord(e, s));
+  ++c->tev_n;
+  return PR_OK;
+}
+
+}  // namespace prh
+
+using namespace prh;
+
+namespace {
 
 constexpr uint32_t STATE_MAGIC = 0x50525354u;  // "PRST"
 constexpr uint32_t STATE_VERSION = 1u;
 
 }  // namespace
 
-struct pr_ctx {
-  int device = 0;
-  int num_sms = 0;
-  int64_t max_rows = 0;
-  int32_t max_requests = 0;
-  // options
-  int32_t topk = 20, renorm = 0, split = 0, overlap = 0;
-  // workspace
-  float* rec = nullptr;          // [max_rows][8] per-row records of pr_route
-  uint32_t* rec_flags = nullptr; // [max_rows]
-  int32_t* req_cnt = nullptr;    // [max_requests] completion counters
-  float* acc = nullptr;          // [max_requests][ACC_WORDS] decode slots
-  uint32_t* flags = nullptr;     // flag word
-  // pr_route_host staging (allocated on first use)
-  void* stage[2] = {nullptr, nullptr};
-  int32_t* stage_chosen[2] = {nullptr, nullptr};
-  int64_t stage_rows = 0;
-  size_t stage_row_bytes = 0;
-  int64_t* h_offsets_dev = nullptr;
-  int32_t h_offsets_cap = 0;
-  float* h_w_dev = nullptr;
-  float* h_out = nullptr;        // [max_requests][NAGG + 1] scores and aggregates
-  uint8_t* h_ship_dev = nullptr;
-  uint32_t* h_flags_dev = nullptr;
-  cudaStream_t copy_stream = nullptr;
-  cudaEvent_t ev_copied[2] = {nullptr, nullptr};
-  cudaEvent_t ev_free[2] = {nullptr, nullptr};
-  // occupancy cache per (dtype, mode)
-  int bps[2][3] = {{0, 0, 0}, {0, 0, 0}};
-  // persistent kernel: CTAs per SM per (dtype, mode, aligned); 0 = not set up yet
-  int ws_bps[2][3][2] = {};
-  // scorer head: activation scratch (rows x prk::HSCR floats), grown on demand
-  float* head_scr = nullptr;
-  int64_t head_scr_rows = 0;
-  bool head_ready = false;
-};
 
 namespace {
 
@@ -201,7 +193,6 @@ pr_status launch_rows(pr_ctx* c, pr_dtype dt, int mode, const prk::Args& a, cuda
   return PR_OK;
 }
 
-bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 size_t esize(pr_dtype dt) { return dt == PR_DTYPE_BF16 ? 2 : 4; }
 
@@ -232,17 +223,8 @@ void fill_row_args(prk::Args& a, const void* logits, pr_dtype dt, int64_t n_rows
   a.aligned = aligned16(logits) && ((row_stride * (int64_t)esize(dt)) % 16) == 0;
 }
 
-float zthreshold(float tau) {
-  const double t = (double)tau;
-  if (!(t > 0.0)) return -INFINITY;
-  if (!(t < 1.0)) return INFINITY;
-  return (float)std::log(t / (1.0 - t));
-}
 
-pr_status set_device(pr_ctx* c) {
-  PR_CUDA(cudaSetDevice(c->device));
-  return PR_OK;
-}
+
 
 }  // namespace
 
@@ -332,6 +314,8 @@ pr_status pr_ctx_destroy(pr_ctx* c) {
   cudaFree(c->h_ship_dev);
   cudaFree(c->h_flags_dev);
   cudaFree(c->head_scr);
+  for (cudaEvent_t e : c->tev)
+    if (e) cudaEventDestroy(e);
   if (c->copy_stream) cudaStreamDestroy(c->copy_stream);
   delete c;
   return PR_OK;
@@ -368,6 +352,10 @@ pr_status pr_ctx_set_option(pr_ctx* c, int32_t option, int32_t value) {
       if (value != 0 && value != 1) return PR_ERR_INVALID_ARG;
       c->overlap = value;
       return PR_OK;
+    case PR_OPT_TIMING:
+      if (value != 0 && value != 1) return PR_ERR_INVALID_ARG;
+      c->timing = value;
+      return PR_OK;
   }
   return PR_ERR_INVALID_ARG;
 }
@@ -382,6 +370,18 @@ pr_status pr_ctx_flags(pr_ctx* c, void* stream, int32_t clear, uint32_t* flags) 
   if (clear) PR_CUDA(cudaMemsetAsync(c->flags, 0, sizeof(uint32_t), s));
   PR_CUDA(cudaStreamSynchronize(s));
   *flags = v;
+  return PR_OK;
+}
+
+pr_status pr_ctx_kernel_times(pr_ctx* c, float* ms, int32_t cap, int32_t* n) {
+  if (!c || !n || cap < 0 || (cap > 0 && !ms)) return PR_ERR_INVALID_ARG;
+  pr_status st = set_device(c);
+  if (st != PR_OK) return st;
+  const int32_t k = c->tev_n > 0 ? c->tev_n - 1 : 0;
+  *n = k;
+  if (k == 0) return PR_OK;
+  PR_CUDA(cudaEventSynchronize(c->tev[k]));
+  for (int32_t i = 0; i < k && i < cap; ++i) PR_CUDA(cudaEventElapsedTime(&ms[i], c->tev[i], c->tev[i + 1]));
   return PR_OK;
 }
 
@@ -536,64 +536,6 @@ pr_status pr_state_import(pr_ctx* c, const void* host_buf, size_t bytes) {
   PR_CUDA(cudaDeviceSynchronize());
   if (body) PR_CUDA(cudaMemcpy(c->acc, static_cast<const char*>(host_buf) + sizeof hdr, body,
                                cudaMemcpyHostToDevice));
-  return PR_OK;
-}
-
-int64_t pr_head_param_count(int32_t n_layers) {
-  if (n_layers < 1 || n_layers > prk::HMAXL) return -1;
-  return prk::head_param_count(n_layers);
-}
-
-pr_status pr_head_score(pr_ctx* c, const float* feat, const uint32_t* row_flags, int64_t n_rows,
-                        const int64_t* offsets, int32_t n_req, const float* w, int32_t n_layers,
-                        float tau, float* score, uint8_t* ship, uint32_t* req_flags,
-                        void* stream) {
-  if (!c || n_req < 0 || n_rows < 0) return PR_ERR_INVALID_ARG;
-  if (n_layers < 1 || n_layers > prk::HMAXL) return PR_ERR_INVALID_ARG;
-  if (n_rows > ((int64_t)1 << 23)) return PR_ERR_INVALID_ARG;  // int row arithmetic per request
-  if (n_req == 0) return PR_OK;
-  if (!offsets || !w || !score || !ship || !req_flags) return PR_ERR_INVALID_ARG;
-  if (n_rows > 0 && !feat) return PR_ERR_INVALID_ARG;
-  if (!aligned16(w)) return PR_ERR_INVALID_ARG;
-  pr_status st = set_device(c);
-  if (st != PR_OK) return st;
-  if (!c->head_ready) {
-    PR_CUDA(cudaFuncSetAttribute(prk::head_requests, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)sizeof(prk::HeadSmem)));
-    c->head_ready = true;
-  }
-  if (n_rows > c->head_scr_rows) {
-    // grow: wait for the kernels that may still use the old scratch
-    PR_CUDA(cudaDeviceSynchronize());
-    cudaFree(c->head_scr);
-    c->head_scr = nullptr;
-    c->head_scr_rows = 0;
-    if (cudaMalloc(&c->head_scr, (size_t)n_rows * prk::HSCR * sizeof(float)) != cudaSuccess) {
-      cudaGetLastError();
-      c->head_scr = nullptr;
-      return PR_ERR_NO_MEMORY;
-    }
-    c->head_scr_rows = n_rows;
-  }
-  prk::HeadArgs a;
-  memset(&a, 0, sizeof a);
-  a.feat = feat;
-  a.row_flags = row_flags;
-  a.n_rows = n_rows;
-  a.offsets = offsets;
-  a.n_req = n_req;
-  a.w = w;
-  a.n_layers = n_layers;
-  a.zthr = zthreshold(tau);
-  a.scratch = c->head_scr;
-  a.score = score;
-  a.ship = ship;
-  a.req_flags = req_flags;
-  a.ctx_flags = c->flags;
-  prk::head_requests<<<(unsigned)n_req, prk::NT, sizeof(prk::HeadSmem),
-                       reinterpret_cast<cudaStream_t>(stream)>>>(a);
-  PR_CUDA(cudaGetLastError());
-  g_launches.fetch_add(1, std::memory_order_relaxed);
   return PR_OK;
 }
 

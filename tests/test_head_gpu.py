@@ -157,3 +157,20 @@ def test_head_rejects_bad_arguments(B, ctx):
             B.pr_head_score(ctx, f, o, w, nl, 0.5)
     with pytest.raises(B.PRError):
         B.pr_head_score(ctx, f, o, w[1:], 2, 0.5)  # weights not 16-byte aligned
+
+
+def test_head_kernel_timing_option(B, ctx):
+    """PR_OPT_TIMING reports one positive duration per kernel (2 L + 3) and
+    leaves the results unchanged."""
+    lengths = [40, 90, 200]
+    feat, offsets = workloads.head_features(lengths, 4700)
+    w = workloads.head_weights(2)
+    s0, _, _ = run_head(B, ctx, feat, offsets, w, 2)
+    B.pr_ctx_set_option(ctx, B.PR_OPT_TIMING, 1)
+    try:
+        s1, _, _ = run_head(B, ctx, feat, offsets, w, 2)
+        times = B.pr_ctx_kernel_times(ctx)
+    finally:
+        B.pr_ctx_set_option(ctx, B.PR_OPT_TIMING, 0)
+    assert np.array_equal(s0, s1)
+    assert len(times) == 2 * 2 + 3 and all(t > 0 for t in times)
