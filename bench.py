@@ -724,6 +724,169 @@ def profiled_head_traffic():
         return None
 
 
+SEL_FILES = ("pr_device.cuh", "pr_select.cuh", "pr_select_api.cu")
+SEL_PROFILE = os.path.join(ROOT, "profiles", "sel_scatter_u32_pool16m.md")
+SEL_N = 1 << 24
+
+
+def sel_oracle_child(n: int):
+    from oracle import selective as osel
+    s, y = W.selective_pool(n)
+    t0 = time.perf_counter()
+    o = osel.selective_metrics(s, y, 0.5)
+    dt = time.perf_counter() - t0
+    print(json.dumps({"seconds": dt, "out": o}))
+    return 0
+
+
+def run_selective_workload(args):
+    """Coverage calibration plus AUROC / AUARC on a 2^24-score validation pool
+    (pr_selective_metrics): one radix sort and the metric scans per step."""
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", init_method="env://")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    from paper_2608_28726_gb300 import build as prbuild
+    prbuild.build()
+    from paper_2608_28726_gb300 import binding as B
+    n, q = SEL_N, 0.5
+    s_h, y_h = W.selective_pool(n)
+    sc, lb = torch.from_numpy(s_h).to(dev), torch.from_numpy(y_h).to(dev)
+    ctx = B.pr_ctx_create(local, max_rows=0, max_requests=1)
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    K = args.steps
+    res = {}
+
+    def step():
+        res["r"] = B.pr_selective_metrics(ctx, sc, q, labels=lb, stream=stream)
+
+    sampler = ClockSampler(local)
+    sampler.start()
+
+    def timed(timing: int):
+        B.pr_ctx_set_option(ctx, B.PR_OPT_TIMING, timing)
+        for _ in range(max(3, args.warmup)):
+            step()
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(K)]
+        kms = []
+        barrier(world)
+        torch.cuda.synchronize(dev)
+        n0 = B.launch_count()
+        for i in range(K):
+            flush.zero_()
+            ev[i][0].record(stream)
+            step()
+            ev[i][1].record(stream)
+            if timing:
+                kms.append(B.pr_ctx_kernel_times(ctx))
+        torch.cuda.synchronize(dev)
+        barrier(world)
+        tot = sum(a.elapsed_time(b) for a, b in ev)
+        return reduce_max(tot, world, dev) / K, B.launch_count() - n0, kms
+
+    t_wall0 = time.time()
+    ms, launches, _ = timed(0)
+    t_wall1 = time.time()
+    iso_ms, _, kms = timed(1)
+    B.pr_ctx_set_option(ctx, B.PR_OPT_TIMING, 0)
+    clocks = sampler.summary(t_wall0, t_wall1)
+    sampler.stop()
+    scatter_ms = float(np.mean([k[i] for k in kms for i in (3, 6, 9, 12)]))
+    per_kernel = np.mean(np.asarray(kms), axis=0).tolist()
+    got = res["r"]
+
+    hs, hy = torch.from_numpy(s_h).pin_memory(), torch.from_numpy(y_h).pin_memory()
+    ds, dy = torch.empty_like(sc), torch.empty_like(lb)
+
+    def e2e_step():
+        ds.copy_(hs, non_blocking=True)
+        dy.copy_(hy, non_blocking=True)
+        return B.pr_selective_metrics(ctx, ds, q, labels=dy, stream=stream)
+
+    e2e_step()
+    e2e_steps = max(3, min(K, 20))
+    barrier(world)
+    t0 = time.perf_counter()
+    for _ in range(e2e_steps):
+        e2e_step()
+    barrier(world)
+    e2e_s = reduce_max(time.perf_counter() - t0, world, dev)
+
+    peaks_file = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    peak = float(json.load(open(peaks_file))["hbm_gbs"]) if os.path.exists(peaks_file) else 6800.0
+    scatter_bytes = 10 * n  # read key + label, write key + label
+    step_bytes = 80 * n
+    achieved = scatter_bytes / (scatter_ms / 1e3) / 1e9
+    if rank == 0:
+        env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1")
+        out = subprocess.run([sys.executable, os.path.abspath(__file__), "--sel-oracle-child",
+                              str(n)], env=env, capture_output=True, text=True, check=True)
+        d = json.loads(out.stdout.strip().splitlines()[-1])
+        o = d["out"]
+        ok = (got["k"] == o["k"] and got["n_ship"] == o["n_ship"] and
+              got["n_finite"] == o["n_finite"] and got["n_pos"] == o["n_pos"] and
+              np.float32(got["tau"]) == np.float32(o["tau"]) and
+              abs(got["auroc"] - o["auroc"]) <= 1e-12 and abs(got["auarc"] - o["auarc"]) <= 1e-9)
+        print(json.dumps({
+            "metric": "validation scores calibrated and ranked per second (coverage tau, AUROC, "
+                      "AUARC; 2^24-score pool)",
+            "value": n * world / (ms / 1e3), "unit": "scores/s", "n_gpus": world, "steps": K,
+            "warmup": max(3, args.warmup), "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "u32", "data": "synthetic",
+            "config": {"workload": "selective metrics: %d seeded scores (sigmoid of N(0,1.5^2), "
+                                   "1%% NaN), labels Bernoulli(score), q = %.2f" % (n, q),
+                       "l2": "256 MB written between timed steps (flush)"},
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                         "frac": achieved / peak, "traffic": profiled_sel_traffic(),
+                         "kernel": "sel_scatter (radix pass)",
+                         "algorithmic_bytes_per_launch": scatter_bytes,
+                         "avg_launch_ms": scatter_ms,
+                         "step_algorithmic_bytes": step_bytes,
+                         "step_achieved_gbs": step_bytes / (ms / 1e3) / 1e9,
+                         "isolated_kernel_ms": per_kernel, "isolated_step_ms": iso_ms},
+            "cpu_baseline": {"value": n / d["seconds"], "unit": "scores/s", "cores": 1,
+                             "kind": "oracle",
+                             "sample": "the whole %d-score pool, float64 numpy oracle" % n},
+            "e2e": {"value": n * world * e2e_steps / e2e_s, "unit": "scores/s",
+                    "h2d_bytes_per_step": 5 * n, "d2h_bytes_per_step": 64,
+                    "api": "pr_selective_metrics after host copies of scores and labels"},
+            "gpu_launches": launches,
+            "clocks": clocks,
+            "parity": {"ok": bool(ok), "tau": got["tau"], "auroc": got["auroc"],
+                       "auarc": got["auarc"]},
+        }))
+    B.pr_ctx_destroy(ctx)
+    return 0
+
+
+def profiled_sel_traffic():
+    """DRAM bytes per sel_scatter launch from the committed ncu summary, if
+    taken on the current source (else None)."""
+    try:
+        text = open(SEL_PROFILE).read()
+    except OSError:
+        return None
+    vals = {}
+    for line in text.splitlines():
+        if ":" in line and line.strip().startswith("- "):
+            k, v = line.strip()[2:].split(":", 1)
+            vals[k.strip()] = v.strip().strip("`")
+    h = hashlib.sha256()
+    for f in SEL_FILES:
+        with open(os.path.join(ROOT, "paper_2608_28726_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    if vals.get("kernel_source_sha") != h.hexdigest()[:16]:
+        return None
+    try:
+        return int(vals["dram_bytes_per_launch"])
+    except (KeyError, ValueError):
+        return None
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -731,22 +894,28 @@ def main():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--workload", default=WORKLOAD,
-                    choices=["full", "tiny", "ragged", "wide", "decode", "head"],
+                    choices=["full", "tiny", "ragged", "wide", "decode", "head", "selective"],
                     help="full (default, the headline line), one of the other verifier "
-                         "workloads, or head (the transformer scorer head)")
+                         "workloads, head (the transformer scorer head) or selective "
+                         "(calibration and ranking metrics)")
     ap.add_argument("--requests", type=int, default=0,
                     help="profiling only: the first N requests of the workload")
     ap.add_argument("--skip-host", action="store_true",
                     help="profiling only: skip the host-memory and oracle legs")
     ap.add_argument("--head-oracle-sample", type=int, default=0, help=argparse.SUPPRESS)
     ap.add_argument("--head-layers", type=int, default=2, help=argparse.SUPPRESS)
+    ap.add_argument("--sel-oracle-child", type=int, default=0, help=argparse.SUPPRESS)
     args = ap.parse_args()
     if args.head_oracle_sample:
         return head_oracle_child(args.head_oracle_sample, args.head_layers)
+    if args.sel_oracle_child:
+        return sel_oracle_child(args.sel_oracle_child)
     if args.impl == "reference":
         return run_reference(args)
     if args.workload == "head":
         return run_head_workload(args)
+    if args.workload == "selective":
+        return run_selective_workload(args)
     if args.workload != WORKLOAD:
         return run_other_workload(args)
     return run_gb300(args)

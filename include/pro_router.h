@@ -107,9 +107,10 @@ typedef enum { PR_DTYPE_F32 = 0, PR_DTYPE_BF16 = 1 } pr_dtype;
                                 anything.  Only for callers whose inputs are complete before
                                 the preceding kernel starts (e.g. back-to-back verifier calls
                                 on resident logits).  Default 0. */
-#define PR_OPT_TIMING 4      /* 1: calls that launch several kernels (pr_head_score) record a CUDA
-                                event after each kernel, for pr_ctx_kernel_times; the kernels
-                                then no longer overlap one another.  Default 0. */
+#define PR_OPT_TIMING 4      /* 1: calls that launch several kernels (pr_head_score,
+                                pr_selective_metrics) record a CUDA event after each kernel, for
+                                pr_ctx_kernel_times; the kernels then no longer overlap one
+                                another.  Default 0. */
 
 typedef struct pr_ctx pr_ctx;
 
@@ -146,7 +147,9 @@ pr_status pr_ctx_flags(pr_ctx* ctx, void* stream, int32_t clear, uint32_t* flags
  * Per-kernel device times (milliseconds, launch order) of the last call made
  * with PR_OPT_TIMING = 1: for pr_head_score the embedding, the first QKV
  * projection, then per layer the attention and the row-local block, then the
- * pool.  Waits for the call's last event.  Writes min(count, cap) values to
+ * pool; for pr_selective_metrics the key transform, per radix pass the
+ * histogram, digit scan and scatter, then the label prefix, the tile scan,
+ * the metrics (with labels) and the final reduction.  Waits for the call's last event.  Writes min(count, cap) values to
  * `ms` and the count to *n (0 if no timed call was made).
  */
 pr_status pr_ctx_kernel_times(pr_ctx* ctx, float* ms, int32_t cap, int32_t* n);
@@ -302,6 +305,43 @@ pr_status pr_head_score(pr_ctx* ctx, const float* feat, const uint32_t* row_flag
                         int64_t n_rows, const int64_t* offsets, int32_t n_req, const float* w,
                         int32_t n_layers, float tau, float* score, uint8_t* ship,
                         uint32_t* req_flags, void* stream);
+
+/* ---- operating point and selective-prediction metrics ------------------------------ */
+
+typedef struct {
+  float tau;           /* threshold: the k-th largest finite score; +inf when k = 0 */
+  int32_t reserved;
+  int64_t n_finite;    /* requests with a finite score (the others never ship) */
+  int64_t k;           /* requests the coverage rule ships: min(floor(q n + 1/2), n_finite) */
+  int64_t n_ship;      /* finite scores >= tau: k plus the ties at tau */
+  int64_t n_pos;       /* correct answers among the finite-scored requests (0 without labels) */
+  double auroc;        /* P(correct scores above incorrect), ties 1/2; NaN without both classes */
+  double auarc;        /* area under accuracy-among-shipped vs ship rate; NaN without labels */
+  double acc_shipped;  /* accuracy among the n_ship requests with score >= tau */
+} pr_selective;
+
+/*
+ * Calibrate the operating point on a validation pool and score the ranking
+ * (Section 3.1: tau is fixed in advance on a validation pool; Section 4.1:
+ * the coverage rule of selective prediction fixes a ship fraction q, and
+ * AUROC / the area under the shipping-accuracy curve measure the ranking).
+ *   scores  device float [n], e.g. the score output of pr_route or
+ *           pr_head_score; non-finite entries (flagged requests) never ship
+ *           and are left out of the metrics
+ *   labels  device uint8 [n] (non-zero = correct) or NULL (calibration only;
+ *           with the pairwise label the AUARC field is the paper's AUACC)
+ *   n       0 <= n < 2^31;  q: ship fraction in [0, 1]
+ *   out     host struct, written before the call returns
+ * A tie group's order is undefined, so AUARC spreads its correct answers
+ * evenly over its ranks (the expectation over orders) and AUROC counts ties
+ * as 1/2.  Runs as one stable radix sort of the scores plus scans on
+ * `stream` (17 kernels) and synchronises it; results are deterministic.  The
+ * context holds a sort workspace of about 15 bytes per score, allocated (or
+ * grown) by the first call with more scores than before -- that call
+ * synchronises the device.
+ */
+pr_status pr_selective_metrics(pr_ctx* ctx, const float* scores, const uint8_t* labels, int64_t n,
+                               double q, pr_selective* out, void* stream);
 
 /* ---- verification without allocation ------------------------------------------------- */
 

@@ -28,6 +28,7 @@ Parity status: AUROC is pinned against brute-force pair counting and
 scikit-learn's roc_auc_score; AUARC against brute-force averaging over every
 order of tied groups on small cases and closed forms (perfect ranking, equal
 scores, all correct); the calibration against its definition by counting.
+The array forms (auroc, auarc) are pinned against the loop forms.
 """
 from __future__ import annotations
 
@@ -65,9 +66,9 @@ def auroc_pairs(scores, labels) -> float:
     return float(((diff > 0).sum() + 0.5 * (diff == 0).sum()) / (pos.size * neg.size))
 
 
-def auroc(scores, labels) -> float:
-    """AUROC from average ranks (Mann-Whitney): the same number as
-    auroc_pairs, in O(n log n)."""
+def auroc_ranks(scores, labels) -> float:
+    """AUROC from average ranks (Mann-Whitney), tie groups walked in a loop:
+    the same number as auroc_pairs in O(n log n)."""
     s = np.asarray(scores, np.float64)
     y = np.asarray(labels).astype(bool)
     keep = np.isfinite(s)
@@ -88,8 +89,29 @@ def auroc(scores, labels) -> float:
     return float((ranks[y].sum() - P * (P + 1) / 2.0) / (P * N))
 
 
-def auarc(scores, labels) -> float:
-    """Area under the shipping-accuracy curve with tie groups averaged."""
+def auroc(scores, labels) -> float:
+    """auroc_ranks with the tie groups found by array operations (for pools of
+    millions of scores)."""
+    s = np.asarray(scores, np.float64)
+    y = np.asarray(labels).astype(bool)
+    keep = np.isfinite(s)
+    s, y = s[keep], y[keep]
+    P, N = int(y.sum()), int((~y).sum())
+    if P == 0 or N == 0:
+        return float("nan")
+    order = np.argsort(s, kind="stable")
+    ss = s[order]
+    start = np.flatnonzero(np.r_[True, ss[1:] != ss[:-1]])
+    end = np.r_[start[1:], ss.size]             # group [start, end), 0-based
+    grp = np.cumsum(np.r_[True, ss[1:] != ss[:-1]]) - 1
+    avg_rank = 0.5 * (start + end - 1) + 1.0    # 1-based average rank of each group
+    rank_sum = avg_rank[grp][y[order]].sum()
+    return float((rank_sum - P * (P + 1) / 2.0) / (P * N))
+
+
+def auarc_loop(scores, labels) -> float:
+    """Area under the shipping-accuracy curve with tie groups averaged, one
+    shipped request at a time."""
     s = np.asarray(scores, np.float64)
     y = np.asarray(labels).astype(np.float64)
     keep = np.isfinite(s)
@@ -113,6 +135,29 @@ def auarc(scores, labels) -> float:
         correct += cg
         i = j + 1
     return total / n
+
+
+def auarc(scores, labels) -> float:
+    """auarc_loop with the tie groups found by array operations."""
+    s = np.asarray(scores, np.float64)
+    y = np.asarray(labels).astype(np.float64)
+    keep = np.isfinite(s)
+    s, y = s[keep], y[keep]
+    n = s.size
+    if n == 0:
+        return float("nan")
+    order = np.argsort(-s, kind="stable")
+    ss, yy = s[order], y[order]
+    new = np.r_[True, ss[1:] != ss[:-1]]
+    start = np.flatnonzero(new)                  # group starts in shipping order
+    size = np.diff(np.r_[start, n])
+    correct = np.add.reduceat(yy, start)
+    before = np.r_[0.0, np.cumsum(correct)[:-1]]  # correct answers shipped before the group
+    grp = np.cumsum(new) - 1
+    k = np.arange(1, n + 1, dtype=np.float64)     # requests shipped
+    m = k - start[grp]                            # members of the own group shipped
+    Ck = before[grp] + m * correct[grp] / size[grp]
+    return float(np.sum(Ck / k) / n)
 
 
 def accuracy_at(scores, labels, tau: float):

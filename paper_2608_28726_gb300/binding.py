@@ -30,7 +30,7 @@ EXPORTS = (
     "pr_token_features", "pr_aggregate_score", "pr_route", "pr_route_host", "pr_decode_step",
     "pr_state_export", "pr_state_import", "pr_status_string", "pr_last_cuda_error",
     "pr_launch_count", "pr_route_noalloc", "pr_head_param_count", "pr_head_score",
-    "pr_ctx_kernel_times",
+    "pr_ctx_kernel_times", "pr_selective_metrics",
 )
 
 if not os.path.exists(LIB):
@@ -57,6 +57,7 @@ _SIGS = {
     "pr_route_noalloc": [_P, ctypes.c_int, _I64, _I64, _I64, _P, _P, _I32, _P, _F32, _F32, _P, _P,
                          _P, _P, _P],
     "pr_ctx_kernel_times": [_P, _P, _I32, ctypes.POINTER(_I32)],
+    "pr_selective_metrics": [_P, _P, _P, _I64, ctypes.c_double, _P, _P],
     "pr_head_score": [_P, _P, _P, _I64, _P, _I32, _P, _I32, _F32, _P, _P, _P, _P],
     "pr_state_export": [_P, _P, ctypes.POINTER(_SZ)],
     "pr_state_import": [_P, _P, _SZ],
@@ -289,3 +290,21 @@ def pr_head_score(ctx, feat, offsets, w, n_layers: int, tau: float, row_flags=No
                               _ptr(w), int(n_layers), float(tau), _ptr(score), _ptr(ship),
                               _ptr(req_flags), _stream(stream)), "pr_head_score")
     return score, ship, req_flags
+
+
+# ---- operating point and selective-prediction metrics ----------------------------------------
+
+class PrSelective(ctypes.Structure):
+    _fields_ = [("tau", ctypes.c_float), ("reserved", ctypes.c_int32), ("n_finite", _I64),
+                ("k", _I64), ("n_ship", _I64), ("n_pos", _I64), ("auroc", ctypes.c_double),
+                ("auarc", ctypes.c_double), ("acc_shipped", ctypes.c_double)]
+
+
+def pr_selective_metrics(ctx, scores, q: float, labels=None, stream=None) -> dict:
+    """Calibrate tau for ship fraction q on device scores; with device labels
+    (uint8, non-zero = correct) also AUROC, AUARC and the shipped accuracy."""
+    res = PrSelective()
+    _check(_lib.pr_selective_metrics(ctx, _ptr(scores), _ptr(labels), scores.numel(), float(q),
+                                     ctypes.byref(res), _stream(stream)), "pr_selective_metrics")
+    return {name: getattr(res, name) for name, _ in PrSelective._fields_ if name != "reserved"}
+

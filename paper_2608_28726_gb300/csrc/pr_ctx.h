@@ -47,6 +47,9 @@ struct pr_ctx {
   int64_t head_scr_rows = 0;
   bool head_ready = false;
   int head_bps_qkv = 1, head_bps_full = 1;  // resident head_rows CTAs per SM
+  // pr_selective_metrics: sort workspace for up to sel_cap scores, grown on demand
+  void* sel_ws = nullptr;
+  int64_t sel_cap = 0;
   // PR_OPT_TIMING: events after each kernel of the last multi-kernel call
   int32_t timing = 0;
   cudaEvent_t tev[PR_MAX_TIMED + 1] = {};

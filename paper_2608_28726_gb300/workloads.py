@@ -308,3 +308,19 @@ def head_features(lengths, seed: int = 4001) -> tuple[np.ndarray, np.ndarray]:
         T = int(lengths[r])
         feat[offsets[r]:offsets[r + 1], 5] = np.arange(1, T + 1) / max(T, 1)
     return feat.astype(np.float32), offsets
+
+
+# ---- validation pools for calibration -----------------------------------------------------
+
+def selective_pool(n: int, seed: int = 5001, nan_frac: float = 0.01):
+    """Seeded stand-in for a validation pool of verifier outputs:
+    (scores float32 [n], labels uint8 [n]).  z ~ N(0, 1.5^2), score =
+    sigmoid(z) rounded to float32 (so equal scores occur as they do in a real
+    pool), label = 1 (correct) with probability equal to the score, and a
+    fraction `nan_frac` of requests flagged (score NaN)."""
+    g = np.random.Generator(np.random.PCG64(seed))
+    z = g.normal(0.0, 1.5, size=n)
+    s = (1.0 / (1.0 + np.exp(-z))).astype(np.float32)
+    y = (g.random(n) < s).astype(np.uint8)
+    s[g.random(n) < nan_frac] = np.float32(np.nan)
+    return s, y

@@ -22,7 +22,15 @@ def tied_scores(n, seed, levels=20, nan_frac=0.0):
 @pytest.mark.parametrize("seed", [1, 2, 3])
 def test_auroc_rank_formula_equals_pair_counting(seed):
     s, y = tied_scores(400, seed, nan_frac=0.05)
+    assert sel.auroc_ranks(s, y) == pytest.approx(sel.auroc_pairs(s, y), abs=1e-12)
     assert sel.auroc(s, y) == pytest.approx(sel.auroc_pairs(s, y), abs=1e-12)
+
+
+@pytest.mark.parametrize("seed", [11, 12])
+def test_array_forms_equal_loop_forms(seed):
+    s, y = tied_scores(20000, seed, levels=300, nan_frac=0.02)
+    assert sel.auroc(s, y) == pytest.approx(sel.auroc_ranks(s, y), abs=1e-12)
+    assert sel.auarc(s, y) == pytest.approx(sel.auarc_loop(s, y), abs=1e-12)
 
 
 def test_auroc_matches_scikit_learn():
@@ -61,6 +69,7 @@ def test_auarc_equals_average_over_tie_orders(seed):
     n = 7
     s = g.integers(0, 3, size=n).astype(float)  # three levels: large tie groups
     y = g.integers(0, 2, size=n)
+    assert sel.auarc_loop(s, y) == pytest.approx(brute_auarc(s, y), abs=1e-12)
     assert sel.auarc(s, y) == pytest.approx(brute_auarc(s, y), abs=1e-12)
 
 
