@@ -324,3 +324,25 @@ def selective_pool(n: int, seed: int = 5001, nan_frac: float = 0.01):
     y = (g.random(n) < s).astype(np.uint8)
     s[g.random(n) < nan_frac] = np.float32(np.nan)
     return s, y
+
+
+# ---- quantile-summary + MLP aggregator weights --------------------------------------------
+
+QMLP_NS, QMLP_H = 28, 64
+
+
+def qmlp_param_count() -> int:
+    return QMLP_H * QMLP_NS + QMLP_H + QMLP_H * QMLP_H + QMLP_H + QMLP_H + 1
+
+
+def qmlp_weights(seed: int = 6001) -> np.ndarray:
+    """Seeded stand-in for the quantile-summary MLP's trained weights (flat
+    float32 in the library's layout): matrices N(0, 1/fan_in), biases
+    N(0, 0.02^2)."""
+    g = np.random.Generator(np.random.PCG64(seed))
+    parts = [g.normal(0.0, 1.0 / np.sqrt(QMLP_NS), QMLP_H * QMLP_NS), g.normal(0.0, 0.02, QMLP_H),
+             g.normal(0.0, 1.0 / np.sqrt(QMLP_H), QMLP_H * QMLP_H), g.normal(0.0, 0.02, QMLP_H),
+             g.normal(0.0, 1.0 / np.sqrt(QMLP_H), QMLP_H), g.normal(0.0, 0.02, 1)]
+    w = np.concatenate(parts).astype(np.float32)
+    assert w.size == qmlp_param_count()
+    return w
