@@ -677,7 +677,8 @@ def run_head_workload(args):
                        "n_layers": n_layers},
             "roofline": {"bound": "alu", "achieved": achieved, "peak": FP32_PEAK_TFLOPS,
                          "unit": "TFLOP/s", "frac": achieved / FP32_PEAK_TFLOPS,
-                         "traffic": profiled_head_traffic(), "kernel": "head_attn",
+                         "traffic": profiled_file_traffic(HEAD_PROFILE, HEAD_FILES),
+                         "kernel": "head_attn",
                          "peak_source": "derived: 152 SMs x 128 fp32 FMA lanes x 2 x 2.07 GHz",
                          "algorithmic_flops_per_launch": attn_flops,
                          "avg_launch_ms": attn_ms,
@@ -700,11 +701,165 @@ def run_head_workload(args):
     return 0
 
 
-def profiled_head_traffic():
-    """DRAM bytes per head_attn launch from the committed ncu summary, if taken on
-    the current head source (else None)."""
+QNT_FILES = ("pr_device.cuh", "pr_quant.cuh", "pr_quant_api.cu")
+QNT_PROFILE = os.path.join(ROOT, "profiles", "qmlp_requests_f32_ragged.md")
+# shared-memory bandwidth: 152 SMs x 32 banks x 4 bytes x 2,070 MHz
+SMEM_PEAK_GBS = 152 * 128 * 2.070e9 / 1e9
+
+
+def qnt_smem_bytes(lengths) -> int:
+    """Algorithmic shared-memory bytes of the in-CTA bitonic sorts: per request
+    of T <= 2,048 rows, n2 = the next power of two, log2(n2)(log2(n2)+1)/2
+    stages, each reading and writing the four n2-key columns once (4 + 4
+    bytes per key)."""
+    tot = 0
+    for T in np.asarray(lengths, np.int64):
+        if T <= 1 or T > 2048:
+            continue
+        n2 = 1 << int(np.ceil(np.log2(T)))
+        st = int(np.log2(n2))
+        tot += (st * (st + 1) // 2) * 4 * n2 * 8
+    return tot
+
+
+def qnt_oracle_child():
+    from oracle import quantile as oq
+    wl = W.make("ragged")
+    feat, offsets = W.head_features(wl.lengths, seed=4001)
+    w = W.qmlp_weights()
+    t0 = time.perf_counter()
+    so, po, fo, mo = oq.quantile_score(feat.astype(np.float64), np.zeros(int(offsets[-1]), np.uint32),
+                                       offsets, w.astype(np.float64), wl.tau)
+    dt = time.perf_counter() - t0
+    print(json.dumps({"seconds": dt, "score": so.tolist(), "ship": po.tolist()}))
+    return 0
+
+
+def run_quantile_workload(args):
+    """The quantile-summary + MLP aggregator on the ragged request layout
+    (1,024 requests, lognormal lengths, 181,659 rows)."""
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", init_method="env://")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    from paper_2608_28726_gb300 import build as prbuild
+    prbuild.build()
+    from paper_2608_28726_gb300 import binding as B
+    wl = W.make("ragged")
+    feat_h, offsets = W.head_features(wl.lengths, seed=4001)
+    w_h = W.qmlp_weights()
+    feat, off = torch.from_numpy(feat_h).to(dev), torch.from_numpy(offsets).to(dev)
+    w = torch.from_numpy(w_h).to(dev)
+    n_req, n_rows = wl.n_req, int(offsets[-1])
+    ctx = B.pr_ctx_create(local, max_rows=0, max_requests=1)
+    stream = torch.cuda.current_stream(dev)
+    score = torch.empty(n_req, device=dev)
+    ship = torch.empty(n_req, dtype=torch.uint8, device=dev)
+    rflags = torch.empty(n_req, dtype=torch.int32, device=dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+
+    def step():
+        B.pr_quantile_score(ctx, feat, off, w, wl.tau, score=score, ship=ship, req_flags=rflags,
+                            want_summary=False, stream=stream)
+
+    K = args.steps
+    sampler = ClockSampler(local)
+    sampler.start()
+    for _ in range(max(3, args.warmup)):
+        step()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(K)]
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    n0 = B.launch_count()
+    t_wall0 = time.time()
+    for i in range(K):
+        flush.zero_()
+        ev[i][0].record(stream)
+        step()
+        ev[i][1].record(stream)
+    torch.cuda.synchronize(dev)
+    t_wall1 = time.time()
+    barrier(world)
+    launches = B.launch_count() - n0
+    ms = reduce_max(sum(a.elapsed_time(b) for a, b in ev), world, dev) / K
+    clocks = sampler.summary(t_wall0, t_wall1)
+    sampler.stop()
+
+    hf, ho = torch.from_numpy(feat_h).pin_memory(), torch.from_numpy(offsets).pin_memory()
+    hs = torch.empty(n_req).pin_memory()
+    hsh = torch.empty(n_req, dtype=torch.uint8).pin_memory()
+    hfl = torch.empty(n_req, dtype=torch.int32).pin_memory()
+    dfeat, doff = torch.empty_like(feat), torch.empty_like(off)
+
+    def e2e_step():
+        dfeat.copy_(hf, non_blocking=True)
+        doff.copy_(ho, non_blocking=True)
+        B.pr_quantile_score(ctx, dfeat, doff, w, wl.tau, score=score, ship=ship, req_flags=rflags,
+                            want_summary=False, stream=stream)
+        hs.copy_(score, non_blocking=True)
+        hsh.copy_(ship, non_blocking=True)
+        hfl.copy_(rflags, non_blocking=True)
+        torch.cuda.synchronize(dev)
+
+    e2e_step()
+    e2e_steps = max(3, min(K, 50))
+    barrier(world)
+    t0 = time.perf_counter()
+    for _ in range(e2e_steps):
+        e2e_step()
+    barrier(world)
+    e2e_s = reduce_max(time.perf_counter() - t0, world, dev)
+
+    sbytes = qnt_smem_bytes(wl.lengths)
+    achieved = sbytes / (ms / 1e3) / 1e9
+    if rank == 0:
+        out = subprocess.run([sys.executable, os.path.abspath(__file__), "--qnt-oracle-child"],
+                             env=dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1",
+                                      MKL_NUM_THREADS="1"),
+                             capture_output=True, text=True, check=True)
+        d = json.loads(out.stdout.strip().splitlines()[-1])
+        so, po = np.asarray(d["score"]), np.asarray(d["ship"])
+        g = score.cpu().numpy().astype(np.float64)
+        ok = bool(np.all(np.abs(g - so) <= 1e-5) and
+                  np.all((ship.cpu().numpy() == po) | (np.abs(so - wl.tau) < 1e-6)))
+        print(json.dumps({
+            "metric": "scored tokens/sec (quantile summary + MLP, 1,024-request ragged layout)",
+            "value": n_rows * world / (ms / 1e3), "unit": UNIT, "n_gpus": world, "steps": K,
+            "warmup": max(3, args.warmup), "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": {"workload": "quantile summary + MLP: %d requests, lognormal lengths "
+                                   "(median 128, 8..1,024; %d rows), seeded feature records and "
+                                   "weights (6,081 floats)" % (n_req, n_rows),
+                       "l2": "256 MB written between timed steps (flush)"},
+            "roofline": {"bound": "alu", "achieved": achieved, "peak": SMEM_PEAK_GBS,
+                         "unit": "GB/s (shared memory)", "frac": achieved / SMEM_PEAK_GBS,
+                         "traffic": profiled_file_traffic(QNT_PROFILE, QNT_FILES),
+                         "kernel": "qmlp_requests",
+                         "peak_source": "derived: 152 SMs x 32 banks x 4 B x 2.07 GHz",
+                         "algorithmic_smem_bytes_per_launch": sbytes, "avg_launch_ms": ms},
+            "cpu_baseline": {"value": n_rows / d["seconds"], "unit": UNIT, "cores": 1,
+                             "kind": "oracle",
+                             "sample": "the whole %d-row workload, float64 numpy oracle" % n_rows},
+            "e2e": {"value": n_rows * world * e2e_steps / e2e_s, "unit": UNIT,
+                    "h2d_bytes_per_step": hf.numel() * 4 + ho.numel() * 8,
+                    "d2h_bytes_per_step": n_req * 9,
+                    "api": "pr_quantile_score with host copies of features, offsets and results"},
+            "gpu_launches": launches,
+            "clocks": clocks,
+            "parity": {"requests_checked": n_req, "ok": ok},
+        }))
+    B.pr_ctx_destroy(ctx)
+    return 0
+
+
+def profiled_file_traffic(path, files):
+    """DRAM bytes per launch from a committed ncu summary, if taken on the
+    current source of `files` (else None)."""
     try:
-        text = open(HEAD_PROFILE).read()
+        text = open(path).read()
     except OSError:
         return None
     vals = {}
@@ -713,7 +868,7 @@ def profiled_head_traffic():
             k, v = line.strip()[2:].split(":", 1)
             vals[k.strip()] = v.strip().strip("`")
     h = hashlib.sha256()
-    for f in HEAD_FILES:
+    for f in files:
         with open(os.path.join(ROOT, "paper_2608_28726_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     if vals.get("kernel_source_sha") != h.hexdigest()[:16]:
@@ -841,7 +996,8 @@ def run_selective_workload(args):
                                    "1%% NaN), labels Bernoulli(score), q = %.2f" % (n, q),
                        "l2": "256 MB written between timed steps (flush)"},
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                         "frac": achieved / peak, "traffic": profiled_sel_traffic(),
+                         "frac": achieved / peak,
+                         "traffic": profiled_file_traffic(SEL_PROFILE, SEL_FILES),
                          "kernel": "sel_scatter (radix pass)",
                          "algorithmic_bytes_per_launch": scatter_bytes,
                          "avg_launch_ms": scatter_ms,
@@ -863,30 +1019,6 @@ def run_selective_workload(args):
     return 0
 
 
-def profiled_sel_traffic():
-    """DRAM bytes per sel_scatter launch from the committed ncu summary, if
-    taken on the current source (else None)."""
-    try:
-        text = open(SEL_PROFILE).read()
-    except OSError:
-        return None
-    vals = {}
-    for line in text.splitlines():
-        if ":" in line and line.strip().startswith("- "):
-            k, v = line.strip()[2:].split(":", 1)
-            vals[k.strip()] = v.strip().strip("`")
-    h = hashlib.sha256()
-    for f in SEL_FILES:
-        with open(os.path.join(ROOT, "paper_2608_28726_gb300", "csrc", f), "rb") as fh:
-            h.update(fh.read())
-    if vals.get("kernel_source_sha") != h.hexdigest()[:16]:
-        return None
-    try:
-        return int(vals["dram_bytes_per_launch"])
-    except (KeyError, ValueError):
-        return None
-
-
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -894,10 +1026,11 @@ def main():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--workload", default=WORKLOAD,
-                    choices=["full", "tiny", "ragged", "wide", "decode", "head", "selective"],
+                    choices=["full", "tiny", "ragged", "wide", "decode", "head", "selective",
+                             "quantile"],
                     help="full (default, the headline line), one of the other verifier "
-                         "workloads, head (the transformer scorer head) or selective "
-                         "(calibration and ranking metrics)")
+                         "workloads, head (the transformer scorer head), quantile (the "
+                         "quantile-summary MLP) or selective (calibration and ranking metrics)")
     ap.add_argument("--requests", type=int, default=0,
                     help="profiling only: the first N requests of the workload")
     ap.add_argument("--skip-host", action="store_true",
@@ -905,7 +1038,10 @@ def main():
     ap.add_argument("--head-oracle-sample", type=int, default=0, help=argparse.SUPPRESS)
     ap.add_argument("--head-layers", type=int, default=2, help=argparse.SUPPRESS)
     ap.add_argument("--sel-oracle-child", type=int, default=0, help=argparse.SUPPRESS)
+    ap.add_argument("--qnt-oracle-child", action="store_true", help=argparse.SUPPRESS)
     args = ap.parse_args()
+    if args.qnt_oracle_child:
+        return qnt_oracle_child()
     if args.head_oracle_sample:
         return head_oracle_child(args.head_oracle_sample, args.head_layers)
     if args.sel_oracle_child:
@@ -916,6 +1052,8 @@ def main():
         return run_head_workload(args)
     if args.workload == "selective":
         return run_selective_workload(args)
+    if args.workload == "quantile":
+        return run_quantile_workload(args)
     if args.workload != WORKLOAD:
         return run_other_workload(args)
     return run_gb300(args)

@@ -107,7 +107,7 @@ typedef enum { PR_DTYPE_F32 = 0, PR_DTYPE_BF16 = 1 } pr_dtype;
                                 anything.  Only for callers whose inputs are complete before
                                 the preceding kernel starts (e.g. back-to-back verifier calls
                                 on resident logits).  Default 0. */
-#define PR_OPT_TIMING 4      /* 1: calls that launch several kernels (pr_head_score,
+#define PR_OPT_TIMING 4      /* 1: the scorer calls (pr_head_score, pr_quantile_score,
                                 pr_selective_metrics) record a CUDA event after each kernel, for
                                 pr_ctx_kernel_times; the kernels then no longer overlap one
                                 another.  Default 0. */
@@ -305,6 +305,36 @@ pr_status pr_head_score(pr_ctx* ctx, const float* feat, const uint32_t* row_flag
                         int64_t n_rows, const int64_t* offsets, int32_t n_req, const float* w,
                         int32_t n_layers, float tau, float* score, uint8_t* ship,
                         uint32_t* req_flags, void* stream);
+
+/* ---- quantile-summary + MLP aggregator ------------------------------------------------ */
+
+#define PR_QMLP_SUMMARY 28   /* summary length: 4 features x 7 quantile levels */
+#define PR_QMLP_PARAMS 6081  /* weights of the 28 -> 64 -> 64 -> 1 MLP */
+
+/*
+ * The verifier-architecture ablation's alternative scorer (Section 4.2,
+ * Table 2, "quantile summary + MLP").  Per request, for each feature x in
+ * (l, m, h, rho) (record slots LOGP, MAXP, TOPK, RHO of Eq. 3) over its T
+ * rows, the quantiles at levels 0, 1/10, 1/4, 1/2, 3/4, 9/10, 1 by linear
+ * interpolation between order statistics (x_(0) <= ... <= x_(T-1); level a/b:
+ * i = floor(a (T-1) / b), f = (a (T-1) mod b) / b, q = x_(i) + f (x_(i+1) -
+ * x_(i))), then z = w3 . ReLU(W2 ReLU(W1 s + b1) + b2) + b3, score =
+ * sigmoid(z), ship = (z >= logit(tau)).
+ *   feat, row_flags, offsets, n_rows: as pr_head_score (flags escalate with
+ *              score NaN, empty requests score 0, bad offsets PR_FLAG_BAD_OFFSETS)
+ *   w          device float [PR_QMLP_PARAMS]: W1[64][28] b1[64] W2[64][64] b2[64]
+ *              w3[64] b3 (row-major, y = W x + b)
+ *   summary    device float [n_req][PR_QMLP_SUMMARY] or NULL: the quantiles,
+ *              feature-major (written for requests that are scored)
+ *   score, ship, req_flags   device [n_req]                     (outputs)
+ * One launch, one CTA per request; requests of up to 2,048 rows are sorted in
+ * shared memory, longer ones use radix selection over global memory (exact,
+ * slower).  fp32, fixed-order sums.  n_rows < 2^31.
+ */
+pr_status pr_quantile_score(pr_ctx* ctx, const float* feat, const uint32_t* row_flags,
+                            int64_t n_rows, const int64_t* offsets, int32_t n_req, const float* w,
+                            float tau, float* summary, float* score, uint8_t* ship,
+                            uint32_t* req_flags, void* stream);
 
 /* ---- operating point and selective-prediction metrics ------------------------------ */
 

@@ -23,6 +23,7 @@ PR_NFEAT, PR_NAGG, PR_MAX_TOPK = 8, 11, 32
 PR_OPT_TOPK, PR_OPT_TOPK_RENORM, PR_OPT_SPLIT, PR_OPT_OVERLAP, PR_OPT_TIMING = 0, 1, 2, 3, 4
 PR_NOALLOC_MAX_ROWS, PR_NOALLOC_MAX_REQUESTS = 16384, 1024
 PR_HEAD_D, PR_HEAD_HEADS, PR_HEAD_FF, PR_HEAD_MAX_LAYERS = 64, 4, 128, 8
+PR_QMLP_SUMMARY, PR_QMLP_PARAMS = 28, 6081
 
 # every symbol include/pro_router.h declares
 EXPORTS = (
@@ -30,7 +31,7 @@ EXPORTS = (
     "pr_token_features", "pr_aggregate_score", "pr_route", "pr_route_host", "pr_decode_step",
     "pr_state_export", "pr_state_import", "pr_status_string", "pr_last_cuda_error",
     "pr_launch_count", "pr_route_noalloc", "pr_head_param_count", "pr_head_score",
-    "pr_ctx_kernel_times", "pr_selective_metrics",
+    "pr_ctx_kernel_times", "pr_selective_metrics", "pr_quantile_score",
 )
 
 if not os.path.exists(LIB):
@@ -57,6 +58,7 @@ _SIGS = {
     "pr_route_noalloc": [_P, ctypes.c_int, _I64, _I64, _I64, _P, _P, _I32, _P, _F32, _F32, _P, _P,
                          _P, _P, _P],
     "pr_ctx_kernel_times": [_P, _P, _I32, ctypes.POINTER(_I32)],
+    "pr_quantile_score": [_P, _P, _P, _I64, _P, _I32, _P, _F32, _P, _P, _P, _P, _P],
     "pr_selective_metrics": [_P, _P, _P, _I64, ctypes.c_double, _P, _P],
     "pr_head_score": [_P, _P, _P, _I64, _P, _I32, _P, _I32, _F32, _P, _P, _P, _P],
     "pr_state_export": [_P, _P, ctypes.POINTER(_SZ)],
@@ -307,4 +309,22 @@ def pr_selective_metrics(ctx, scores, q: float, labels=None, stream=None) -> dic
     _check(_lib.pr_selective_metrics(ctx, _ptr(scores), _ptr(labels), scores.numel(), float(q),
                                      ctypes.byref(res), _stream(stream)), "pr_selective_metrics")
     return {name: getattr(res, name) for name, _ in PrSelective._fields_ if name != "reserved"}
+
+
+# ---- quantile-summary + MLP aggregator ----------------------------------------------------------
+
+def pr_quantile_score(ctx, feat, offsets, w, tau: float, row_flags=None, summary=None, score=None,
+                      ship=None, req_flags=None, want_summary: bool = True, stream=None):
+    n_req = offsets.numel() - 1
+    dev = feat.device
+    if summary is None and want_summary:
+        summary = torch.empty(n_req, PR_QMLP_SUMMARY, dtype=torch.float32, device=dev)
+    score = torch.empty(n_req, dtype=torch.float32, device=dev) if score is None else score
+    ship = torch.empty(n_req, dtype=torch.uint8, device=dev) if ship is None else ship
+    req_flags = torch.empty(n_req, dtype=torch.int32, device=dev) if req_flags is None else req_flags
+    _check(_lib.pr_quantile_score(ctx, _ptr(feat), _ptr(row_flags), feat.size(0), _ptr(offsets),
+                                  n_req, _ptr(w), float(tau), _ptr(summary), _ptr(score),
+                                  _ptr(ship), _ptr(req_flags), _stream(stream)),
+           "pr_quantile_score")
+    return score, ship, req_flags, summary
 

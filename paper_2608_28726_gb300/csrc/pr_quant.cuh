@@ -1,0 +1,244 @@
+// The quantile-summary + MLP aggregator on the GPU (Pro-Router, Section 4.2,
+// Table 2: the verifier-architecture ablation's alternative to the
+// transformer head).  Per request: for each of the four Eq. 3 features (l, m,
+// h, rho) over its T rows, the quantiles at levels a/b (q_level_a / q_level_b; linear
+// interpolation between order statistics), a 28-number summary, then a
+// 28 -> 64 -> 64 -> 1 ReLU MLP and a sigmoid.
+//
+// One CTA per request.  Up to Q_CAP rows the four feature columns are loaded
+// into shared memory as order-preserving 32-bit keys and bitonic-sorted
+// together; longer requests find each needed order statistic by radix
+// selection (four 8-bit passes of shared histograms over the request's rows in
+// global memory).  Both give the exact order statistics.  The MLP runs in the
+// same CTA with fixed-order sums.
+#pragma once
+
+#include "pr_device.cuh"
+
+namespace prk {
+
+constexpr int Q_NT = 256;
+constexpr int Q_NQ = 7;             // quantile levels
+constexpr int Q_NS = 4 * Q_NQ;      // summary length
+constexpr int Q_H = 64;             // hidden width
+constexpr int Q_CAP = 2048;         // rows sorted in shared memory
+__constant__ int32_t q_level_a[Q_NQ] = {0, 1, 1, 1, 3, 9, 1};
+__constant__ int32_t q_level_b[Q_NQ] = {1, 10, 4, 2, 4, 10, 1};
+
+// weight offsets (floats)
+constexpr int QW_W1 = 0, QW_B1 = QW_W1 + Q_H * Q_NS, QW_W2 = QW_B1 + Q_H,
+              QW_B2 = QW_W2 + Q_H * Q_H, QW_W3 = QW_B2 + Q_H, QW_B3 = QW_W3 + Q_H,
+              QW_SIZE = QW_B3 + 1;
+
+struct QArgs {
+  const float* feat;
+  const uint32_t* row_flags;
+  int64_t n_rows;
+  const int64_t* offsets;
+  int32_t n_req;
+  const float* w;
+  float zthr;
+  float* summary;  // [n_req][28] or null
+  float* score;
+  uint8_t* ship;
+  uint32_t* req_flags;
+  uint32_t* ctx_flags;
+};
+
+__device__ __forceinline__ uint32_t q_key(float x) {
+  const uint32_t u = __float_as_uint(x);
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+__device__ __forceinline__ float q_unkey(uint32_t k) {
+  return __uint_as_float((k & 0x80000000u) ? (k & 0x7fffffffu) : ~k);
+}
+
+// record slot of feature f: l, m, h, rho
+__device__ __forceinline__ int q_slot(int f) { return f == 0 ? 0 : f == 1 ? 1 : f == 2 ? 4 : 5; }
+
+// Key of rank r (0-based, ascending) among the keys of feature f in rows
+// [lo, lo + T), by radix selection over global memory.  Whole CTA.
+__device__ uint32_t q_select(const float* __restrict__ feat, int64_t lo, int T, int f, int r,
+                             uint32_t* hist, uint32_t* bcast) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  uint32_t prefix = 0, mask = 0;
+  uint32_t rank = (uint32_t)r;
+  const int slot = q_slot(f);
+  for (int shift = 24; shift >= 0; shift -= 8) {
+    hist[tid] = 0;
+    __syncthreads();
+    for (int t = tid; t < T; t += Q_NT) {
+      const uint32_t k = q_key(feat[(lo + t) * NFEAT + slot]);
+      if ((k & mask) == prefix) atomicAdd(&hist[(k >> shift) & 0xff], 1u);
+    }
+    __syncthreads();
+    if (warp == 0) {  // the digit whose cumulative count passes `rank`
+      uint32_t c[8], s = 0;
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        c[e] = hist[lane * 8 + e];
+        s += c[e];
+      }
+      uint32_t x = s;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_up_sync(FULL, x, o);
+        if (lane >= o) x += y;
+      }
+      const unsigned hit = __ballot_sync(FULL, x > rank);
+      const int L = __ffs(hit) - 1;  // first lane whose inclusive count passes rank
+      if (lane == L) {
+        uint32_t cum = x - s;
+        int d = lane * 8;
+        for (int e = 0; e < 8; ++e, ++d) {
+          if (rank < cum + c[e]) break;
+          cum += c[e];
+        }
+        bcast[0] = (uint32_t)d;
+        bcast[1] = rank - cum;
+      }
+    }
+    __syncthreads();
+    prefix |= bcast[0] << shift;
+    mask |= 0xffu << shift;
+    rank = bcast[1];
+    __syncthreads();
+  }
+  return prefix;
+}
+
+__global__ void __launch_bounds__(Q_NT) qmlp_requests(const QArgs a) {
+  extern __shared__ __align__(16) uint32_t qs[];  // [4][n2] keys (shared-memory path)
+  __shared__ float qv[Q_NS];
+  __shared__ float h1[Q_H], h2[Q_H];
+  __shared__ uint32_t hist[256], bcast[2], wfl[Q_NT / 32];
+  __shared__ float zpart[2];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int64_t r = blockIdx.x;
+  const int64_t lo = a.offsets[r], hi = a.offsets[r + 1];
+  if (lo < 0 || hi < lo || hi > a.n_rows) {
+    if (tid == 0) {
+      a.score[r] = NAN;
+      a.ship[r] = 0;
+      a.req_flags[r] = FLAG_BAD_OFFSETS;
+      atomicOr(a.ctx_flags, FLAG_BAD_OFFSETS);
+    }
+    return;
+  }
+  const int T = (int)(hi - lo);
+  if (T == 0) {
+    if (tid == 0) {
+      a.score[r] = 0.f;
+      a.ship[r] = 0;
+      a.req_flags[r] = FLAG_EMPTY_REQ;
+    }
+    return;
+  }
+  uint32_t fl = 0;
+  if (a.row_flags)
+    for (int t = tid; t < T; t += Q_NT) fl |= a.row_flags[lo + t];
+  fl = __reduce_or_sync(FULL, fl);
+  if (lane == 0) wfl[warp] = fl;
+  __syncthreads();
+  fl = 0;
+#pragma unroll
+  for (int w2 = 0; w2 < Q_NT / 32; ++w2) fl |= wfl[w2];
+  if (fl & (FLAG_NONFINITE | FLAG_BAD_CHOSEN)) {
+    if (tid == 0) {
+      a.score[r] = NAN;
+      a.ship[r] = 0;
+      a.req_flags[r] = fl;
+    }
+    return;
+  }
+
+  if (T <= Q_CAP) {
+    int ln2 = 0;  // n2 = 2^ln2 >= T
+    while ((1 << ln2) < T) ++ln2;
+    const int n2 = 1 << ln2;
+    for (int i = tid; i < 4 * n2; i += Q_NT) {
+      const int f = i >> ln2, t = i & (n2 - 1);
+      qs[i] = t < T ? q_key(a.feat[(lo + t) * NFEAT + q_slot(f)]) : 0xffffffffu;
+    }
+    __syncthreads();
+    // bitonic sort of the four columns, ascending (powers of two: shifts, masks)
+    const int half = n2 >> 1, lh = ln2 - 1;
+    for (int k = 2; k <= n2; k <<= 1) {
+      for (int j = k >> 1; j > 0; j >>= 1) {
+        for (int idx = tid; idx < 4 * half; idx += Q_NT) {
+          const int f = idx >> lh, t = idx & (half - 1);
+          const int i = ((t & ~(j - 1)) << 1) | (t & (j - 1));
+          const int l = i + j;
+          uint32_t* col = qs + (f << ln2);
+          const uint32_t x = col[i], y = col[l];
+          const bool up = (i & k) == 0;
+          if ((x > y) == up) {
+            col[i] = y;
+            col[l] = x;
+          }
+        }
+        __syncthreads();
+      }
+    }
+    if (tid < Q_NS) {
+      const int f = tid / Q_NQ, j = tid - f * Q_NQ;
+      const int64_t num = (int64_t)q_level_a[j] * (T - 1);
+      const int b = q_level_b[j];
+      const int lo_i = (int)(num / b), rem = (int)(num - (int64_t)lo_i * b);
+      const uint32_t* col = qs + (f << ln2);
+      const float xl = q_unkey(col[lo_i]);
+      float q = xl;
+      if (rem) {
+        const float xh = q_unkey(col[min(lo_i + 1, T - 1)]);
+        q = xl + ((float)rem / (float)b) * (xh - xl);
+      }
+      qv[tid] = q;
+    }
+  } else {
+    for (int f = 0; f < 4; ++f)
+      for (int j = 0; j < Q_NQ; ++j) {
+        const int64_t num = (int64_t)q_level_a[j] * (T - 1);
+        const int b = q_level_b[j];
+        const int lo_i = (int)(num / b), rem = (int)(num - (int64_t)lo_i * b);
+        const float xl = q_unkey(q_select(a.feat, lo, T, f, lo_i, hist, bcast));
+        float q = xl;
+        if (rem) {
+          const float xh = q_unkey(q_select(a.feat, lo, T, f, min(lo_i + 1, T - 1), hist, bcast));
+          q = xl + ((float)rem / (float)b) * (xh - xl);
+        }
+        if (tid == 0) qv[f * Q_NQ + j] = q;
+      }
+  }
+  __syncthreads();
+
+  // MLP 28 -> 64 -> 64 -> 1 (sums in input order)
+  const float* W = a.w;
+  if (tid < Q_H) {
+    float s = __ldg(W + QW_B1 + tid);
+    for (int i = 0; i < Q_NS; ++i) s = fmaf(__ldg(W + QW_W1 + tid * Q_NS + i), qv[i], s);
+    h1[tid] = fmaxf(s, 0.f);
+  }
+  __syncthreads();
+  if (tid < Q_H) {
+    float s = __ldg(W + QW_B2 + tid);
+    for (int i = 0; i < Q_H; ++i) s = fmaf(__ldg(W + QW_W2 + tid * Q_H + i), h1[i], s);
+    h2[tid] = fmaxf(s, 0.f);
+  }
+  __syncthreads();
+  if (warp < 2) {
+    float z = __ldg(W + QW_W3 + tid) * h2[tid];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) z += __shfl_xor_sync(FULL, z, o);
+    if (lane == 0) zpart[warp] = z;
+  }
+  if (a.summary && tid < Q_NS) a.summary[r * Q_NS + tid] = qv[tid];
+  __syncthreads();
+  if (tid == 0) {
+    const float z = (zpart[0] + zpart[1]) + __ldg(W + QW_B3);
+    a.score[r] = 1.f / (1.f + expf(-z));
+    a.ship[r] = (z >= a.zthr) ? 1 : 0;
+    a.req_flags[r] = fl;
+  }
+}
+
+}  // namespace prk
