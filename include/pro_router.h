@@ -69,6 +69,8 @@ typedef enum { PR_DTYPE_F32 = 0, PR_DTYPE_BF16 = 1 } pr_dtype;
 #define PR_FLAG_EMPTY_REQ 4u   /* request with T = 0 */
 #define PR_FLAG_BAD_OFFSETS 8u /* offsets not monotone / outside the row range */
 #define PR_FLAG_BAD_SLOT 16u   /* decode slot id outside [0, n_slots) */
+#define PR_FLAG_TIMEOUT 32u    /* a bounded device-side wait ran out: that call's outputs are
+                                  not valid (context flag word only) */
 
 /* per-row feature record, PR_NFEAT floats */
 #define PR_NFEAT 8
@@ -107,8 +109,9 @@ typedef enum { PR_DTYPE_F32 = 0, PR_DTYPE_BF16 = 1 } pr_dtype;
                                 anything.  Only for callers whose inputs are complete before
                                 the preceding kernel starts (e.g. back-to-back verifier calls
                                 on resident logits).  Default 0. */
-#define PR_OPT_TIMING 4      /* 1: the scorer calls (pr_head_score, pr_quantile_score,
-                                pr_selective_metrics) record a CUDA event after each kernel, for
+#define PR_OPT_TIMING 4      /* 1: the calls after the verifier's (pr_head_score,
+                                pr_quantile_score, pr_selective_metrics, pr_lmhead_features)
+                                record a CUDA event after each kernel, for
                                 pr_ctx_kernel_times; the kernels then no longer overlap one
                                 another.  Default 0. */
 
@@ -305,6 +308,32 @@ pr_status pr_head_score(pr_ctx* ctx, const float* feat, const uint32_t* row_flag
                         int64_t n_rows, const int64_t* offsets, int32_t n_req, const float* w,
                         int32_t n_layers, float tau, float* score, uint8_t* ship,
                         uint32_t* req_flags, void* stream);
+
+/* ---- LM head fused with the row reduction --------------------------------------------- */
+
+/*
+ * pr_token_features without logits in memory: the rows' logits x = W h are
+ * computed on the tensor cores (tcgen05, bf16 inputs, fp32 accumulation) and
+ * reduced to the Eq. 3 row record in the GEMM's epilogue, so the [n_rows][V]
+ * logit matrix is never written (Section 3.1: the features are a side product
+ * of the small model's own decoding).
+ *   hidden   device bf16 [n_rows][d], row-major, 16-byte aligned (the final
+ *            hidden states of the small model)
+ *   weight   device bf16 [vocab][d], row-major, 16-byte aligned (the LM head;
+ *            x_v = sum_k weight[v][k] hidden[row][k])
+ *   d        hidden size, a multiple of 8
+ *   chosen, topk, offsets, n_req, feat, top2, row_flags: as pr_token_features
+ * The record has pr_token_features' slots and conventions, computed from the
+ * fp32 logits; uses the context's PR_OPT_TOPK_RENORM.  Two launches on
+ * `stream`; the context holds a state buffer of 288 bytes per row and
+ * vocabulary split (grown on demand; that call synchronises the device).  A
+ * device-side wait that runs out (2 s) raises PR_FLAG_TIMEOUT in the context
+ * flag word.
+ */
+pr_status pr_lmhead_features(pr_ctx* ctx, const void* hidden, const void* weight, int64_t n_rows,
+                             int64_t d, int64_t vocab, const int32_t* chosen, int32_t topk,
+                             const int64_t* offsets, int32_t n_req, float* feat, int32_t* top2,
+                             uint32_t* row_flags, void* stream);
 
 /* ---- quantile-summary + MLP aggregator ------------------------------------------------ */
 

@@ -18,7 +18,7 @@ from .build import LIB
 PR_OK, PR_ERR_INVALID_ARG, PR_ERR_UNSUPPORTED, PR_ERR_CUDA, PR_ERR_NO_MEMORY = 0, -1, -2, -3, -4
 PR_DTYPE_F32, PR_DTYPE_BF16 = 0, 1
 PR_FLAG_NONFINITE, PR_FLAG_BAD_CHOSEN, PR_FLAG_EMPTY_REQ = 1, 2, 4
-PR_FLAG_BAD_OFFSETS, PR_FLAG_BAD_SLOT = 8, 16
+PR_FLAG_BAD_OFFSETS, PR_FLAG_BAD_SLOT, PR_FLAG_TIMEOUT = 8, 16, 32
 PR_NFEAT, PR_NAGG, PR_MAX_TOPK = 8, 11, 32
 PR_OPT_TOPK, PR_OPT_TOPK_RENORM, PR_OPT_SPLIT, PR_OPT_OVERLAP, PR_OPT_TIMING = 0, 1, 2, 3, 4
 PR_NOALLOC_MAX_ROWS, PR_NOALLOC_MAX_REQUESTS = 16384, 1024
@@ -31,7 +31,7 @@ EXPORTS = (
     "pr_token_features", "pr_aggregate_score", "pr_route", "pr_route_host", "pr_decode_step",
     "pr_state_export", "pr_state_import", "pr_status_string", "pr_last_cuda_error",
     "pr_launch_count", "pr_route_noalloc", "pr_head_param_count", "pr_head_score",
-    "pr_ctx_kernel_times", "pr_selective_metrics", "pr_quantile_score",
+    "pr_ctx_kernel_times", "pr_selective_metrics", "pr_quantile_score", "pr_lmhead_features",
 )
 
 if not os.path.exists(LIB):
@@ -58,6 +58,7 @@ _SIGS = {
     "pr_route_noalloc": [_P, ctypes.c_int, _I64, _I64, _I64, _P, _P, _I32, _P, _F32, _F32, _P, _P,
                          _P, _P, _P],
     "pr_ctx_kernel_times": [_P, _P, _I32, ctypes.POINTER(_I32)],
+    "pr_lmhead_features": [_P, _P, _P, _I64, _I64, _I64, _P, _I32, _P, _I32, _P, _P, _P, _P],
     "pr_quantile_score": [_P, _P, _P, _I64, _P, _I32, _P, _F32, _P, _P, _P, _P, _P],
     "pr_selective_metrics": [_P, _P, _P, _I64, ctypes.c_double, _P, _P],
     "pr_head_score": [_P, _P, _P, _I64, _P, _I32, _P, _I32, _F32, _P, _P, _P, _P],
@@ -327,4 +328,27 @@ def pr_quantile_score(ctx, feat, offsets, w, tau: float, row_flags=None, summary
                                   _ptr(ship), _ptr(req_flags), _stream(stream)),
            "pr_quantile_score")
     return score, ship, req_flags, summary
+
+
+# ---- LM head fused with the row reduction ---------------------------------------------------
+
+def pr_lmhead_features(ctx, hidden, weight, chosen, topk: int = 20, offsets=None, feat=None,
+                       top2=None, row_flags=None, stream=None):
+    """Row records of the logits weight @ hidden[r] (bf16 [n][d] and [V][d])
+    without materialising the logits."""
+    if hidden.dtype != torch.bfloat16 or weight.dtype != torch.bfloat16:
+        raise TypeError("hidden and weight must be bfloat16")
+    if not (hidden.is_contiguous() and weight.is_contiguous()) or hidden.size(1) != weight.size(1):
+        raise ValueError("hidden [n][d] and weight [V][d] must be contiguous with the same d")
+    n, d = hidden.shape
+    V = weight.size(0)
+    dev = hidden.device
+    feat = torch.empty(n, PR_NFEAT, dtype=torch.float32, device=dev) if feat is None else feat
+    top2 = torch.empty(n, 2, dtype=torch.int32, device=dev) if top2 is None else top2
+    row_flags = torch.empty(n, dtype=torch.int32, device=dev) if row_flags is None else row_flags
+    n_req = 0 if offsets is None else offsets.numel() - 1
+    _check(_lib.pr_lmhead_features(ctx, _ptr(hidden), _ptr(weight), n, d, V, _ptr(chosen),
+                                   int(topk), _ptr(offsets), n_req, _ptr(feat), _ptr(top2),
+                                   _ptr(row_flags), _stream(stream)), "pr_lmhead_features")
+    return feat, top2, row_flags
 

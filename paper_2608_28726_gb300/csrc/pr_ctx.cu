@@ -150,6 +150,7 @@ pr_status pr_ctx_destroy(pr_ctx* c) {
   cudaFree(c->h_flags_dev);
   cudaFree(c->head_scr);
   cudaFree(c->sel_ws);
+  cudaFree(c->lm_parts);
   for (cudaEvent_t e : c->tev)
     if (e) cudaEventDestroy(e);
   if (c->copy_stream) cudaStreamDestroy(c->copy_stream);

@@ -50,6 +50,10 @@ struct pr_ctx {
   // pr_selective_metrics: sort workspace for up to sel_cap scores, grown on demand
   void* sel_ws = nullptr;
   int64_t sel_cap = 0;
+  // pr_lmhead_features: per-(row, split) states, grown on demand
+  void* lm_parts = nullptr;
+  size_t lm_parts_bytes = 0;
+  bool lm_ready = false;
   // PR_OPT_TIMING: events after each kernel of the last multi-kernel call
   int32_t timing = 0;
   cudaEvent_t tev[PR_MAX_TIMED + 1] = {};

@@ -1158,7 +1158,8 @@ struct AggArgs {
   uint32_t* ctx_flags;
 };
 
-__global__ void __launch_bounds__(NT) pool_requests(const AggArgs a) {
+// internal linkage: the header is included by more than one translation unit
+static __global__ void __launch_bounds__(NT) pool_requests(const AggArgs a) {
   const int lane = threadIdx.x & 31;
   const int64_t r = (int64_t)blockIdx.x * NWARP + (threadIdx.x >> 5);
   if (r >= a.n_req) return;

@@ -1,0 +1,141 @@
+// Host side of pr_lmhead_features: argument checks, the TMA tensor maps of the
+// hidden states and the LM-head weights, the vocabulary split and the launches
+// of the kernels in pr_lmhead.cuh.
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstring>
+
+#include "pr_ctx.h"
+#include "pr_lmhead.cuh"
+
+using namespace prh;
+
+static_assert(prk::LM_ERR_TIMEOUT == PR_FLAG_TIMEOUT, "flag bit");
+
+namespace {
+
+typedef CUresult (*EncodeTiled)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+// the driver's tensor-map encoder, looked up once through the runtime (no link
+// against the driver library)
+EncodeTiled encoder() {
+  static EncodeTiled fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiled>(p);
+  }
+  return fn;
+}
+
+// row-major bf16 matrix [rows][d] read in boxes of 64 columns x box_rows rows,
+// 128-byte swizzle, zero fill outside the matrix
+bool make_map(CUtensorMap* map, const void* base, int64_t rows, int64_t d, uint32_t box_rows) {
+  EncodeTiled enc = encoder();
+  if (!enc) return false;
+  const cuuint64_t dims[2] = {(cuuint64_t)d, (cuuint64_t)rows};
+  const cuuint64_t strides[1] = {(cuuint64_t)d * 2};
+  const cuuint32_t box[2] = {(cuuint32_t)prk::LM_BK, box_rows};
+  const cuuint32_t estr[2] = {1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
+             box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) ==
+         CUDA_SUCCESS;
+}
+
+}  // namespace
+
+extern "C" {
+
+pr_status pr_lmhead_features(pr_ctx* c, const void* hidden, const void* weight, int64_t n_rows,
+                             int64_t d, int64_t vocab, const int32_t* chosen, int32_t topk,
+                             const int64_t* offsets, int32_t n_req, float* feat, int32_t* top2,
+                             uint32_t* row_flags, void* stream) {
+  if (!c || n_rows < 0 || n_rows > 0x7fffffffLL || vocab <= 0 || vocab > 0x7fffffffLL)
+    return PR_ERR_INVALID_ARG;
+  if (d <= 0 || d % 8 != 0 || d > (int64_t)1 << 20) return PR_ERR_INVALID_ARG;
+  if (topk < 1 || topk > PR_MAX_TOPK || n_req < 0 || (offsets && n_req < 1))
+    return PR_ERR_INVALID_ARG;
+  if (n_rows == 0) return PR_OK;
+  if (!hidden || !weight || !chosen || !feat || !top2 || !row_flags) return PR_ERR_INVALID_ARG;
+  if (!aligned16(hidden) || !aligned16(weight)) return PR_ERR_INVALID_ARG;
+  pr_status st = set_device(c);
+  if (st != PR_OK) return st;
+  if (!c->lm_ready) {
+    PR_CUDA(cudaFuncSetAttribute(prk::lm_fused<20>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)prk::LM_SMEM));
+    PR_CUDA(cudaFuncSetAttribute(prk::lm_fused<32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)prk::LM_SMEM));
+    c->lm_ready = true;
+  }
+  CUtensorMap ma, mb;
+  if (!make_map(&ma, hidden, n_rows, d, prk::LM_BM) || !make_map(&mb, weight, vocab, d, prk::LM_BN))
+    return PR_ERR_UNSUPPORTED;
+  const int64_t mtiles = (n_rows + prk::LM_BM - 1) / prk::LM_BM;
+  const int64_t ntiles = (vocab + prk::LM_BN - 1) / prk::LM_BN;
+  if (mtiles > 0x7fffffffLL) return PR_ERR_INVALID_ARG;
+  // vocabulary splits: about one CTA per SM in total
+  const int64_t nsplit =
+      std::max<int64_t>(1, std::min<int64_t>(ntiles, (c->num_sms + mtiles / 2) / mtiles));
+  const size_t part_bytes = (size_t)nsplit * (size_t)n_rows * sizeof(prk::LmPart);
+  if (part_bytes > c->lm_parts_bytes) {
+    PR_CUDA(cudaDeviceSynchronize());  // the old buffer may still be in use
+    cudaFree(c->lm_parts);
+    c->lm_parts = nullptr;
+    c->lm_parts_bytes = 0;
+    if (cudaMalloc(&c->lm_parts, part_bytes) != cudaSuccess) {
+      cudaGetLastError();
+      c->lm_parts = nullptr;
+      return PR_ERR_NO_MEMORY;
+    }
+    c->lm_parts_bytes = part_bytes;
+  }
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if ((st = timing_begin(c, s)) != PR_OK) return st;
+  prk::LmArgs la;
+  memset(&la, 0, sizeof la);
+  la.n_rows = n_rows;
+  la.vocab = vocab;
+  la.d = (int32_t)d;
+  la.kblocks = (int32_t)((d + prk::LM_BK - 1) / prk::LM_BK);
+  la.ntiles = (int32_t)ntiles;
+  la.chosen = chosen;
+  la.parts = static_cast<prk::LmPart*>(c->lm_parts);
+  la.err = c->flags;
+  const int kc = topk > 2 ? topk : 2;
+  const dim3 grid((unsigned)mtiles, (unsigned)nsplit);
+  if (kc <= 20)
+    prk::lm_fused<20><<<grid, prk::LM_NT, prk::LM_SMEM, s>>>(ma, mb, la);
+  else
+    prk::lm_fused<32><<<grid, prk::LM_NT, prk::LM_SMEM, s>>>(ma, mb, la);
+  PR_CUDA(cudaGetLastError());
+  if ((st = timing_mark(c, s)) != PR_OK) return st;
+  prk::Args a;
+  memset(&a, 0, sizeof a);
+  a.n_rows = n_rows;
+  a.vocab = vocab;
+  a.chosen = chosen;
+  a.topk = topk;
+  a.kc = kc;
+  a.renorm = c->renorm;
+  a.offsets = offsets;
+  a.n_req = offsets ? n_req : 0;
+  a.feat = feat;
+  a.top2 = top2;
+  a.row_flags = row_flags;
+  a.ctx_flags = c->flags;
+  prk::lm_merge<<<(unsigned)((n_rows + 7) / 8), 256, 0, s>>>(a, la.parts, (int)nsplit);
+  PR_CUDA(cudaGetLastError());
+  g_launches.fetch_add(2, std::memory_order_relaxed);
+  return timing_mark(c, s);
+}
+
+}  // extern "C"
