@@ -701,6 +701,201 @@ def run_head_workload(args):
     return 0
 
 
+LM_FILES = ("pr_device.cuh", "pr_kernels.cuh", "pr_lmhead.cuh", "pr_lmhead_api.cu")
+LM_PROFILE = os.path.join(ROOT, "profiles", "lm_fused_bf16_full_response.md")
+LM_D = 3584
+
+
+def lm_oracle_child(n_sample: int):
+    """The float64 oracle on the first n_sample rows of the LM-head workload
+    (inputs regenerated on the CPU from the same seeds)."""
+    from oracle import lmhead
+    wl = W.make(WORKLOAD)
+    hidden, weight, chosen = W.lmhead_inputs(wl.n_rows, LM_D, wl.vocab, device="cpu")
+    hb = hidden[:n_sample].contiguous().view(torch.int16).numpy().view(np.uint16)
+    wb = weight.contiguous().view(torch.int16).numpy().view(np.uint16)
+    t0 = time.perf_counter()
+    o = lmhead.features(hb, wb, chosen[:n_sample].numpy(), K=20,
+                        offsets=np.array([0, n_sample], np.int64))
+    dt = time.perf_counter() - t0
+    print(json.dumps({"seconds": dt, "feat": o["feat"].tolist()}))
+    return 0
+
+
+def run_lmhead_workload(args):
+    """The LM head fused with the row reduction on the full-response batch:
+    8,847 hidden states of d = 3,584 against a 151,936 x 3,584 bf16 head."""
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", init_method="env://")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    from paper_2608_28726_gb300 import build as prbuild
+    prbuild.build()
+    from paper_2608_28726_gb300 import binding as B
+    wl = W.make(WORKLOAD)
+    n, V, d = wl.n_rows, wl.vocab, LM_D
+    # generated on the CPU (the oracle's child process draws the same values)
+    hidden, weight, chosen = (t.to(dev) for t in W.lmhead_inputs(n, d, V, device="cpu"))
+    off = torch.from_numpy(wl.offsets).to(dev)
+    ctx = B.pr_ctx_create(local, max_rows=n, max_requests=wl.n_req)
+    stream = torch.cuda.current_stream(dev)
+    feat = torch.empty(n, 8, device=dev)
+    top2 = torch.empty(n, 2, dtype=torch.int32, device=dev)
+    rf = torch.empty(n, dtype=torch.int32, device=dev)
+
+    def step():
+        B.pr_lmhead_features(ctx, hidden, weight, chosen, 20, offsets=off, feat=feat, top2=top2,
+                             row_flags=rf, stream=stream)
+
+    K = args.steps
+    sampler = ClockSampler(local)
+    sampler.start()
+    for _ in range(max(3, args.warmup)):
+        step()
+    torch.cuda.synchronize(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    n0 = B.launch_count()
+    t_wall0 = time.time()
+    e0.record(stream)
+    for _ in range(K):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    t_wall1 = time.time()
+    barrier(world)
+    launches = B.launch_count() - n0
+    ms = reduce_max(e0.elapsed_time(e1), world, dev) / K
+    clocks = sampler.summary(t_wall0, t_wall1)
+    # per kernel (PR_OPT_TIMING)
+    B.pr_ctx_set_option(ctx, B.PR_OPT_TIMING, 1)
+    kms = []
+    for _ in range(max(3, min(K, 10))):
+        step()
+        kms.append(B.pr_ctx_kernel_times(ctx))
+    B.pr_ctx_set_option(ctx, B.PR_OPT_TIMING, 0)
+    fused_ms, merge_ms = [float(x) for x in np.mean(np.asarray(kms), axis=0)]
+    # each thread-block cluster shape forced in turn (cm x cs)
+    shapes_ms = {}
+    for shape in (11, 21, 12, 22):
+        B.pr_ctx_set_option(ctx, B.PR_OPT_LMHEAD_CLUSTER, shape)
+        for _ in range(2):
+            step()
+        s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s0.record(stream)
+        for _ in range(5):
+            step()
+        s1.record(stream)
+        torch.cuda.synchronize(dev)
+        shapes_ms["%dx%d" % (shape // 10, shape % 10)] = s0.elapsed_time(s1) / 5
+    B.pr_ctx_set_option(ctx, B.PR_OPT_LMHEAD_CLUSTER, 0)
+    flags = B.pr_ctx_flags(ctx, clear=True)
+    # the unfused path for comparison: cuBLAS writes the bf16 logits, then the
+    # verifier reads them back (pr_token_features)
+    logits = torch.empty(n, V, dtype=torch.bfloat16, device=dev)
+    ufeat = torch.empty_like(feat)
+
+    def unfused():
+        torch.matmul(hidden, weight.t(), out=logits)
+        B.pr_token_features(ctx, logits, chosen, 20, offsets=off, feat=ufeat, stream=stream)
+
+    for _ in range(3):
+        unfused()
+    torch.cuda.synchronize(dev)
+    u0, u1, u2 = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+    KU = max(3, min(K, 20))
+    gemm_ms = feat_ms = 0.0
+    for _ in range(KU):
+        u0.record(stream)
+        torch.matmul(hidden, weight.t(), out=logits)
+        u1.record(stream)
+        B.pr_token_features(ctx, logits, chosen, 20, offsets=off, feat=ufeat, stream=stream)
+        u2.record(stream)
+        torch.cuda.synchronize(dev)
+        gemm_ms += u0.elapsed_time(u1)
+        feat_ms += u1.elapsed_time(u2)
+    gemm_ms /= KU
+    feat_ms /= KU
+    del logits
+    sampler.stop()
+
+    # e2e: the step's hidden states from pinned host memory, its records back
+    hh = hidden.cpu().pin_memory()
+    hfeat = torch.empty(n, 8).pin_memory()
+    dh = torch.empty_like(hidden)
+
+    def e2e_step():
+        dh.copy_(hh, non_blocking=True)
+        B.pr_lmhead_features(ctx, dh, weight, chosen, 20, offsets=off, feat=feat, top2=top2,
+                             row_flags=rf, stream=stream)
+        hfeat.copy_(feat, non_blocking=True)
+        torch.cuda.synchronize(dev)
+
+    e2e_step()
+    e2e_steps = max(3, min(K, 10))
+    barrier(world)
+    t0 = time.perf_counter()
+    for _ in range(e2e_steps):
+        e2e_step()
+    barrier(world)
+    e2e_s = reduce_max(time.perf_counter() - t0, world, dev)
+
+    flops = 2.0 * n * d * V
+    peaks_file = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    peaks = json.load(open(peaks_file)) if os.path.exists(peaks_file) else {}
+    peak = float(peaks.get("bf16_tflops_sustained", 1700.0))
+    achieved = flops / (fused_ms / 1e3) / 1e12
+    if rank == 0:
+        n_sample = 4
+        out = subprocess.run([sys.executable, os.path.abspath(__file__), "--lm-oracle-child",
+                              str(n_sample)],
+                             env=dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1",
+                                      MKL_NUM_THREADS="1"),
+                             capture_output=True, text=True, check=True)
+        dd = json.loads(out.stdout.strip().splitlines()[-1])
+        fo = np.asarray(dd["feat"], np.float64)
+        fg = feat[:n_sample].cpu().numpy().astype(np.float64)
+        fg[:, 5] = fo[:, 5]  # rho: the sample is one request of n_sample rows on the oracle side
+        ok = bool(np.all(np.abs(fg - fo) <= 1e-4 + 1e-4 * np.abs(fo))) and flags == 0
+        print(json.dumps({
+            "metric": "verified tokens/sec with the LM head fused (logits never written), "
+                      "V=151,936, d=3,584",
+            "value": n * world / (ms / 1e3), "unit": UNIT, "n_gpus": world, "steps": K,
+            "warmup": max(3, args.warmup), "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": "LM head + row features: %d hidden states (the full-response "
+                                   "layout), d=%d, V=%d bf16 head (1.09 GB), seeded" % (n, d, V),
+                       "l2": "inputs (1.15 GB) larger than L2 (129 MB), no flush"},
+            "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak,
+                         "unit": "TFLOP/s", "frac": achieved / peak,
+                         "traffic": profiled_file_traffic(LM_PROFILE, LM_FILES),
+                         "kernel": "lm_fused (tcgen05)",
+                         "peak_source": "measured cuBLAS bf16, sustained (%.1f burst)" %
+                                        float(peaks.get("bf16_tflops", 0.0)),
+                         "algorithmic_flops_per_launch": flops, "avg_launch_ms": fused_ms,
+                         "merge_ms": merge_ms, "step_ms_by_cluster_shape": shapes_ms},
+            "unfused": {"cublas_gemm_ms": gemm_ms, "pr_token_features_ms": feat_ms,
+                        "ms_per_step": gemm_ms + feat_ms,
+                        "logit_bytes_written_and_read": n * V * 2,
+                        "speedup_of_fused": (gemm_ms + feat_ms) / ms},
+            "cpu_baseline": {"value": n_sample / dd["seconds"], "unit": UNIT, "cores": 1,
+                             "kind": "oracle",
+                             "sample": "rows 0..%d: float64 product and features" % (n_sample - 1)},
+            "e2e": {"value": n * world * e2e_steps / e2e_s, "unit": UNIT,
+                    "h2d_bytes_per_step": n * d * 2, "d2h_bytes_per_step": n * 32,
+                    "api": "pr_lmhead_features after a host copy of the hidden states "
+                           "(the head's weights resident)"},
+            "gpu_launches": launches,
+            "clocks": clocks,
+            "parity": {"rows_checked": n_sample, "ok": ok, "flags": flags},
+        }))
+    B.pr_ctx_destroy(ctx)
+    return 0
+
+
 QNT_FILES = ("pr_device.cuh", "pr_quant.cuh", "pr_quant_api.cu")
 QNT_PROFILE = os.path.join(ROOT, "profiles", "qmlp_requests_f32_ragged.md")
 # shared-memory bandwidth: 152 SMs x 32 banks x 4 bytes x 2,070 MHz
@@ -1027,10 +1222,11 @@ def main():
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--workload", default=WORKLOAD,
                     choices=["full", "tiny", "ragged", "wide", "decode", "head", "selective",
-                             "quantile"],
+                             "quantile", "lmhead"],
                     help="full (default, the headline line), one of the other verifier "
                          "workloads, head (the transformer scorer head), quantile (the "
-                         "quantile-summary MLP) or selective (calibration and ranking metrics)")
+                         "quantile-summary MLP), selective (calibration and ranking metrics) "
+                         "or lmhead (the LM head fused with the row reduction)")
     ap.add_argument("--requests", type=int, default=0,
                     help="profiling only: the first N requests of the workload")
     ap.add_argument("--skip-host", action="store_true",
@@ -1039,7 +1235,10 @@ def main():
     ap.add_argument("--head-layers", type=int, default=2, help=argparse.SUPPRESS)
     ap.add_argument("--sel-oracle-child", type=int, default=0, help=argparse.SUPPRESS)
     ap.add_argument("--qnt-oracle-child", action="store_true", help=argparse.SUPPRESS)
+    ap.add_argument("--lm-oracle-child", type=int, default=0, help=argparse.SUPPRESS)
     args = ap.parse_args()
+    if args.lm_oracle_child:
+        return lm_oracle_child(args.lm_oracle_child)
     if args.qnt_oracle_child:
         return qnt_oracle_child()
     if args.head_oracle_sample:
@@ -1054,6 +1253,8 @@ def main():
         return run_selective_workload(args)
     if args.workload == "quantile":
         return run_quantile_workload(args)
+    if args.workload == "lmhead":
+        return run_lmhead_workload(args)
     if args.workload != WORKLOAD:
         return run_other_workload(args)
     return run_gb300(args)

@@ -109,6 +109,10 @@ typedef enum { PR_DTYPE_F32 = 0, PR_DTYPE_BF16 = 1 } pr_dtype;
                                 anything.  Only for callers whose inputs are complete before
                                 the preceding kernel starts (e.g. back-to-back verifier calls
                                 on resident logits).  Default 0. */
+#define PR_OPT_LMHEAD_CLUSTER 5 /* pr_lmhead_features' thread-block cluster: 0 = none (the
+                                default: measured fastest), or 11, 21, 12, 22 for cm x cs =
+                                1x1, 2x1, 1x2, 2x2 (cm CTAs share weight slices, cs share
+                                hidden-state slices through TMA multicast). */
 #define PR_OPT_TIMING 4      /* 1: the calls after the verifier's (pr_head_score,
                                 pr_quantile_score, pr_selective_metrics, pr_lmhead_features)
                                 record a CUDA event after each kernel, for

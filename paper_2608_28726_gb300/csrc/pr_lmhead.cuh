@@ -4,21 +4,29 @@
 // and reduced to the Eq. 3 row state in the epilogue, so they never reach
 // device memory.
 //
-//   lm_fused   grid (128-row tiles, vocabulary splits), 192 threads:
-//              warp 0   TMA producer: 64-wide K blocks of H (128 x 64) and W
-//                       (256 x 64), 128-byte swizzle, a 4-stage ring;
+//   lm_fused   grid (vocabulary splits, 256-row tiles), 320 threads:
+//              warp 0   TMA producer: 64-wide K blocks of H (256 x 64) and W
+//                       (256 x 64), 128-byte swizzle, a 3-stage ring;
 //              warp 1   TMEM owner and MMA issuer: tcgen05.mma kind::f16 (bf16
 //                       in, fp32 accumulate), M = 128, N = 256, K = 16 per
-//                       instruction, into one of two 128 x 256 fp32 TMEM
-//                       accumulators (512 columns);
-//              warps 2-5 epilogue: tcgen05.ld of a finished accumulator, one
-//                       row per thread, folded into the row's online (max,
+//                       instruction; the two 128-row halves of the tile share
+//                       each W block and accumulate into two 128 x 256 fp32
+//                       TMEM accumulators (all 512 columns);
+//              warps 2-9 epilogue: tcgen05.ld of the finished accumulators,
+//                       one row per thread, folded into the row's online (max,
 //                       sum of 2^t, sum of t 2^t) state, an exact running
 //                       top-KC list and the chosen token's logit; the state of
-//                       each (row, split) goes to a small buffer.
+//                       each (row, split) goes to a small buffer.  Each W
+//                       block is read once per 256 rows: half the L2 traffic
+//                       of 128-row tiles for the same MMA work.
 //   lm_merge   one warp per row: merges the splits' states in split order
 //              and writes the feature record with the verifier's own row
 //              finalisation (row_finish).
+// With a thread-block cluster of cm x cs CTAs, the cm CTAs of one split (same
+// W tiles, different rows) and the cs CTAs of one row tile (same H tiles,
+// different splits) each load a slice of the shared tile and multicast it;
+// each stage is released to every CTA that writes into it by a multicast
+// tcgen05.commit.  This divides the L2 traffic per MMA by up to four.
 // Every mbarrier wait is bounded (2 s of %globaltimer); a wait that runs out
 // sets an error flag and stops the CTA's loops; the producer then waits
 // (bounded) for its copies in flight, the MMA issuer for its own MMAs, and the
@@ -32,11 +40,13 @@
 
 namespace prk {
 
-constexpr int LM_BM = 128, LM_BN = 256, LM_BK = 64, LM_STAGES = 4;
-constexpr int LM_A_BYTES = LM_BM * LM_BK * 2;          // 16 KB
+constexpr int LM_BM = 256, LM_BN = 256, LM_BK = 64, LM_STAGES = 3;
+constexpr int LM_MH = 128;                             // rows per MMA (M)
+constexpr int LM_A_BYTES = LM_BM * LM_BK * 2;          // 32 KB
 constexpr int LM_B_BYTES = LM_BN * LM_BK * 2;          // 32 KB
 constexpr int LM_STAGE_BYTES = LM_A_BYTES + LM_B_BYTES;
-constexpr int LM_NT = 192;
+constexpr int LM_NT = 320;
+constexpr int LM_EPI_WARPS = 8;
 constexpr int LM_TMEM_COLS = 512;                      // two 256-column fp32 accumulators
 constexpr size_t LM_SMEM = (size_t)LM_STAGES * LM_STAGE_BYTES + 1024 + 256;
 constexpr uint64_t LM_WAIT_NS = 2000000000ull;         // a wait gives up after 2 s
@@ -46,7 +56,7 @@ constexpr uint32_t LM_ERR_TIMEOUT = 32u;                 // PR_FLAG_TIMEOUT in t
 // 4-5 = 1), bf16 A and B (bits 7-9, 10-12 = 1), both K-major (bits 15, 16 =
 // 0), N / 8 in bits 17-22, M / 16 in bits 24-28
 constexpr uint32_t LM_IDESC = (1u << 4) | (1u << 7) | (1u << 10) |
-                              ((uint32_t)(LM_BN >> 3) << 17) | ((uint32_t)(LM_BM >> 4) << 24);
+                              ((uint32_t)(LM_BN >> 3) << 17) | ((uint32_t)(LM_MH >> 4) << 24);
 
 struct LmPart {            // one row's state over one vocabulary split
   float m, S, U, xy;       // base-2 (m, S, U); the chosen token's logit if in range
@@ -57,6 +67,8 @@ struct LmPart {            // one row's state over one vocabulary split
 struct LmArgs {
   int64_t n_rows, vocab;
   int32_t d, kblocks, ntiles;
+  int32_t tiles_per_split;  // equal for every split (the last may run past V: masked)
+  int32_t cm, cs;           // cluster shape: CTAs sharing W slices (M), sharing H slices (split)
   const int32_t* chosen;
   LmPart* parts;           // [nsplit][n_rows]
   uint32_t* err;           // error word
@@ -122,6 +134,18 @@ __device__ __forceinline__ void lm_tma_load(const CUtensorMap* map, void* dst, u
       : "memory");
 }
 
+// the same load delivered to the CTAs of `mask` in the cluster: each receives
+// the box at the same shared-memory offset and the bytes on its own mbarrier
+// at the same offset
+__device__ __forceinline__ void lm_tma_load_mc(const CUtensorMap* map, void* dst, uint64_t* bar,
+                                               int x, int y, uint16_t mask) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      ".multicast::cluster [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(lm_smem(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(lm_smem(bar)), "h"(mask)
+      : "memory");
+}
+
 // shared-memory matrix descriptor of a K-major operand written by TMA with the
 // 128-byte swizzle: rows of 128 bytes (64 bf16), 8-row atoms of 1,024 bytes
 // (stride byte offset), start address >> 4 in bits 0-13, leading byte offset
@@ -145,6 +169,28 @@ __device__ __forceinline__ void lm_mma(uint32_t dtmem, uint64_t adesc, uint64_t 
       "l"(adesc), "l"(bdesc), "r"(LM_IDESC), "r"(accumulate)
       : "memory");
 }
+// arrive on the mbarrier (same offset) of every CTA in `mask` once every
+// tcgen05.mma this thread issued has completed
+__device__ __forceinline__ void lm_commit_mc(uint64_t* bar, uint16_t mask) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+      " [%0], %1;" ::"r"(lm_smem(bar)),
+      "h"(mask)
+      : "memory");
+}
+__device__ __forceinline__ void lm_cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::
+                   : "memory");
+}
+__device__ __forceinline__ uint32_t lm_cluster_id(int dim) {
+  uint32_t v;
+  if (dim == 0)
+    asm volatile("mov.u32 %0, %%cluster_ctaid.x;" : "=r"(v));
+  else
+    asm volatile("mov.u32 %0, %%cluster_ctaid.y;" : "=r"(v));
+  return v;
+}
+
 // arrive on the mbarrier once every tcgen05.mma this thread issued has completed
 __device__ __forceinline__ void lm_commit(uint64_t* bar) {
   asm volatile(
@@ -177,6 +223,20 @@ __device__ __forceinline__ void lm_tmem_ld32(uint32_t taddr, float (&v)[32]) {
   for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
 }
 
+// v[j] for a run-time j without indexing the register array (a select tree)
+__device__ __forceinline__ float lm_pick(const float (&v)[32], uint32_t j) {
+  float a[16], b[8], c[4], d[2];
+#pragma unroll
+  for (int i = 0; i < 16; ++i) a[i] = (j & 1u) ? v[2 * i + 1] : v[2 * i];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) b[i] = (j & 2u) ? a[2 * i + 1] : a[2 * i];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) c[i] = (j & 4u) ? b[2 * i + 1] : b[2 * i];
+#pragma unroll
+  for (int i = 0; i < 2; ++i) d[i] = (j & 8u) ? c[2 * i + 1] : c[2 * i];
+  return (j & 16u) ? d[1] : d[0];
+}
+
 // insert key k into the descending list L (L[KC-1] the smallest kept)
 template <int KC>
 __device__ __forceinline__ void lm_insert(uint64_t (&L)[KC], uint64_t k) {
@@ -199,25 +259,35 @@ __global__ void __launch_bounds__(LM_NT, 1)
                                            ~(uintptr_t)1023);
   uint64_t* full = reinterpret_cast<uint64_t*>(sm + LM_STAGES * LM_STAGE_BYTES);
   uint64_t* empty = full + LM_STAGES;
-  uint64_t* tfull = empty + LM_STAGES;
-  uint64_t* tempty = tfull + 2;
-  uint64_t* mdone = tempty + 2;  // the MMA issuer's own completion
+  uint64_t* tfull = empty + LM_STAGES;   // both accumulators hold a finished tile
+  uint64_t* tempty = tfull + 1;          // the epilogue has read them
+  uint64_t* mdone = tempty + 1;          // the MMA issuer's own completion
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mdone + 1);
   volatile uint32_t* abort_ = tmem_slot + 1;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int mt = blockIdx.x, split = blockIdx.y, nsplit = gridDim.y;
-  const int t0 = (int)((int64_t)split * a.ntiles / nsplit);
-  const int t1 = (int)((int64_t)(split + 1) * a.ntiles / nsplit);
+  // grid x = vocabulary split (fastest), y = 256-row tile: a wave of CTAs covers a
+  // few row tiles across all splits, so the H tiles it re-reads and the W tiles
+  // it streams together fit in L2
+  const int split = blockIdx.x, mt = blockIdx.y;
+  const int t0 = split * a.tiles_per_split, t1 = t0 + a.tiles_per_split;
+  // cluster position (cluster dims cs x cm): pm along the rows (CTAs with the
+  // same ps share W slices, cm of them), ps along the splits (CTAs with the same
+  // pm share H slices, cs of them); rank = ps + pm cs
+  const int ps = a.cs > 1 ? (int)lm_cluster_id(0) : 0;
+  const int pm = a.cm > 1 ? (int)lm_cluster_id(1) : 0;
+  uint16_t mask_h = 0, mask_w = 0;  // CTAs receiving my H slice / my W slice
+  for (int s2 = 0; s2 < a.cs; ++s2) mask_h |= (uint16_t)(1u << (s2 + pm * a.cs));
+  for (int m2 = 0; m2 < a.cm; ++m2) mask_w |= (uint16_t)(1u << (ps + m2 * a.cs));
+  const uint16_t mask_rel = mask_h | mask_w;  // writers into my stages = readers of mine
+  const bool clustered = a.cm * a.cs > 1;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < LM_STAGES; ++s) {
       lm_mbar_init(full + s, 1);
-      lm_mbar_init(empty + s, 1);
+      lm_mbar_init(empty + s, (uint32_t)(a.cm + a.cs - 1));  // one release per writer's reader
     }
-    for (int b = 0; b < 2; ++b) {
-      lm_mbar_init(tfull + b, 1);
-      lm_mbar_init(tempty + b, 4);  // one arrival per epilogue warp
-    }
+    lm_mbar_init(tfull, 1);
+    lm_mbar_init(tempty, LM_EPI_WARPS);  // one arrival per epilogue warp
     lm_mbar_init(mdone, 1);
     *abort_ = 0u;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -231,6 +301,7 @@ __global__ void __launch_bounds__(LM_NT, 1)
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
   __syncthreads();
+  if (clustered) lm_cluster_sync();  // every CTA's barriers exist before any remote use
   lm_fence_after();
   const uint32_t tmem = *tmem_slot;
 
@@ -246,9 +317,17 @@ __global__ void __launch_bounds__(LM_NT, 1)
             break;
           }
           uint8_t* st = sm + s * LM_STAGE_BYTES;
-          lm_mbar_expect(full + s, LM_STAGE_BYTES);
-          lm_tma_load(&tmA, st, full + s, kb * LM_BK, mt * LM_BM);
-          lm_tma_load(&tmB, st + LM_A_BYTES, full + s, kb * LM_BK, t * LM_BN);
+          lm_mbar_expect(full + s, LM_STAGE_BYTES);  // all slices, from every writer
+          if (!clustered) {
+            lm_tma_load(&tmA, st, full + s, kb * LM_BK, mt * LM_BM);
+            lm_tma_load(&tmB, st + LM_A_BYTES, full + s, kb * LM_BK, t * LM_BN);
+          } else {
+            const int ha = LM_BM / a.cs, wb = LM_BN / a.cm;  // slice rows
+            lm_tma_load_mc(&tmA, st + ps * ha * 128, full + s, kb * LM_BK, mt * LM_BM + ps * ha,
+                           mask_h);
+            lm_tma_load_mc(&tmB, st + LM_A_BYTES + pm * wb * 128, full + s, kb * LM_BK,
+                           t * LM_BN + pm * wb, mask_w);
+          }
         }
       // the copies still in flight land before the CTA exits (already true
       // unless a wait gave up): wait, bounded, for the last stages' loads
@@ -261,11 +340,9 @@ __global__ void __launch_bounds__(LM_NT, 1)
     if (lane == 0) {  // ---- MMA issuer
       int it = 0;
       for (int i = 0, t = t0; t < t1 && !*abort_; ++t, ++i) {
-        const int buf = i & 1;
-        const uint32_t use = (uint32_t)(i >> 1);
-        if (!lm_wait(tempty + buf, (use & 1u) ^ 1u, abort_, a.err)) break;
+        // the epilogue has read the previous tile out of both accumulators
+        if (!lm_wait(tempty, ((uint32_t)i & 1u) ^ 1u, abort_, a.err)) break;
         lm_fence_after();
-        const uint32_t dt = tmem + (uint32_t)(buf * LM_BN);
         bool ok = true;
         for (int kb = 0; kb < a.kblocks; ++kb, ++it) {
           const int s = it % LM_STAGES;
@@ -277,82 +354,106 @@ __global__ void __launch_bounds__(LM_NT, 1)
           lm_fence_after();
           const uint32_t sa = lm_smem(sm + s * LM_STAGE_BYTES), sb = sa + LM_A_BYTES;
 #pragma unroll
-          for (int k = 0; k < LM_BK / 16; ++k)  // K = 16 per MMA: 32 bytes along the row
-            lm_mma(dt, lm_sdesc(sa + 32 * k), lm_sdesc(sb + 32 * k), (kb | k) != 0 ? 1u : 0u);
-          lm_commit(empty + s);  // the stage is free once these MMAs have read it
+          for (int k = 0; k < LM_BK / 16; ++k) {  // K = 16 per MMA: 32 bytes along the row
+            const uint64_t bd = lm_sdesc(sb + 32 * k);
+            const uint32_t acc = (kb | k) != 0 ? 1u : 0u;
+            lm_mma(tmem, lm_sdesc(sa + 32 * k), bd, acc);                       // rows 0-127
+            lm_mma(tmem + LM_BN, lm_sdesc(sa + LM_MH * 128 + 32 * k), bd, acc);  // rows 128-255
+          }
+          // the stage is free, in every CTA that writes into it, once these MMAs
+          // have read it
+          if (clustered)
+            lm_commit_mc(empty + s, mask_rel);
+          else
+            lm_commit(empty + s);
         }
         if (!ok) break;
-        lm_commit(tfull + buf);
+        lm_commit(tfull);
       }
       // every MMA this thread issued has completed before TMEM is freed
       lm_commit(mdone);
       volatile uint32_t no_abort = 0u;
       lm_wait(mdone, 0u, &no_abort, a.err);
     }
-  } else {  // ---- epilogue: warps 2..5, TMEM lanes 32 (warp % 4) ..
-    const int q = warp & 3;
-    const int64_t row = (int64_t)mt * LM_BM + 32 * q + lane;
+  } else {  // ---- epilogue: warps 2..9, TMEM lanes 32 (warp % 4) .., accumulator h
+    const int q = warp & 3, h = (warp - 2) >> 2;
+    const int64_t row = (int64_t)mt * LM_BM + LM_MH * h + 32 * q + lane;
     const bool live = row < a.n_rows;
     const int32_t y = live ? a.chosen[row] : -1;
-    float m = M2_INIT, S = 0.f, U = 0.f, xy = NAN;
+    const int32_t V = (int32_t)a.vocab;
+    float m = M2_INIT, xy = NAN;
+    float2 S2 = make_float2(0.f, 0.f), U2 = make_float2(0.f, 0.f);  // even / odd columns
     bool bad = false, has_y = false;
     uint64_t L[KC];
 #pragma unroll
     for (int j = 0; j < KC; ++j) L[j] = 0ull;
+    float thr = -INFINITY;  // value of the KC-th key kept (-inf while the list is not full)
     for (int i = 0, t = t0; t < t1; ++t, ++i) {
-      const int buf = i & 1;
-      const uint32_t use = (uint32_t)(i >> 1);
       int ok = 1;
-      if (lane == 0) ok = lm_wait(tfull + buf, use & 1u, abort_, a.err) ? 1 : 0;
+      if (lane == 0) ok = lm_wait(tfull, (uint32_t)i & 1u, abort_, a.err) ? 1 : 0;
       ok = __shfl_sync(FULL, ok, 0);  // the warp stays converged for tcgen05.ld
       if (!ok) break;
       lm_fence_after();
-      const uint32_t tbase = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * LM_BN);
+      const uint32_t tbase = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(h * LM_BN);
       for (int c = 0; c < LM_BN / 32; ++c) {
         float v[32];
         lm_tmem_ld32(tbase + 32 * c, v);
-        const int64_t col0 = (int64_t)t * LM_BN + 32 * c;
-        // masked columns (past the vocabulary) count as -inf
-        float cmax = -INFINITY;
+        const int32_t col0 = t * LM_BN + 32 * c;
+        const bool whole = col0 + 32 <= V;  // false only in the last vocabulary tile
+        if (!whole) {
 #pragma unroll
-        for (int j = 0; j < 32; ++j) {
-          if (col0 + j >= a.vocab) v[j] = -INFINITY;
-          if (isnan(v[j]) || v[j] == INFINITY) bad = true;
-          cmax = fmaxf(cmax, v[j]);
+          for (int j = 0; j < 32; ++j)
+            if (col0 + j >= V) v[j] = -INFINITY;
         }
+        float cmax = v[0];
+#pragma unroll
+        for (int j = 1; j < 32; ++j) cmax = fmaxf(cmax, v[j]);
+        if (cmax == INFINITY) bad = true;  // NaN reaches S and U and is flagged there
         const float tm = cmax * L2E;
         if (tm > m) {
-          if (S != 0.f) {
-            const float dl = m - tm, f = ex2(dl);
-            U = f * fmaf(dl, S, U);
-            S *= f;
-          }
+          const float dl = m - tm, f = ex2(dl);
+          const float2 f2 = make_float2(f, f), dl2 = make_float2(dl, dl);
+          U2 = __fmul2_rn(f2, __ffma2_rn(dl2, S2, U2));
+          S2 = __fmul2_rn(S2, f2);
           m = tm;
         }
+        const float2 nm = make_float2(-m, -m), l2e = make_float2(L2E, L2E);
+        const float2 lo2 = make_float2(-1e30f, -1e30f);
 #pragma unroll
-        for (int j = 0; j < 32; ++j) {
-          const float dd = fmaxf(fmaf(v[j], L2E, -m), -1e30f);  // -inf -> a finite 0 weight
-          const float e = ex2(dd);
-          S += e;
-          U = fmaf(e, dd, U);
+        for (int j = 0; j < 32; j += 2) {
+          float2 dd = __ffma2_rn(make_float2(v[j], v[j + 1]), l2e, nm);
+          if (!whole) dd = make_float2(fmaxf(dd.x, lo2.x), fmaxf(dd.y, lo2.y));  // -inf -> 0 weight
+          const float2 e = make_float2(ex2(dd.x), ex2(dd.y));
+          S2 = __fadd2_rn(S2, e);
+          U2 = __ffma2_rn(e, dd, U2);
         }
+        // chosen token: one chunk of the whole sweep holds it
+        const uint32_t yo = (uint32_t)(y - col0);
+        if (yo < 32u && (int32_t)yo + col0 < V) {
+          xy = lm_pick(v, yo);
+          has_y = true;
+        }
+        // top-KC: only chunks whose maximum reaches the list's threshold
+        if (cmax >= thr) {
+          uint32_t mask = 0u;
 #pragma unroll
-        for (int j = 0; j < 32; ++j) {  // fully unrolled: v stays in registers
-          const int64_t col = col0 + j;
-          if (col < a.vocab) {
-            const uint64_t k = make_key(v[j], (uint32_t)col);
-            if (k > L[KC - 1]) lm_insert<KC>(L, k);
-            if (col == y) {
-              xy = v[j];
-              has_y = true;
+          for (int j = 0; j < 32; ++j) mask |= (v[j] >= thr && col0 + j < V ? 1u : 0u) << j;
+          while (mask) {
+            const uint32_t j = (uint32_t)__ffs(mask) - 1u;
+            mask &= mask - 1u;
+            const uint64_t k = make_key(lm_pick(v, j), (uint32_t)(col0 + (int32_t)j));
+            if (k > L[KC - 1]) {
+              lm_insert<KC>(L, k);
+              if (L[KC - 1] != 0ull) thr = key_val(L[KC - 1]);
             }
           }
         }
       }
       lm_fence_before();
       __syncwarp();
-      if (lane == 0) lm_mbar_arrive(tempty + buf);
+      if (lane == 0) lm_mbar_arrive(tempty);
     }
+    const float S = S2.x + S2.y, U = U2.x + U2.y;
     if (live) {
       LmPart* p = a.parts + (int64_t)split * a.n_rows + row;
       p->m = m;
@@ -366,6 +467,7 @@ __global__ void __launch_bounds__(LM_NT, 1)
     }
   }
   __syncthreads();
+  if (clustered) lm_cluster_sync();  // no CTA leaves while others may still write into it
   if (warp == 1) {
     lm_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),

@@ -76,15 +76,47 @@ pr_status pr_lmhead_features(pr_ctx* c, const void* hidden, const void* weight, 
                                  (int)prk::LM_SMEM));
     c->lm_ready = true;
   }
-  CUtensorMap ma, mb;
-  if (!make_map(&ma, hidden, n_rows, d, prk::LM_BM) || !make_map(&mb, weight, vocab, d, prk::LM_BN))
-    return PR_ERR_UNSUPPORTED;
   const int64_t mtiles = (n_rows + prk::LM_BM - 1) / prk::LM_BM;
   const int64_t ntiles = (vocab + prk::LM_BN - 1) / prk::LM_BN;
   if (mtiles > 0x7fffffffLL) return PR_ERR_INVALID_ARG;
-  // vocabulary splits: about one CTA per SM in total
-  const int64_t nsplit =
-      std::max<int64_t>(1, std::min<int64_t>(ntiles, (c->num_sms + mtiles / 2) / mtiles));
+  const int kc = topk > 2 ? topk : 2;
+  const void* kern = kc <= 20 ? reinterpret_cast<const void*>(&prk::lm_fused<20>)
+                              : reinterpret_cast<const void*>(&prk::lm_fused<32>);
+  // Launch shape.  Splits of the vocabulary run along grid x (fastest), 256-row
+  // tiles along y, so a wave of one CTA per SM covers num_sms / nsplit row
+  // tiles across all splits; nsplit near sqrt(num_sms) keeps a wave's H tiles
+  // plus its in-flight W tiles small (~25 tiles of 1.8 MB), and among those the
+  // count with the least idle tail in the last wave is taken.  Thread-block
+  // clusters (cm x cs CTAs sharing W / H slices through TMA multicast) only when
+  // forced: measured slower, since every stage then waits for its slowest reader.
+  int cm = 1, cs = 1;
+  if (c->lm_force) {
+    cm = c->lm_force / 10;
+    cs = c->lm_force % 10;
+  }
+  const int64_t mt_pad = (mtiles + cm - 1) / cm * cm;
+  int64_t nsplit = 1;
+  {
+    double best = 1e30;
+    for (int64_t ns = std::max<int64_t>(cs, 8); ns <= 24; ns += cs) {
+      if (ns > (ntiles + cs - 1) / cs * cs) break;
+      const int64_t ctas = mt_pad * ns;
+      const int64_t waves = (ctas + c->num_sms - 1) / c->num_sms;
+      const double waste = (double)(waves * c->num_sms - ctas) / (double)(waves * c->num_sms);
+      const double score = waste + 0.002 * std::abs((double)ns - 12.0);
+      if (score < best) {
+        best = score;
+        nsplit = ns;
+      }
+    }
+    if (best == 1e30) nsplit = std::max<int64_t>(cs, std::min<int64_t>(ntiles, c->num_sms / mt_pad) / cs * cs);
+    if (nsplit < 1) nsplit = cs;
+  }
+  const int64_t per_split = (ntiles + nsplit - 1) / nsplit;
+  CUtensorMap ma, mb;
+  if (!make_map(&ma, hidden, n_rows, d, (uint32_t)(prk::LM_BM / cs)) ||
+      !make_map(&mb, weight, vocab, d, (uint32_t)(prk::LM_BN / cm)))
+    return PR_ERR_UNSUPPORTED;
   const size_t part_bytes = (size_t)nsplit * (size_t)n_rows * sizeof(prk::LmPart);
   if (part_bytes > c->lm_parts_bytes) {
     PR_CUDA(cudaDeviceSynchronize());  // the old buffer may still be in use
@@ -107,16 +139,28 @@ pr_status pr_lmhead_features(pr_ctx* c, const void* hidden, const void* weight, 
   la.d = (int32_t)d;
   la.kblocks = (int32_t)((d + prk::LM_BK - 1) / prk::LM_BK);
   la.ntiles = (int32_t)ntiles;
+  la.tiles_per_split = (int32_t)per_split;
+  la.cm = cm;
+  la.cs = cs;
   la.chosen = chosen;
   la.parts = static_cast<prk::LmPart*>(c->lm_parts);
   la.err = c->flags;
-  const int kc = topk > 2 ? topk : 2;
-  const dim3 grid((unsigned)mtiles, (unsigned)nsplit);
-  if (kc <= 20)
-    prk::lm_fused<20><<<grid, prk::LM_NT, prk::LM_SMEM, s>>>(ma, mb, la);
-  else
-    prk::lm_fused<32><<<grid, prk::LM_NT, prk::LM_SMEM, s>>>(ma, mb, la);
-  PR_CUDA(cudaGetLastError());
+  cudaLaunchConfig_t cfg;
+  memset(&cfg, 0, sizeof cfg);
+  cfg.gridDim = dim3((unsigned)nsplit, (unsigned)mt_pad);
+  cfg.blockDim = dim3(prk::LM_NT);
+  cfg.dynamicSmemBytes = prk::LM_SMEM;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = (unsigned)cs;
+  attr[0].val.clusterDim.y = (unsigned)cm;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = cm * cs > 1 ? 1 : 0;
+  void* kargs[] = {&ma, &mb, &la};
+  PR_CUDA(cudaLaunchKernelExC(&cfg, kern, kargs));
+  c->lm_cluster = cm * 10 + cs;
   if ((st = timing_mark(c, s)) != PR_OK) return st;
   prk::Args a;
   memset(&a, 0, sizeof a);

@@ -346,3 +346,30 @@ def qmlp_weights(seed: int = 6001) -> np.ndarray:
     w = np.concatenate(parts).astype(np.float32)
     assert w.size == qmlp_param_count()
     return w
+
+
+# ---- LM-head inputs --------------------------------------------------------------------
+
+def lmhead_inputs(n_rows: int, d: int = 3584, vocab: int = 151936, seed: int = 8001,
+                  device="cuda"):
+    """Seeded stand-ins for the small model's final hidden states and LM head
+    (trained weights are not available): hidden bf16 [n_rows][d] with N(0, 1)
+    entries and a per-row scale U(0.5, 2); weight bf16 [vocab][d] with
+    N(0, (2 / sqrt(d))^2) entries, so the logits have a scale of a few units;
+    emitted token ids uniform in [0, vocab).  d = 3,584 is the hidden size the
+    paper quotes for the small model (Table 2)."""
+    dev = torch.device(device)
+    g = torch.Generator(device=dev)
+    g.manual_seed(seed)
+    h = torch.randn(n_rows, d, generator=g, device=dev)
+    h *= 0.5 + 1.5 * torch.rand(n_rows, 1, generator=g, device=dev)
+    hidden = h.to(torch.bfloat16)
+    del h
+    weight = torch.empty(vocab, d, dtype=torch.bfloat16, device=dev)
+    step = 8192
+    for v0 in range(0, vocab, step):  # in slices: no fp32 copy of the whole matrix
+        v1 = min(vocab, v0 + step)
+        weight[v0:v1] = (torch.randn(v1 - v0, d, generator=g, device=dev) *
+                         (2.0 / d ** 0.5)).to(torch.bfloat16)
+    chosen = torch.randint(0, vocab, (n_rows,), generator=g, device=dev, dtype=torch.int32)
+    return hidden, weight, chosen

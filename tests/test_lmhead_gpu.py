@@ -98,6 +98,17 @@ def test_lmhead_flags_and_rho(B, ctx):
     assert np.isnan(fg[3, 0]) and np.isnan(fg[7, 0])
 
 
+@pytest.mark.parametrize("shape", [11, 21, 12, 22])
+def test_lmhead_cluster_shapes(B, ctx, shape):
+    """Every cluster shape (cm CTAs sharing weight slices x cs sharing hidden
+    slices through TMA multicast) gives the same records."""
+    B.pr_ctx_set_option(ctx, B.PR_OPT_LMHEAD_CLUSTER, shape)
+    try:
+        check(B, ctx, 600, 320, 7000, seed=40 + shape)
+    finally:
+        B.pr_ctx_set_option(ctx, B.PR_OPT_LMHEAD_CLUSTER, 0)
+
+
 def test_lmhead_large_vocab_and_hidden(B, ctx):
     """d = 3,584 (the small model's hidden size) and V = 151,936 on a few rows."""
     check(B, ctx, 8, 3584, 151936, seed=7)
