@@ -109,10 +109,6 @@ typedef enum { PR_DTYPE_F32 = 0, PR_DTYPE_BF16 = 1 } pr_dtype;
                                 anything.  Only for callers whose inputs are complete before
                                 the preceding kernel starts (e.g. back-to-back verifier calls
                                 on resident logits).  Default 0. */
-#define PR_OPT_LMHEAD_CLUSTER 5 /* pr_lmhead_features' thread-block cluster: 0 = none (the
-                                default: measured fastest), or 11, 21, 12, 22 for cm x cs =
-                                1x1, 2x1, 1x2, 2x2 (cm CTAs share weight slices, cs share
-                                hidden-state slices through TMA multicast). */
 #define PR_OPT_TIMING 4      /* 1: the calls after the verifier's (pr_head_score,
                                 pr_quantile_score, pr_selective_metrics, pr_lmhead_features)
                                 record a CUDA event after each kernel, for
@@ -329,7 +325,8 @@ pr_status pr_head_score(pr_ctx* ctx, const float* feat, const uint32_t* row_flag
  *   chosen, topk, offsets, n_req, feat, top2, row_flags: as pr_token_features
  * The record has pr_token_features' slots and conventions, computed from the
  * fp32 logits; uses the context's PR_OPT_TOPK_RENORM.  Two launches on
- * `stream`; the context holds a state buffer of 288 bytes per row and
+ * `stream` (the first in thread-block clusters of two CTAs sharing each
+ * tcgen05 MMA); the context holds a state buffer of 576 bytes per row and
  * vocabulary split (grown on demand; that call synchronises the device).  A
  * device-side wait that runs out (2 s) raises PR_FLAG_TIMEOUT in the context
  * flag word.

@@ -21,7 +21,6 @@ PR_FLAG_NONFINITE, PR_FLAG_BAD_CHOSEN, PR_FLAG_EMPTY_REQ = 1, 2, 4
 PR_FLAG_BAD_OFFSETS, PR_FLAG_BAD_SLOT, PR_FLAG_TIMEOUT = 8, 16, 32
 PR_NFEAT, PR_NAGG, PR_MAX_TOPK = 8, 11, 32
 PR_OPT_TOPK, PR_OPT_TOPK_RENORM, PR_OPT_SPLIT, PR_OPT_OVERLAP, PR_OPT_TIMING = 0, 1, 2, 3, 4
-PR_OPT_LMHEAD_CLUSTER = 5
 PR_NOALLOC_MAX_ROWS, PR_NOALLOC_MAX_REQUESTS = 16384, 1024
 PR_HEAD_D, PR_HEAD_HEADS, PR_HEAD_FF, PR_HEAD_MAX_LAYERS = 64, 4, 128, 8
 PR_QMLP_SUMMARY, PR_QMLP_PARAMS = 28, 6081

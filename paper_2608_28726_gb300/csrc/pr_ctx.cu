@@ -193,11 +193,6 @@ pr_status pr_ctx_set_option(pr_ctx* c, int32_t option, int32_t value) {
       if (value != 0 && value != 1) return PR_ERR_INVALID_ARG;
       c->timing = value;
       return PR_OK;
-    case PR_OPT_LMHEAD_CLUSTER:
-      if (value != 0 && value != 11 && value != 21 && value != 12 && value != 22)
-        return PR_ERR_INVALID_ARG;
-      c->lm_force = value;
-      return PR_OK;
   }
   return PR_ERR_INVALID_ARG;
 }

@@ -54,8 +54,6 @@ struct pr_ctx {
   void* lm_parts = nullptr;
   size_t lm_parts_bytes = 0;
   bool lm_ready = false;
-  int lm_cluster = 0;     // cluster shape of the last launch (10 cm + cs), for diagnostics
-  int lm_force = 0;       // PR_OPT_LMHEAD_CLUSTER
   // PR_OPT_TIMING: events after each kernel of the last multi-kernel call
   int32_t timing = 0;
   cudaEvent_t tev[PR_MAX_TIMED + 1] = {};

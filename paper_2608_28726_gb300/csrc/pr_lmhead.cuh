@@ -4,33 +4,43 @@
 // and reduced to the Eq. 3 row state in the epilogue, so they never reach
 // device memory.
 //
-//   lm_fused   grid (vocabulary splits, 256-row tiles), 320 threads:
-//              warp 0   TMA producer: 64-wide K blocks of H (256 x 64) and W
-//                       (256 x 64), 128-byte swizzle, a 3-stage ring;
-//              warp 1   TMEM owner and MMA issuer: tcgen05.mma kind::f16 (bf16
-//                       in, fp32 accumulate), M = 128, N = 256, K = 16 per
-//                       instruction; the two 128-row halves of the tile share
-//                       each W block and accumulate into two 128 x 256 fp32
-//                       TMEM accumulators (all 512 columns);
-//              warps 2-9 epilogue: tcgen05.ld of the finished accumulators,
-//                       one row per thread, folded into the row's online (max,
-//                       sum of 2^t, sum of t 2^t) state, an exact running
-//                       top-KC list and the chosen token's logit; the state of
-//                       each (row, split) goes to a small buffer.  Each W
-//                       block is read once per 256 rows: half the L2 traffic
-//                       of 128-row tiles for the same MMA work.
-//   lm_merge   one warp per row: merges the splits' states in split order
+//   lm_fused   2 x (row pairs x vocabulary splits) CTAs in thread-block
+//              clusters of two along x, 320 threads; a pair (256 rows, one
+//              split) per cluster, in bands of row pairs: a wave streams few
+//              splits' W tiles past one band's H rows, both held in L2.
+//              The pair shares one tcgen05.mma of M = 256 (cta_group::2):
+//              the CTA of rank r holds rows 128 r .. of the pair's 256 rows
+//              of H and rows 128 r .. of each 256-row tile of W, and its TMEM
+//              receives its own 128 rows of the 256 x 256 logit tile.
+//              warp 0   (both CTAs) TMA producer: K blocks of 128 (two boxes
+//                       of 64 with the 128-byte swizzle) of its H rows and W
+//                       half tile, a 3-stage ring of 64 KB stages; every load
+//                       completes on the rank-0 CTA's stage barrier, which
+//                       expects the bytes of both CTAs;
+//              warp 1   owns the pair's TMEM (allocated by both CTAs
+//                       together); in the rank-0 CTA it issues the MMAs (bf16
+//                       in, fp32 accumulate, K = 16 each, 8 per stage) into
+//                       one of two 256-column accumulators, so tile i + 1
+//                       accumulates while the epilogue reads tile i, and
+//                       releases stages and finished tiles to both CTAs by a
+//                       multicast tcgen05.commit;
+//              warps 2-9 (both CTAs) epilogue: warp w reads TMEM lanes 32 (w %
+//                       4) .. and one 128-column half of the tile, one row per
+//                       thread, folded into the row's online (max, sum of 2^t,
+//                       sum of t 2^t) state, an exact running top-KC list and
+//                       the chosen token's logit; each warp reports a read
+//                       accumulator to the rank-0 CTA; the state of each (row,
+//                       split, half) goes to a small buffer.
+//              A W block is read from L2 once per 256 rows, an H block once
+//              per 256 vocabulary columns.
+//   lm_merge   one warp per row: merges the parts' states in split order
 //              and writes the feature record with the verifier's own row
 //              finalisation (row_finish).
-// With a thread-block cluster of cm x cs CTAs, the cm CTAs of one split (same
-// W tiles, different rows) and the cs CTAs of one row tile (same H tiles,
-// different splits) each load a slice of the shared tile and multicast it;
-// each stage is released to every CTA that writes into it by a multicast
-// tcgen05.commit.  This divides the L2 traffic per MMA by up to four.
 // Every mbarrier wait is bounded (2 s of %globaltimer); a wait that runs out
-// sets an error flag and stops the CTA's loops; the producer then waits
-// (bounded) for its copies in flight, the MMA issuer for its own MMAs, and the
-// CTA frees its TMEM before it exits.
+// sets an error flag and stops that role's loop; the roles of the other CTA
+// then run out of their own waits, the rank-0 producer waits (bounded) for
+// the copies in flight, the MMA issuer for its own MMAs, and both CTAs free
+// the pair's TMEM together before they exit.
 #pragma once
 
 #include <cuda.h>
@@ -40,13 +50,18 @@
 
 namespace prk {
 
-constexpr int LM_BM = 256, LM_BN = 256, LM_BK = 64, LM_STAGES = 3;
-constexpr int LM_MH = 128;                             // rows per MMA (M)
-constexpr int LM_A_BYTES = LM_BM * LM_BK * 2;          // 32 KB
-constexpr int LM_B_BYTES = LM_BN * LM_BK * 2;          // 32 KB
+constexpr int LM_BM = 128;                             // rows of H per CTA (256 per pair)
+constexpr int LM_BN = 256;                             // vocabulary columns per tile (MMA N)
+constexpr int LM_BK = 128;                             // K per stage: two 64-wide swizzle boxes
+constexpr int LM_STAGES = 3;
+constexpr int LM_A_BYTES = LM_BM * LM_BK * 2;          // 32 KB: this CTA's rows of H
+constexpr int LM_B_BYTES = (LM_BN / 2) * LM_BK * 2;    // 32 KB: this CTA's half of the W tile
+constexpr int LM_BOX_K = 64;                           // box width: one 128-byte swizzle row
+constexpr int LM_BOX_BYTES = 128 * LM_BOX_K * 2;       // one 128-row box
 constexpr int LM_STAGE_BYTES = LM_A_BYTES + LM_B_BYTES;
 constexpr int LM_NT = 320;
 constexpr int LM_EPI_WARPS = 8;
+constexpr int LM_HALVES = 2;                           // column halves of a tile (epilogue)
 constexpr int LM_TMEM_COLS = 512;                      // two 256-column fp32 accumulators
 constexpr size_t LM_SMEM = (size_t)LM_STAGES * LM_STAGE_BYTES + 1024 + 256;
 constexpr uint64_t LM_WAIT_NS = 2000000000ull;         // a wait gives up after 2 s
@@ -54,11 +69,11 @@ constexpr uint32_t LM_ERR_TIMEOUT = 32u;                 // PR_FLAG_TIMEOUT in t
 
 // instruction descriptor of tcgen05.mma kind::f16: fp32 accumulator (bits
 // 4-5 = 1), bf16 A and B (bits 7-9, 10-12 = 1), both K-major (bits 15, 16 =
-// 0), N / 8 in bits 17-22, M / 16 in bits 24-28
+// 0), N / 8 in bits 17-22, M / 16 in bits 24-28 (M = 256: the pair's rows)
 constexpr uint32_t LM_IDESC = (1u << 4) | (1u << 7) | (1u << 10) |
-                              ((uint32_t)(LM_BN >> 3) << 17) | ((uint32_t)(LM_MH >> 4) << 24);
+                              ((uint32_t)(LM_BN >> 3) << 17) | ((uint32_t)((2 * LM_BM) >> 4) << 24);
 
-struct LmPart {            // one row's state over one vocabulary split
+struct LmPart {            // one row's state over one column half of one vocabulary split
   float m, S, U, xy;       // base-2 (m, S, U); the chosen token's logit if in range
   uint32_t bad, has_y, pad0, pad1;
   uint64_t top[32];        // descending keys (value, lower index first); 0 = empty
@@ -67,10 +82,11 @@ struct LmPart {            // one row's state over one vocabulary split
 struct LmArgs {
   int64_t n_rows, vocab;
   int32_t d, kblocks, ntiles;
-  int32_t tiles_per_split;  // equal for every split (the last may run past V: masked)
-  int32_t cm, cs;           // cluster shape: CTAs sharing W slices (M), sharing H slices (split)
+  int32_t tiles_per_split;  // the last split stops at the last tile
+  int32_t nsplit, npairs;   // vocabulary splits; 256-row pairs (CTA pairs per split)
+  int32_t band;             // row pairs per band of the launch order
   const int32_t* chosen;
-  LmPart* parts;           // [nsplit][n_rows]
+  LmPart* parts;           // [nsplit][LM_HALVES][n_rows]
   uint32_t* err;           // error word
 };
 
@@ -123,29 +139,6 @@ __device__ __forceinline__ bool lm_wait(uint64_t* b, uint32_t parity, volatile u
   return false;
 }
 
-// 2-D TMA load of a box at (x = K element, y = row) into shared memory,
-// completing bytes on the mbarrier
-__device__ __forceinline__ void lm_tma_load(const CUtensorMap* map, void* dst, uint64_t* bar,
-                                            int x, int y) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%2, %3}], [%4];" ::"r"(lm_smem(dst)),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(lm_smem(bar))
-      : "memory");
-}
-
-// the same load delivered to the CTAs of `mask` in the cluster: each receives
-// the box at the same shared-memory offset and the bytes on its own mbarrier
-// at the same offset
-__device__ __forceinline__ void lm_tma_load_mc(const CUtensorMap* map, void* dst, uint64_t* bar,
-                                               int x, int y, uint16_t mask) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
-      ".multicast::cluster [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(lm_smem(dst)),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(lm_smem(bar)), "h"(mask)
-      : "memory");
-}
-
 // shared-memory matrix descriptor of a K-major operand written by TMA with the
 // 128-byte swizzle: rows of 128 bytes (64 bf16), 8-row atoms of 1,024 bytes
 // (stride byte offset), start address >> 4 in bits 0-13, leading byte offset
@@ -160,49 +153,45 @@ __device__ __forceinline__ uint64_t lm_sdesc(uint32_t saddr) {
   return d;
 }
 
-__device__ __forceinline__ void lm_mma(uint32_t dtmem, uint64_t adesc, uint64_t bdesc,
-                                       uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(dtmem),
-      "l"(adesc), "l"(bdesc), "r"(LM_IDESC), "r"(accumulate)
-      : "memory");
-}
-// arrive on the mbarrier (same offset) of every CTA in `mask` once every
-// tcgen05.mma this thread issued has completed
-__device__ __forceinline__ void lm_commit_mc(uint64_t* bar, uint16_t mask) {
-  asm volatile(
-      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
-      " [%0], %1;" ::"r"(lm_smem(bar)),
-      "h"(mask)
-      : "memory");
-}
 __device__ __forceinline__ void lm_cluster_sync() {
   asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::
                    : "memory");
 }
-__device__ __forceinline__ uint32_t lm_cluster_id(int dim) {
+__device__ __forceinline__ uint32_t lm_cluster_x() {
   uint32_t v;
-  if (dim == 0)
-    asm volatile("mov.u32 %0, %%cluster_ctaid.x;" : "=r"(v));
-  else
-    asm volatile("mov.u32 %0, %%cluster_ctaid.y;" : "=r"(v));
+  asm volatile("mov.u32 %0, %%cluster_ctaid.x;" : "=r"(v));
   return v;
 }
 
-// arrive on the mbarrier once every tcgen05.mma this thread issued has completed
-__device__ __forceinline__ void lm_commit(uint64_t* bar) {
-  asm volatile(
-      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-          lm_smem(bar))
-      : "memory");
-}
 __device__ __forceinline__ void lm_fence_before() {
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
 }
 __device__ __forceinline__ void lm_fence_after() {
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+// ---- CTA-pair forms (tcgen05 cta_group::2)
+
+// shared::cluster address of the same variable in the CTA of the given rank
+__device__ __forceinline__ uint32_t lm_mapa(const void* p, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(lm_smem(p)), "r"(rank));
+  return r;
+}
+// 2-D TMA load into this CTA's shared memory whose completion is counted on an
+// mbarrier of either CTA of the pair (a shared::cluster address)
+__device__ __forceinline__ void lm_tma_load_pair(const CUtensorMap* map, void* dst, uint32_t bar,
+                                                 int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3}], [%4];" ::"r"(lm_smem(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+      : "memory");
+}
+// arrive on an mbarrier of another CTA of the cluster (release at cluster scope)
+__device__ __forceinline__ void lm_arrive_remote(uint32_t bar) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar)
+               : "memory");
 }
 
 // 32 consecutive fp32 columns of this warp's 32 TMEM lanes (lane = row)
@@ -237,18 +226,122 @@ __device__ __forceinline__ float lm_pick(const float (&v)[32], uint32_t j) {
   return (j & 16u) ? d[1] : d[0];
 }
 
-// insert key k into the descending list L (L[KC-1] the smallest kept)
+// insert (ov, col) into the list (Lv, Li) sorted by descending value code;
+// the caller has checked ov > Lv[KC-1].  Columns reach a thread in increasing
+// order, so a new entry goes after every kept entry of equal value: that is
+// the order of the keys (value, lower index first).  All comparisons are
+// against the old list, so the KC steps are independent: gt[j] = ov > Lv[j] is
+// false then true along the list, and entry j becomes entry j-1 where
+// gt[j-1], the new one where gt[j] alone, else stays.
 template <int KC>
-__device__ __forceinline__ void lm_insert(uint64_t (&L)[KC], uint64_t k) {
-  L[KC - 1] = k;
+__device__ __forceinline__ void lm_insert(uint32_t (&Lv)[KC], uint32_t (&Li)[KC], uint32_t ov,
+                                          uint32_t col) {
+  bool gt[KC];
+#pragma unroll
+  for (int j = 0; j < KC; ++j) gt[j] = ov > Lv[j];
 #pragma unroll
   for (int j = KC - 1; j > 0; --j) {
-    const uint64_t a = L[j - 1], b = L[j];
-    const bool sw = b > a;
-    L[j - 1] = sw ? b : a;
-    L[j] = sw ? a : b;
+    Lv[j] = gt[j - 1] ? Lv[j - 1] : (gt[j] ? ov : Lv[j]);
+    Li[j] = gt[j - 1] ? Li[j - 1] : (gt[j] ? col : Li[j]);
   }
+  Lv[0] = gt[0] ? ov : Lv[0];
+  Li[0] = gt[0] ? col : Li[0];
 }
+
+// One row's running state over the columns an epilogue thread folds in:
+// online base-2 (m, S, U) with S and U kept as even / odd column pairs, the
+// chosen token's logit, and the exact top-KC entries as order-preserving value
+// codes (0 = empty) with their columns.
+template <int KC>
+struct LmRow {
+  float m, xy, thr;  // thr: value of the KC-th entry kept (-inf while the list is not full)
+  float2 S2, U2;
+  bool bad, has_y;
+  uint32_t Lv[KC], Li[KC];
+
+  __device__ __forceinline__ void init() {
+    m = M2_INIT;
+    xy = NAN;
+    thr = -INFINITY;
+    S2 = make_float2(0.f, 0.f);
+    U2 = make_float2(0.f, 0.f);
+    bad = has_y = false;
+#pragma unroll
+    for (int j = 0; j < KC; ++j) Lv[j] = Li[j] = 0u;
+  }
+
+  // fold 32 consecutive logits v of columns col0 .. col0 + 31 (those >= V are
+  // outside the vocabulary); y is the row's chosen token
+  __device__ __forceinline__ void chunk(float (&v)[32], int32_t col0, int32_t V, int32_t y) {
+    const bool whole = col0 + 32 <= V;  // false only in the last vocabulary tile
+    if (!whole) {
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (col0 + j >= V) v[j] = -INFINITY;
+    }
+    float cmax = v[0];
+#pragma unroll
+    for (int j = 1; j < 32; ++j) cmax = fmaxf(cmax, v[j]);
+    if (cmax == INFINITY) bad = true;  // NaN reaches S and U and is flagged there
+    const float tm = cmax * L2E;
+    if (tm > m) {
+      const float dl = m - tm, f = ex2(dl);
+      const float2 f2 = make_float2(f, f), dl2 = make_float2(dl, dl);
+      U2 = __fmul2_rn(f2, __ffma2_rn(dl2, S2, U2));
+      S2 = __fmul2_rn(S2, f2);
+      m = tm;
+    }
+    const float2 nm = make_float2(-m, -m), l2e = make_float2(L2E, L2E);
+    const float2 lo2 = make_float2(-1e30f, -1e30f);
+#pragma unroll
+    for (int j = 0; j < 32; j += 2) {
+      float2 dd = __ffma2_rn(make_float2(v[j], v[j + 1]), l2e, nm);
+      if (!whole) dd = make_float2(fmaxf(dd.x, lo2.x), fmaxf(dd.y, lo2.y));  // -inf -> 0 weight
+      const float2 e = make_float2(ex2(dd.x), ex2(dd.y));
+      S2 = __fadd2_rn(S2, e);
+      U2 = __ffma2_rn(e, dd, U2);
+    }
+    // chosen token: one chunk of the whole sweep holds it
+    const uint32_t yo = (uint32_t)(y - col0);
+    if (yo < 32u && (int32_t)yo + col0 < V) {
+      xy = lm_pick(v, yo);
+      has_y = true;
+    }
+    // top-KC: only chunks whose maximum reaches the list's threshold
+    if (cmax >= thr) {
+      uint32_t mask = 0u;
+#pragma unroll
+      for (int j = 0; j < 32; ++j) mask |= (v[j] >= thr ? 1u : 0u) << j;
+      if (!whole) {  // columns < V only (0 <= V - col0 < 32 here, or none)
+        const int32_t nv = V - col0;
+        mask &= nv > 0 ? (1u << nv) - 1u : 0u;
+      }
+      while (mask) {
+        const uint32_t j = (uint32_t)__ffs(mask) - 1u;
+        mask &= mask - 1u;
+        const uint32_t ov = ord(lm_pick(v, j));
+        if (ov > Lv[KC - 1]) {
+          lm_insert<KC>(Lv, Li, ov, (uint32_t)col0 + j);
+          if (Lv[KC - 1] != 0u) thr = unord(Lv[KC - 1]);
+        }
+      }
+    }
+  }
+
+  __device__ __forceinline__ void store(LmPart* p) const {
+    p->m = m;
+    p->S = S2.x + S2.y;
+    p->U = U2.x + U2.y;
+    p->xy = xy;
+    p->bad = bad ? 1u : 0u;
+    p->has_y = has_y ? 1u : 0u;
+#pragma unroll
+    for (int j = 0; j < 32; ++j)  // the keys of make_key
+      p->top[j] = (j < KC && Lv[j] != 0u)
+                      ? ((uint64_t)Lv[j] << 32) | (uint64_t)(0xffffffffu - Li[j])
+                      : 0ull;
+  }
+};
 
 template <int KC>
 __global__ void __launch_bounds__(LM_NT, 1)
@@ -259,90 +352,98 @@ __global__ void __launch_bounds__(LM_NT, 1)
                                            ~(uintptr_t)1023);
   uint64_t* full = reinterpret_cast<uint64_t*>(sm + LM_STAGES * LM_STAGE_BYTES);
   uint64_t* empty = full + LM_STAGES;
-  uint64_t* tfull = empty + LM_STAGES;   // both accumulators hold a finished tile
-  uint64_t* tempty = tfull + 1;          // the epilogue has read them
-  uint64_t* mdone = tempty + 1;          // the MMA issuer's own completion
+  uint64_t* tfull = empty + LM_STAGES;   // [2] accumulator b holds a finished tile
+  uint64_t* tempty = tfull + 2;          // [2] (rank 0) both epilogues have read accumulator b
+  uint64_t* mdone = tempty + 2;          // (rank 0) the MMA issuer's own completion
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mdone + 1);
   volatile uint32_t* abort_ = tmem_slot + 1;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  // grid x = vocabulary split (fastest), y = 256-row tile: a wave of CTAs covers a
-  // few row tiles across all splits, so the H tiles it re-reads and the W tiles
-  // it streams together fit in L2
-  const int split = blockIdx.x, mt = blockIdx.y;
-  const int t0 = split * a.tiles_per_split, t1 = t0 + a.tiles_per_split;
-  // cluster position (cluster dims cs x cm): pm along the rows (CTAs with the
-  // same ps share W slices, cm of them), ps along the splits (CTAs with the same
-  // pm share H slices, cs of them); rank = ps + pm cs
-  const int ps = a.cs > 1 ? (int)lm_cluster_id(0) : 0;
-  const int pm = a.cm > 1 ? (int)lm_cluster_id(1) : 0;
-  uint16_t mask_h = 0, mask_w = 0;  // CTAs receiving my H slice / my W slice
-  for (int s2 = 0; s2 < a.cs; ++s2) mask_h |= (uint16_t)(1u << (s2 + pm * a.cs));
-  for (int m2 = 0; m2 < a.cm; ++m2) mask_w |= (uint16_t)(1u << (ps + m2 * a.cs));
-  const uint16_t mask_rel = mask_h | mask_w;  // writers into my stages = readers of mine
-  const bool clustered = a.cm * a.cs > 1;
+  const uint32_t rank = lm_cluster_x();
+  const bool lead = rank == 0u;
+  // launch order: bands of `band` row pairs; within a band all its pairs of
+  // one split, then the next split; the last band may be shorter
+  int split, pr;
+  {
+    const int u = (int)(blockIdx.x >> 1), G = a.band, per_band = G * a.nsplit;
+    const int full_bands = a.npairs / G, b = u / per_band;
+    if (b < full_bands) {
+      const int r = u - b * per_band;
+      split = r / G;
+      pr = b * G + (r - split * G);
+    } else {
+      const int rem = a.npairs - full_bands * G, r = u - full_bands * per_band;
+      split = r / rem;
+      pr = full_bands * G + (r - split * rem);
+    }
+  }
+  const int mt = 2 * pr + (int)rank;
+  const int t0 = split * a.tiles_per_split;
+  const int t1 = min(t0 + a.tiles_per_split, a.ntiles);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < LM_STAGES; ++s) {
       lm_mbar_init(full + s, 1);
-      lm_mbar_init(empty + s, (uint32_t)(a.cm + a.cs - 1));  // one release per writer's reader
+      lm_mbar_init(empty + s, 1);
     }
-    lm_mbar_init(tfull, 1);
-    lm_mbar_init(tempty, LM_EPI_WARPS);  // one arrival per epilogue warp
+    for (int b = 0; b < 2; ++b) {
+      lm_mbar_init(tfull + b, 1);
+      lm_mbar_init(tempty + b, 2 * LM_EPI_WARPS);  // every epilogue warp of both CTAs
+    }
     lm_mbar_init(mdone, 1);
     *abort_ = 0u;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
   if (warp == 1) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                      lm_smem(tmem_slot)),
                  "r"(LM_TMEM_COLS)
                  : "memory");
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
   }
   __syncthreads();
-  if (clustered) lm_cluster_sync();  // every CTA's barriers exist before any remote use
+  lm_cluster_sync();  // both CTAs' barriers and TMEM exist before any remote use
   lm_fence_after();
   const uint32_t tmem = *tmem_slot;
+  const uint32_t full0 = lm_mapa(full, 0u), tempty0 = lm_mapa(tempty, 0u);
 
   if (warp == 0) {
-    if (lane == 0) {  // ---- TMA producer
+    if (lane == 0) {  // ---- TMA producer (both CTAs)
       int it = 0;
       for (int t = t0; t < t1 && !*abort_; ++t)
         for (int kb = 0; kb < a.kblocks; ++kb, ++it) {
           const int s = it % LM_STAGES;
           const uint32_t ph = (uint32_t)(it / LM_STAGES) & 1u;
           if (!lm_wait(empty + s, ph ^ 1u, abort_, a.err)) {
-            t = t1;  // leave both loops
+            t = t1;
             break;
           }
           uint8_t* st = sm + s * LM_STAGE_BYTES;
-          lm_mbar_expect(full + s, LM_STAGE_BYTES);  // all slices, from every writer
-          if (!clustered) {
-            lm_tma_load(&tmA, st, full + s, kb * LM_BK, mt * LM_BM);
-            lm_tma_load(&tmB, st + LM_A_BYTES, full + s, kb * LM_BK, t * LM_BN);
-          } else {
-            const int ha = LM_BM / a.cs, wb = LM_BN / a.cm;  // slice rows
-            lm_tma_load_mc(&tmA, st + ps * ha * 128, full + s, kb * LM_BK, mt * LM_BM + ps * ha,
-                           mask_h);
-            lm_tma_load_mc(&tmB, st + LM_A_BYTES + pm * wb * 128, full + s, kb * LM_BK,
-                           t * LM_BN + pm * wb, mask_w);
+          if (lead) lm_mbar_expect(full + s, 2 * LM_STAGE_BYTES);  // both CTAs' bytes
+          for (int hk = 0; hk < LM_BK / LM_BOX_K; ++hk) {  // boxes, 16 KB apart
+            const int x = kb * LM_BK + LM_BOX_K * hk;
+            lm_tma_load_pair(&tmA, st + hk * LM_BOX_BYTES, full0 + 8u * (uint32_t)s, x,
+                             mt * LM_BM);
+            lm_tma_load_pair(&tmB, st + LM_A_BYTES + hk * LM_BOX_BYTES, full0 + 8u * (uint32_t)s,
+                             x, t * LM_BN + (int)rank * (LM_BN / 2));
           }
         }
-      // the copies still in flight land before the CTA exits (already true
-      // unless a wait gave up): wait, bounded, for the last stages' loads
-      for (int j = it - 1; j >= 0 && j >= it - LM_STAGES; --j) {
-        volatile uint32_t no_abort = 0u;
-        lm_wait(full + j % LM_STAGES, (uint32_t)(j / LM_STAGES) & 1u, &no_abort, a.err);
-      }
+      // rank 0's stage barriers count both CTAs' copies: it waits, bounded,
+      // for the last stages, so no copy is in flight when the pair exits
+      if (lead)
+        for (int j = it - 1; j >= 0 && j >= it - LM_STAGES; --j) {
+          volatile uint32_t no_abort = 0u;
+          lm_wait(full + j % LM_STAGES, (uint32_t)(j / LM_STAGES) & 1u, &no_abort, a.err);
+        }
     }
   } else if (warp == 1) {
-    if (lane == 0) {  // ---- MMA issuer
+    if (lane == 0 && lead) {  // ---- MMA issuer (rank 0)
       int it = 0;
       for (int i = 0, t = t0; t < t1 && !*abort_; ++t, ++i) {
-        // the epilogue has read the previous tile out of both accumulators
-        if (!lm_wait(tempty, ((uint32_t)i & 1u) ^ 1u, abort_, a.err)) break;
+        const int b = i & 1;
+        if (!lm_wait(tempty + b, (((uint32_t)i >> 1) & 1u) ^ 1u, abort_, a.err)) break;
         lm_fence_after();
+        const uint32_t dt = tmem + (uint32_t)(b * LM_BN);
         bool ok = true;
         for (int kb = 0; kb < a.kblocks; ++kb, ++it) {
           const int s = it % LM_STAGES;
@@ -354,139 +455,89 @@ __global__ void __launch_bounds__(LM_NT, 1)
           lm_fence_after();
           const uint32_t sa = lm_smem(sm + s * LM_STAGE_BYTES), sb = sa + LM_A_BYTES;
 #pragma unroll
-          for (int k = 0; k < LM_BK / 16; ++k) {  // K = 16 per MMA: 32 bytes along the row
-            const uint64_t bd = lm_sdesc(sb + 32 * k);
-            const uint32_t acc = (kb | k) != 0 ? 1u : 0u;
-            lm_mma(tmem, lm_sdesc(sa + 32 * k), bd, acc);                       // rows 0-127
-            lm_mma(tmem + LM_BN, lm_sdesc(sa + LM_MH * 128 + 32 * k), bd, acc);  // rows 128-255
+          for (int k = 0; k < LM_BK / 16; ++k) {  // K = 16: 32 bytes along a box row
+            const uint32_t ko = (uint32_t)((k / (LM_BOX_K / 16)) * LM_BOX_BYTES +
+                                           32 * (k % (LM_BOX_K / 16)));
+            asm volatile(
+                "{\n\t.reg .pred p;\n\t"
+                "setp.ne.b32 p, %4, 0;\n\t"
+                "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(dt),
+                "l"(lm_sdesc(sa + ko)), "l"(lm_sdesc(sb + ko)), "r"(LM_IDESC),
+                "r"((kb | k) != 0 ? 1u : 0u)
+                : "memory");
           }
-          // the stage is free, in every CTA that writes into it, once these MMAs
-          // have read it
-          if (clustered)
-            lm_commit_mc(empty + s, mask_rel);
-          else
-            lm_commit(empty + s);
+          // stage s is free in both CTAs once these MMAs have read it
+          asm volatile(
+              "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::"
+              "cluster.b64 [%0], %1;" ::"r"(lm_smem(empty + s)),
+              "h"((uint16_t)3)
+              : "memory");
         }
         if (!ok) break;
-        lm_commit(tfull);
+        asm volatile(
+            "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::"
+            "cluster.b64 [%0], %1;" ::"r"(lm_smem(tfull + b)),
+            "h"((uint16_t)3)
+            : "memory");
       }
-      // every MMA this thread issued has completed before TMEM is freed
-      lm_commit(mdone);
+      asm volatile(
+          "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::"
+          "cluster.b64 [%0], %1;" ::"r"(lm_smem(mdone)),
+          "h"((uint16_t)1)
+          : "memory");
       volatile uint32_t no_abort = 0u;
       lm_wait(mdone, 0u, &no_abort, a.err);
     }
-  } else {  // ---- epilogue: warps 2..9, TMEM lanes 32 (warp % 4) .., accumulator h
-    const int q = warp & 3, h = (warp - 2) >> 2;
-    const int64_t row = (int64_t)mt * LM_BM + LM_MH * h + 32 * q + lane;
+  } else {  // ---- epilogue (both CTAs): TMEM lanes 32 (warp % 4) .., column half hc
+    const int q = warp & 3, hc = (warp - 2) >> 2;
+    const int64_t row = (int64_t)mt * LM_BM + 32 * q + lane;
     const bool live = row < a.n_rows;
     const int32_t y = live ? a.chosen[row] : -1;
     const int32_t V = (int32_t)a.vocab;
-    float m = M2_INIT, xy = NAN;
-    float2 S2 = make_float2(0.f, 0.f), U2 = make_float2(0.f, 0.f);  // even / odd columns
-    bool bad = false, has_y = false;
-    uint64_t L[KC];
-#pragma unroll
-    for (int j = 0; j < KC; ++j) L[j] = 0ull;
-    float thr = -INFINITY;  // value of the KC-th key kept (-inf while the list is not full)
+    LmRow<KC> st;
+    st.init();
     for (int i = 0, t = t0; t < t1; ++t, ++i) {
+      const int b = i & 1;
       int ok = 1;
-      if (lane == 0) ok = lm_wait(tfull, (uint32_t)i & 1u, abort_, a.err) ? 1 : 0;
-      ok = __shfl_sync(FULL, ok, 0);  // the warp stays converged for tcgen05.ld
+      if (lane == 0) ok = lm_wait(tfull + b, ((uint32_t)i >> 1) & 1u, abort_, a.err) ? 1 : 0;
+      ok = __shfl_sync(FULL, ok, 0);
       if (!ok) break;
       lm_fence_after();
-      const uint32_t tbase = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(h * LM_BN);
-      for (int c = 0; c < LM_BN / 32; ++c) {
+      const int hw = LM_BN / LM_HALVES;
+      const uint32_t tbase =
+          tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(b * LM_BN + hc * hw);
+      for (int c = 0; c < hw / 32; ++c) {
         float v[32];
         lm_tmem_ld32(tbase + 32 * c, v);
-        const int32_t col0 = t * LM_BN + 32 * c;
-        const bool whole = col0 + 32 <= V;  // false only in the last vocabulary tile
-        if (!whole) {
-#pragma unroll
-          for (int j = 0; j < 32; ++j)
-            if (col0 + j >= V) v[j] = -INFINITY;
-        }
-        float cmax = v[0];
-#pragma unroll
-        for (int j = 1; j < 32; ++j) cmax = fmaxf(cmax, v[j]);
-        if (cmax == INFINITY) bad = true;  // NaN reaches S and U and is flagged there
-        const float tm = cmax * L2E;
-        if (tm > m) {
-          const float dl = m - tm, f = ex2(dl);
-          const float2 f2 = make_float2(f, f), dl2 = make_float2(dl, dl);
-          U2 = __fmul2_rn(f2, __ffma2_rn(dl2, S2, U2));
-          S2 = __fmul2_rn(S2, f2);
-          m = tm;
-        }
-        const float2 nm = make_float2(-m, -m), l2e = make_float2(L2E, L2E);
-        const float2 lo2 = make_float2(-1e30f, -1e30f);
-#pragma unroll
-        for (int j = 0; j < 32; j += 2) {
-          float2 dd = __ffma2_rn(make_float2(v[j], v[j + 1]), l2e, nm);
-          if (!whole) dd = make_float2(fmaxf(dd.x, lo2.x), fmaxf(dd.y, lo2.y));  // -inf -> 0 weight
-          const float2 e = make_float2(ex2(dd.x), ex2(dd.y));
-          S2 = __fadd2_rn(S2, e);
-          U2 = __ffma2_rn(e, dd, U2);
-        }
-        // chosen token: one chunk of the whole sweep holds it
-        const uint32_t yo = (uint32_t)(y - col0);
-        if (yo < 32u && (int32_t)yo + col0 < V) {
-          xy = lm_pick(v, yo);
-          has_y = true;
-        }
-        // top-KC: only chunks whose maximum reaches the list's threshold
-        if (cmax >= thr) {
-          uint32_t mask = 0u;
-#pragma unroll
-          for (int j = 0; j < 32; ++j) mask |= (v[j] >= thr && col0 + j < V ? 1u : 0u) << j;
-          while (mask) {
-            const uint32_t j = (uint32_t)__ffs(mask) - 1u;
-            mask &= mask - 1u;
-            const uint64_t k = make_key(lm_pick(v, j), (uint32_t)(col0 + (int32_t)j));
-            if (k > L[KC - 1]) {
-              lm_insert<KC>(L, k);
-              if (L[KC - 1] != 0ull) thr = key_val(L[KC - 1]);
-            }
-          }
-        }
+        st.chunk(v, t * LM_BN + hc * hw + 32 * c, V, y);
       }
       lm_fence_before();
       __syncwarp();
-      if (lane == 0) lm_mbar_arrive(tempty);
+      if (lane == 0) lm_arrive_remote(tempty0 + 8u * (uint32_t)b);
     }
-    const float S = S2.x + S2.y, U = U2.x + U2.y;
-    if (live) {
-      LmPart* p = a.parts + (int64_t)split * a.n_rows + row;
-      p->m = m;
-      p->S = S;
-      p->U = U;
-      p->xy = xy;
-      p->bad = bad ? 1u : 0u;
-      p->has_y = has_y ? 1u : 0u;
-#pragma unroll
-      for (int j = 0; j < 32; ++j) p->top[j] = j < KC ? L[j] : 0ull;
-    }
+    if (live) st.store(a.parts + ((int64_t)split * LM_HALVES + hc) * a.n_rows + row);
   }
   __syncthreads();
-  if (clustered) lm_cluster_sync();  // no CTA leaves while others may still write into it
+  lm_cluster_sync();  // the MMAs into both TMEMs are complete; no remote arrival is pending
   if (warp == 1) {
     lm_fence_after();
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem),
                  "r"(LM_TMEM_COLS)
                  : "memory");
   }
 }
 
-// one warp per row: merge the splits in order, then the verifier's row
-// finalisation (features, top-2 indices, flags)
+// one warp per row: merge the parts (splits x column halves) in order, then
+// the verifier's row finalisation (features, top-2 indices, flags)
 __global__ void __launch_bounds__(256) lm_merge(const Args a, const LmPart* __restrict__ parts,
-                                                int nsplit) {
+                                                int nparts) {
   const int lane = threadIdx.x & 31;
   const int64_t row = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
   if (row >= a.n_rows) return;
   float m = M2_INIT, S = 0.f, U = 0.f, xy = NAN;
   bool bad = false;
   uint64_t E = 0ull;
-  for (int s = 0; s < nsplit; ++s) {
+  for (int s = 0; s < nparts; ++s) {
     const LmPart& p = parts[(int64_t)s * a.n_rows + row];
     lse_merge(m, S, U, p.m, p.S, p.U);
     bad |= p.bad != 0u;

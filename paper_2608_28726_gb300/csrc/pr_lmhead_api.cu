@@ -36,14 +36,14 @@ EncodeTiled encoder() {
   return fn;
 }
 
-// row-major bf16 matrix [rows][d] read in boxes of 64 columns x box_rows rows,
-// 128-byte swizzle, zero fill outside the matrix
+// row-major bf16 matrix [rows][d] read in boxes of LM_BOX_K = 64 columns x
+// box_rows rows, 128-byte swizzle, zero fill outside the matrix
 bool make_map(CUtensorMap* map, const void* base, int64_t rows, int64_t d, uint32_t box_rows) {
   EncodeTiled enc = encoder();
   if (!enc) return false;
   const cuuint64_t dims[2] = {(cuuint64_t)d, (cuuint64_t)rows};
   const cuuint64_t strides[1] = {(cuuint64_t)d * 2};
-  const cuuint32_t box[2] = {(cuuint32_t)prk::LM_BK, box_rows};
+  const cuuint32_t box[2] = {(cuuint32_t)prk::LM_BOX_K, box_rows};
   const cuuint32_t estr[2] = {1, 1};
   return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
              box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -82,24 +82,16 @@ pr_status pr_lmhead_features(pr_ctx* c, const void* hidden, const void* weight, 
   const int kc = topk > 2 ? topk : 2;
   const void* kern = kc <= 20 ? reinterpret_cast<const void*>(&prk::lm_fused<20>)
                               : reinterpret_cast<const void*>(&prk::lm_fused<32>);
-  // Launch shape.  Splits of the vocabulary run along grid x (fastest), 256-row
-  // tiles along y, so a wave of one CTA per SM covers num_sms / nsplit row
-  // tiles across all splits; nsplit near sqrt(num_sms) keeps a wave's H tiles
-  // plus its in-flight W tiles small (~25 tiles of 1.8 MB), and among those the
-  // count with the least idle tail in the last wave is taken.  Thread-block
-  // clusters (cm x cs CTAs sharing W / H slices through TMA multicast) only when
-  // forced: measured slower, since every stage then waits for its slowest reader.
-  int cm = 1, cs = 1;
-  if (c->lm_force) {
-    cm = c->lm_force / 10;
-    cs = c->lm_force % 10;
-  }
-  const int64_t mt_pad = (mtiles + cm - 1) / cm * cm;
+  // Launch shape: nsplit vocabulary splits (around 12; among those the count
+  // with the least idle tail in the last wave of one CTA per SM), CTA pairs of
+  // 256 rows ordered in bands of `band` row pairs, whose H rows (256 d bf16
+  // each) fill about a quarter of L2: a wave then holds one band's H plus the
+  // W tiles of a few splits, each read from DRAM about once per wave.
+  const int64_t mt_pad = (mtiles + 1) / 2 * 2;
   int64_t nsplit = 1;
   {
     double best = 1e30;
-    for (int64_t ns = std::max<int64_t>(cs, 8); ns <= 24; ns += cs) {
-      if (ns > (ntiles + cs - 1) / cs * cs) break;
+    for (int64_t ns = 8; ns <= 24 && ns <= ntiles; ++ns) {
       const int64_t ctas = mt_pad * ns;
       const int64_t waves = (ctas + c->num_sms - 1) / c->num_sms;
       const double waste = (double)(waves * c->num_sms - ctas) / (double)(waves * c->num_sms);
@@ -109,15 +101,15 @@ pr_status pr_lmhead_features(pr_ctx* c, const void* hidden, const void* weight, 
         nsplit = ns;
       }
     }
-    if (best == 1e30) nsplit = std::max<int64_t>(cs, std::min<int64_t>(ntiles, c->num_sms / mt_pad) / cs * cs);
-    if (nsplit < 1) nsplit = cs;
+    if (best == 1e30) nsplit = std::max<int64_t>(1, std::min<int64_t>(ntiles, c->num_sms / mt_pad));
   }
   const int64_t per_split = (ntiles + nsplit - 1) / nsplit;
-  CUtensorMap ma, mb;
-  if (!make_map(&ma, hidden, n_rows, d, (uint32_t)(prk::LM_BM / cs)) ||
-      !make_map(&mb, weight, vocab, d, (uint32_t)(prk::LM_BN / cm)))
+  CUtensorMap ma, mb;  // boxes of 128 rows x 64 columns: a CTA's H rows, half a W tile
+  if (!make_map(&ma, hidden, n_rows, d, (uint32_t)prk::LM_BM) ||
+      !make_map(&mb, weight, vocab, d, (uint32_t)(prk::LM_BN / 2)))
     return PR_ERR_UNSUPPORTED;
-  const size_t part_bytes = (size_t)nsplit * (size_t)n_rows * sizeof(prk::LmPart);
+  const int64_t nparts = nsplit * prk::LM_HALVES;
+  const size_t part_bytes = (size_t)nparts * (size_t)n_rows * sizeof(prk::LmPart);
   if (part_bytes > c->lm_parts_bytes) {
     PR_CUDA(cudaDeviceSynchronize());  // the old buffer may still be in use
     cudaFree(c->lm_parts);
@@ -140,27 +132,31 @@ pr_status pr_lmhead_features(pr_ctx* c, const void* hidden, const void* weight, 
   la.kblocks = (int32_t)((d + prk::LM_BK - 1) / prk::LM_BK);
   la.ntiles = (int32_t)ntiles;
   la.tiles_per_split = (int32_t)per_split;
-  la.cm = cm;
-  la.cs = cs;
+  la.nsplit = (int32_t)nsplit;
+  la.npairs = (int32_t)(mt_pad / 2);
+  {
+    const int64_t h_pair = 256 * d * 2, budget = (int64_t)32 << 20;
+    la.band = (int32_t)std::max<int64_t>(1, std::min<int64_t>(la.npairs, budget / h_pair));
+  }
   la.chosen = chosen;
   la.parts = static_cast<prk::LmPart*>(c->lm_parts);
   la.err = c->flags;
   cudaLaunchConfig_t cfg;
   memset(&cfg, 0, sizeof cfg);
-  cfg.gridDim = dim3((unsigned)nsplit, (unsigned)mt_pad);
+  if (mt_pad * nsplit > 0x7fffffffLL) return PR_ERR_INVALID_ARG;
+  cfg.gridDim = dim3((unsigned)(mt_pad * nsplit));
   cfg.blockDim = dim3(prk::LM_NT);
   cfg.dynamicSmemBytes = prk::LM_SMEM;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = (unsigned)cs;
-  attr[0].val.clusterDim.y = (unsigned)cm;
+  attr[0].id = cudaLaunchAttributeClusterDimension;  // a CTA pair lies along x
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = cm * cs > 1 ? 1 : 0;
+  cfg.numAttrs = 1;
   void* kargs[] = {&ma, &mb, &la};
   PR_CUDA(cudaLaunchKernelExC(&cfg, kern, kargs));
-  c->lm_cluster = cm * 10 + cs;
   if ((st = timing_mark(c, s)) != PR_OK) return st;
   prk::Args a;
   memset(&a, 0, sizeof a);
@@ -176,7 +172,7 @@ pr_status pr_lmhead_features(pr_ctx* c, const void* hidden, const void* weight, 
   a.top2 = top2;
   a.row_flags = row_flags;
   a.ctx_flags = c->flags;
-  prk::lm_merge<<<(unsigned)((n_rows + 7) / 8), 256, 0, s>>>(a, la.parts, (int)nsplit);
+  prk::lm_merge<<<(unsigned)((n_rows + 7) / 8), 256, 0, s>>>(a, la.parts, (int)nparts);
   PR_CUDA(cudaGetLastError());
   g_launches.fetch_add(2, std::memory_order_relaxed);
   return timing_mark(c, s);

@@ -80,7 +80,8 @@ def test_lmhead_one_tile(B, ctx):
 @pytest.mark.parametrize("n,d,V", [(1, 64, 256), (130, 128, 1000), (257, 192, 4097),
                                    (300, 520, 2304)])
 def test_lmhead_ragged_shapes(B, ctx, n, d, V):
-    # row tiles of 128, vocabulary tiles of 256 and K blocks of 64 with ragged tails
+    # row tiles of 128 (CTA pairs of 256; n = 300 leaves one CTA without rows), vocabulary
+    # tiles of 256 and K blocks of 128 (two boxes of 64) with ragged tails
     check(B, ctx, n, d, V, seed=n + d + V)
 
 
@@ -98,17 +99,6 @@ def test_lmhead_flags_and_rho(B, ctx):
     assert np.isnan(fg[3, 0]) and np.isnan(fg[7, 0])
 
 
-@pytest.mark.parametrize("shape", [11, 21, 12, 22])
-def test_lmhead_cluster_shapes(B, ctx, shape):
-    """Every cluster shape (cm CTAs sharing weight slices x cs sharing hidden
-    slices through TMA multicast) gives the same records."""
-    B.pr_ctx_set_option(ctx, B.PR_OPT_LMHEAD_CLUSTER, shape)
-    try:
-        check(B, ctx, 600, 320, 7000, seed=40 + shape)
-    finally:
-        B.pr_ctx_set_option(ctx, B.PR_OPT_LMHEAD_CLUSTER, 0)
-
-
 def test_lmhead_large_vocab_and_hidden(B, ctx):
     """d = 3,584 (the small model's hidden size) and V = 151,936 on a few rows."""
     check(B, ctx, 8, 3584, 151936, seed=7)
@@ -121,3 +111,28 @@ def test_lmhead_is_deterministic(B, ctx):
     torch.cuda.synchronize()
     for x, y in zip(a, b):
         assert torch.equal(x.view(torch.int32), y.view(torch.int32))
+
+
+def test_lmhead_full_batch_sampled_rows(B, ctx):
+    """The benchmark's batch in its launch configuration (8,847 rows x d =
+    3,584 x V = 151,936: 13 vocabulary splits, row pairs in bands of 18):
+    rows at tile, pair and band boundaries and the last rows against the
+    oracle, computed row by row."""
+    from paper_2608_28726_gb300 import workloads as W
+    n, d, V = 8847, 3584, 151936
+    h, w, chosen = W.lmhead_inputs(n, d, V, device="cpu")
+    feat, top2, rf = B.pr_lmhead_features(ctx, h.cuda(), w.cuda(), chosen.cuda(), 20)
+    torch.cuda.synchronize()
+    assert B.pr_ctx_flags(ctx) & B.PR_FLAG_TIMEOUT == 0
+    rows = np.array([0, 1, 127, 128, 255, 256, 4607, 4608, 8703, 8704, 8845, 8846])
+    o = lmhead.features(bits(h[rows]), bits(w), chosen.numpy()[rows], K=20)
+    assert_close(feat.cpu().numpy()[rows], o["feat"], "features", rtol=TOL, atol=TOL)
+    assert np.array_equal(rf.cpu().numpy()[rows].view(np.uint32), o["row_flags"])
+    x = o["logits"]
+    srt = -np.sort(-x, axis=1)
+    tg = top2.cpu().numpy()[rows]
+    for i in range(len(rows)):
+        if srt[i, 0] - srt[i, 1] > 1e-3 and srt[i, 1] - srt[i, 2] > 1e-3:
+            assert list(tg[i]) == list(o["idx"][i]), rows[i]
+        else:
+            assert x[i, tg[i, 0]] >= srt[i, 0] - 1e-3
