@@ -416,14 +416,23 @@ def run_other_workload(args):
                 torch.empty(S, dtype=torch.int32, device=dev))
         state = {"t": 0}
 
+        def decode_call(t, st):
+            B.pr_decode_step(ctx, x_all[t * S:(t + 1) * S], slot, ch_all[t * S:(t + 1) * S], eos[t],
+                             w, tr.b, tr.tau, *outs, stream=st)
+
         def step():
             t = state["t"]
             if t == T:
                 B.pr_ctx_reset(ctx, stream=stream)
                 t = 0
-            B.pr_decode_step(ctx, x_all[t * S:(t + 1) * S], slot, ch_all[t * S:(t + 1) * S], eos[t],
-                             w, tr.b, tr.tau, *outs, stream=stream)
+            decode_call(t, stream)
             state["t"] = t + 1
+
+        def graph_body(st):  # a context reset and the whole trace
+            B.pr_ctx_reset(ctx, stream=st)
+            for t in range(T):
+                decode_call(t, st)
+            return T
 
         rows_per_step = S
         bytes_per_step = S * (wl.vocab * 2 + 4 + 1 + 4) + S * 4
@@ -450,14 +459,22 @@ def run_other_workload(args):
         chunk = wl.chunk_rows or wl.n_rows
         state = {"c": 0}
 
-        def step():
-            c = state["c"] % copies
-            state["c"] += 1
+        def route_call(c, st):
             for lo in range(0, wl.n_rows, chunk):
                 hi = min(wl.n_rows, lo + chunk)
                 B.pr_route(ctx, xs[c][lo:hi], chs[c][lo:hi], off, w, wl.b, wl.tau, row_base=lo,
                            score=outs[0], ship=outs[1], req_flags=outs[2], agg=None,
-                           stream=stream, want_agg=False)
+                           stream=st, want_agg=False)
+
+        def step():
+            c = state["c"] % copies
+            state["c"] += 1
+            route_call(c, stream)
+
+        def graph_body(st):  # one step on each rotated copy
+            for c in range(copies):
+                route_call(c, st)
+            return copies
 
         rows_per_step = wl.n_rows
         bytes_per_step = algorithmic_bytes(wl)
@@ -489,6 +506,34 @@ def run_other_workload(args):
 
     isolated_ms, _ = timed(0)
     ms, launches = timed(1)
+    stream_ms = ms
+    graph_info = None
+    if name in ("tiny", "decode"):
+        # launch-bound loops: the steps captured in one CUDA graph (tiny: one
+        # step per rotated copy; decode: a reset and the whole trace), replayed
+        gr = torch.cuda.CUDAGraph()
+        n0 = B.launch_count()
+        with torch.cuda.graph(gr, capture_error_mode="thread_local"):
+            per = graph_body(torch.cuda.current_stream(dev))
+        nodes = B.launch_count() - n0
+        gst = torch.cuda.current_stream(dev)
+        for _ in range(2):
+            gr.replay()
+        torch.cuda.synchronize(dev)
+        reps = max(3, -(-1000 // per))
+        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        barrier(world)
+        torch.cuda.synchronize(dev)
+        ev0.record(gst)
+        for _ in range(reps):
+            gr.replay()
+        ev1.record(gst)
+        torch.cuda.synchronize(dev)
+        barrier(world)
+        ms = reduce_max(ev0.elapsed_time(ev1), world, dev) / (reps * per)
+        launches = nodes * reps
+        K = reps * per
+        graph_info = {"steps_per_graph": per, "replays": reps, "kernels_per_graph": nodes}
     B.pr_ctx_set_option(ctx, B.PR_OPT_OVERLAP, 0)
     peaks_file = os.path.join(ROOT, "MEASURED_PEAKS.json")
     peak = float(json.load(open(peaks_file))["hbm_gbs"]) if os.path.exists(peaks_file) else 6800.0
@@ -499,12 +544,17 @@ def run_other_workload(args):
             "value": rows_per_step * world / (ms / 1e3), "unit": UNIT, "n_gpus": world, "steps": K,
             "warmup": max(3, args.warmup), "ms_per_step": ms, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": dtype, "data": "synthetic",
-            "config": {"workload": desc, "rows_per_step_per_gpu": rows_per_step},
+            "config": {"workload": desc, "rows_per_step_per_gpu": rows_per_step,
+                       "timing": ("CUDA graph replays (%d steps per graph, %d replays)" %
+                                  (graph_info["steps_per_graph"], graph_info["replays"])
+                                  if graph_info else "stream of back-to-back calls")},
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak, "traffic": None,
                          "algorithmic_bytes_per_step": bytes_per_step,
+                         "stream_ms_per_step": stream_ms,
                          "isolated_ms_per_step": isolated_ms,
                          "isolated_frac": bytes_per_step / (isolated_ms / 1e3) / 1e9 / peak},
+            "graph": graph_info,
             "gpu_launches": launches}))
     B.pr_ctx_destroy(ctx)
     return 0
