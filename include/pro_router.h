@@ -336,6 +336,16 @@ pr_status pr_lmhead_features(pr_ctx* ctx, const void* hidden, const void* weight
                              const int64_t* offsets, int32_t n_req, float* feat, int32_t* top2,
                              uint32_t* row_flags, void* stream);
 
+/*
+ * Failure-detection self-test: runs the bounded device-side wait that
+ * pr_lmhead_features' kernels use on an mbarrier that nothing completes, with
+ * a limit of `limit_ns` nanoseconds (0 .. 2e9) instead of 2 s.  *completed (host)
+ * receives 0 when the wait ran out, and the run-out raises PR_FLAG_TIMEOUT in
+ * the context flag word, exactly as a stalled pr_lmhead_features would; the
+ * context stays usable.  One launch on the default stream, synchronous.
+ */
+pr_status pr_selftest_wait(pr_ctx* ctx, int64_t limit_ns, int32_t* completed);
+
 /* ---- quantile-summary + MLP aggregator ------------------------------------------------ */
 
 #define PR_QMLP_SUMMARY 28   /* summary length: 4 features x 7 quantile levels */

@@ -32,6 +32,7 @@ EXPORTS = (
     "pr_state_export", "pr_state_import", "pr_status_string", "pr_last_cuda_error",
     "pr_launch_count", "pr_route_noalloc", "pr_head_param_count", "pr_head_score",
     "pr_ctx_kernel_times", "pr_selective_metrics", "pr_quantile_score", "pr_lmhead_features",
+    "pr_selftest_wait",
 )
 
 if not os.path.exists(LIB):
@@ -59,6 +60,7 @@ _SIGS = {
                          _P, _P, _P],
     "pr_ctx_kernel_times": [_P, _P, _I32, ctypes.POINTER(_I32)],
     "pr_lmhead_features": [_P, _P, _P, _I64, _I64, _I64, _P, _I32, _P, _I32, _P, _P, _P, _P],
+    "pr_selftest_wait": [_P, _I64, ctypes.POINTER(_I32)],
     "pr_quantile_score": [_P, _P, _P, _I64, _P, _I32, _P, _F32, _P, _P, _P, _P, _P],
     "pr_selective_metrics": [_P, _P, _P, _I64, ctypes.c_double, _P, _P],
     "pr_head_score": [_P, _P, _P, _I64, _P, _I32, _P, _I32, _F32, _P, _P, _P, _P],
@@ -352,3 +354,10 @@ def pr_lmhead_features(ctx, hidden, weight, chosen, topk: int = 20, offsets=None
                                    _ptr(row_flags), _stream(stream)), "pr_lmhead_features")
     return feat, top2, row_flags
 
+
+def pr_selftest_wait(ctx, limit_ns: int) -> bool:
+    """The library's bounded device wait on an mbarrier nothing completes;
+    returns whether it completed (False: it ran out and raised PR_FLAG_TIMEOUT)."""
+    done = _I32(-1)
+    _check(_lib.pr_selftest_wait(ctx, int(limit_ns), ctypes.byref(done)), "pr_selftest_wait")
+    return done.value == 1

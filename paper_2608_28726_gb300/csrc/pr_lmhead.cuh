@@ -124,14 +124,14 @@ __device__ __forceinline__ uint64_t lm_clock() {
   return t;
 }
 __device__ __forceinline__ bool lm_wait(uint64_t* b, uint32_t parity, volatile uint32_t* abort_,
-                                        uint32_t* err) {
+                                        uint32_t* err, uint64_t limit_ns = LM_WAIT_NS) {
   if (lm_mbar_test(b, parity)) return true;
   const uint64_t t0 = lm_clock();
   for (uint32_t i = 1;; ++i) {
     if (lm_mbar_test(b, parity)) return true;
     if ((i & 255u) == 0u) {
       if (*abort_) return false;
-      if (lm_clock() - t0 > LM_WAIT_NS) break;
+      if (lm_clock() - t0 > limit_ns) break;
     }
   }
   *abort_ = 1u;
@@ -525,6 +525,18 @@ __global__ void __launch_bounds__(LM_NT, 1)
                  "r"(LM_TMEM_COLS)
                  : "memory");
   }
+}
+
+// The bounded wait on an mbarrier that nothing completes, with the given
+// limit: *completed = 0 and PR_FLAG_TIMEOUT in *err once it runs out (one
+// thread; the failure path of lm_fused's waits, exercised without a stall).
+__global__ void lm_wait_probe(uint32_t* err, uint64_t limit_ns, int32_t* completed) {
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ uint32_t abort_flag;
+  lm_mbar_init(&bar, 1);
+  abort_flag = 0u;
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  *completed = lm_wait(&bar, 0u, &abort_flag, err, limit_ns) ? 1 : 0;
 }
 
 // one warp per row: merge the parts (splits x column halves) in order, then

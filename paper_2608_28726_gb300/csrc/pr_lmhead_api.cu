@@ -178,4 +178,19 @@ pr_status pr_lmhead_features(pr_ctx* c, const void* hidden, const void* weight, 
   return timing_mark(c, s);
 }
 
+pr_status pr_selftest_wait(pr_ctx* c, int64_t limit_ns, int32_t* completed) {
+  if (!c || !completed || limit_ns < 0 || limit_ns > 2000000000LL) return PR_ERR_INVALID_ARG;
+  pr_status st = set_device(c);
+  if (st != PR_OK) return st;
+  int32_t* d = nullptr;
+  PR_CUDA(cudaMalloc(&d, sizeof(int32_t)));
+  prk::lm_wait_probe<<<1, 1>>>(c->flags, (uint64_t)limit_ns, d);
+  cudaError_t e = cudaGetLastError();
+  if (e == cudaSuccess) e = cudaMemcpy(completed, d, sizeof(int32_t), cudaMemcpyDeviceToHost);
+  cudaFree(d);
+  if (e != cudaSuccess) return cuda_fail(e, "pr_selftest_wait");
+  g_launches.fetch_add(1, std::memory_order_relaxed);
+  return PR_OK;
+}
+
 }  // extern "C"

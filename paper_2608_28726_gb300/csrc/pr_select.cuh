@@ -126,20 +126,35 @@ __global__ void __launch_bounds__(SEL_NT) sel_hist(const uint32_t* __restrict__ 
   counts[(int64_t)threadIdx.x * ntiles + blockIdx.x] = c;
 }
 
-// CTA d: exclusive scan of counts[d][0 .. ntiles) in place; total[d] = the sum
+// CTA d: exclusive scan of counts[d][0 .. ntiles) in place; total[d] = the sum.
+// Windows of 8,192 counts are staged in shared memory with coalesced loads
+// (one padding word per 32 so that a thread's 32 consecutive counts sit in 32
+// banks); thread t scans counts [32 t, 32 t + 32) of the window, one block scan
+// gives every thread its start, and the prefixes go back with coalesced
+// stores.
+constexpr int SEL_SCAN_W = SEL_NT * 32;  // counts per window
+
 __global__ void __launch_bounds__(SEL_NT) sel_scan_digit(uint32_t* __restrict__ counts,
                                                          int64_t ntiles,
                                                          uint32_t* __restrict__ total) {
+  __shared__ uint32_t buf[SEL_SCAN_W + SEL_SCAN_W / 32];
   __shared__ uint32_t ws[SEL_NT / 32];
-  __shared__ uint32_t carry;
   uint32_t* c = counts + (int64_t)blockIdx.x * ntiles;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  if (threadIdx.x == 0) carry = 0;
-  __syncthreads();
-  for (int64_t t0 = 0; t0 < ntiles; t0 += SEL_NT) {
-    const int64_t t = t0 + threadIdx.x;
-    const uint32_t v = t < ntiles ? c[t] : 0u;
-    uint32_t x = v;  // inclusive warp scan
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  uint32_t carry = 0;
+  for (int64_t w0 = 0; w0 < ntiles; w0 += SEL_SCAN_W) {
+    const int m = ntiles - w0 < SEL_SCAN_W ? (int)(ntiles - w0) : SEL_SCAN_W;
+#pragma unroll 8
+    for (int i = 0; i < 32; ++i) {
+      const int idx = i * SEL_NT + tid;
+      buf[idx + (idx >> 5)] = idx < m ? c[w0 + idx] : 0u;
+    }
+    __syncthreads();
+    uint32_t* mine = buf + tid * 33;
+    uint32_t sum = 0;
+#pragma unroll
+    for (int j = 0; j < 32; ++j) sum += mine[j];
+    uint32_t x = sum;  // inclusive scan of the thread sums
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
       const uint32_t y = __shfl_up_sync(FULL, x, o);
@@ -147,19 +162,28 @@ __global__ void __launch_bounds__(SEL_NT) sel_scan_digit(uint32_t* __restrict__ 
     }
     if (lane == 31) ws[warp] = x;
     __syncthreads();
-    uint32_t wbase = 0, all = 0;
+    uint32_t run = carry + x - sum, all = 0;
 #pragma unroll
     for (int w = 0; w < SEL_NT / 32; ++w) {
-      if (w < warp) wbase += ws[w];
+      if (w < warp) run += ws[w];
       all += ws[w];
     }
-    const uint32_t c0 = carry;
-    if (t < ntiles) c[t] = c0 + wbase + x - v;
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+      const uint32_t v = mine[j];
+      mine[j] = run;
+      run += v;
+    }
     __syncthreads();
-    if (threadIdx.x == 0) carry = c0 + all;
-    __syncthreads();
+#pragma unroll 8
+    for (int i = 0; i < 32; ++i) {
+      const int idx = i * SEL_NT + tid;
+      if (idx < m) c[w0 + idx] = buf[idx + (idx >> 5)];
+    }
+    carry += all;
+    __syncthreads();  // buf and ws are reused by the next window
   }
-  if (threadIdx.x == 0) total[blockIdx.x] = carry;
+  if (tid == 0) total[blockIdx.x] = carry;
 }
 
 // Stable scatter of one tile by the digit at `shift`.  Warp w owns items

@@ -57,7 +57,7 @@ def check(B, ctx, n, d, V, seed, topk=20, offsets=None, chosen_override=None):
     feat, top2, rf = B.pr_lmhead_features(ctx, h.cuda(), w.cuda(), chosen.cuda(), topk,
                                           offsets=off_d)
     torch.cuda.synchronize()
-    assert B.pr_ctx_flags(ctx) & B.PR_FLAG_TIMEOUT == 0
+    assert (B.pr_ctx_flags(ctx) & B.PR_FLAG_TIMEOUT) == 0
     o = lmhead.features(bits(h), bits(w), chosen.numpy(), K=topk, offsets=offsets)
     fg = feat.cpu().numpy()
     assert_close(fg, o["feat"], "features", rtol=TOL, atol=TOL)
@@ -123,7 +123,7 @@ def test_lmhead_full_batch_sampled_rows(B, ctx):
     h, w, chosen = W.lmhead_inputs(n, d, V, device="cpu")
     feat, top2, rf = B.pr_lmhead_features(ctx, h.cuda(), w.cuda(), chosen.cuda(), 20)
     torch.cuda.synchronize()
-    assert B.pr_ctx_flags(ctx) & B.PR_FLAG_TIMEOUT == 0
+    assert (B.pr_ctx_flags(ctx) & B.PR_FLAG_TIMEOUT) == 0
     rows = np.array([0, 1, 127, 128, 255, 256, 4607, 4608, 8703, 8704, 8845, 8846])
     o = lmhead.features(bits(h[rows]), bits(w), chosen.numpy()[rows], K=20)
     assert_close(feat.cpu().numpy()[rows], o["feat"], "features", rtol=TOL, atol=TOL)
@@ -136,3 +136,16 @@ def test_lmhead_full_batch_sampled_rows(B, ctx):
             assert list(tg[i]) == list(o["idx"][i]), rows[i]
         else:
             assert x[i, tg[i, 0]] >= srt[i, 0] - 1e-3
+
+
+def test_bounded_wait_runs_out_and_flags(B, ctx):
+    """Failure detection without a stall: the kernels' bounded mbarrier wait,
+    run on a barrier nothing completes with a 1 ms limit, gives up, raises
+    PR_FLAG_TIMEOUT in the context flag word, and the context keeps working."""
+    B.pr_ctx_flags(ctx, clear=True)
+    assert B.pr_selftest_wait(ctx, 1_000_000) is False
+    assert B.pr_ctx_flags(ctx, clear=True) & B.PR_FLAG_TIMEOUT
+    assert B.pr_ctx_flags(ctx) == 0
+    check(B, ctx, 130, 128, 1000, seed=77)  # asserts the flag stays clear
+    with pytest.raises(B.PRError):
+        B.pr_selftest_wait(ctx, -1)
