@@ -5,12 +5,18 @@
 // interpolation between order statistics), a 28-number summary, then a
 // 28 -> 64 -> 64 -> 1 ReLU MLP and a sigmoid.
 //
-// One CTA per request.  Up to Q_CAP rows the four feature columns are loaded
-// into shared memory as order-preserving 32-bit keys and bitonic-sorted
-// together; longer requests find each needed order statistic by radix
-// selection (four 8-bit passes of shared histograms over the request's rows in
-// global memory).  Both give the exact order statistics.  The MLP runs in the
-// same CTA with fixed-order sums.
+// One CTA per request.  Up to Q_SMALL rows each thread takes one row and
+// computes the exact stable rank of its four keys (order-preserving 32-bit
+// keys, one 16-byte word per row in shared memory, read by all threads at
+// once): the count of smaller keys plus equal keys of earlier rows; the row
+// whose rank is a needed index hands its value over.  Up to Q_CAP rows the
+// four columns are bitonic-sorted together: up to 1,024 rows each thread
+// holds a run of keys in registers (register and warp-shuffle stages, one
+// stage through shared memory), above that in shared memory; longer requests
+// find each needed order statistic by radix selection (four 8-bit passes of
+// shared histograms over the request's rows in global memory).  All three
+// give the exact order statistics.  The MLP runs in the same CTA with
+// fixed-order sums.
 #pragma once
 
 #include "pr_device.cuh"
@@ -22,6 +28,7 @@ constexpr int Q_NQ = 7;             // quantile levels
 constexpr int Q_NS = 4 * Q_NQ;      // summary length
 constexpr int Q_H = 64;             // hidden width
 constexpr int Q_CAP = 2048;         // rows sorted in shared memory
+constexpr int Q_SMALL = 256;        // rows ranked by counting (one per thread)
 __constant__ int32_t q_level_a[Q_NQ] = {0, 1, 1, 1, 3, 9, 1};
 __constant__ int32_t q_level_b[Q_NQ] = {1, 10, 4, 2, 4, 10, 1};
 
@@ -29,6 +36,25 @@ __constant__ int32_t q_level_b[Q_NQ] = {1, 10, 4, 2, 4, 10, 1};
 constexpr int QW_W1 = 0, QW_B1 = QW_W1 + Q_H * Q_NS, QW_W2 = QW_B1 + Q_H,
               QW_B2 = QW_W2 + Q_H * Q_H, QW_W3 = QW_B2 + Q_H, QW_B3 = QW_W3 + Q_H,
               QW_SIZE = QW_B3 + 1;
+
+// the MLP's weights in shared memory once the keys are done with (they reuse
+// the key buffer): rows padded to an odd stride, so that the 64 threads of a
+// layer, one output each, read 64 different banks
+constexpr int QS_W1 = 0, QS_B1 = Q_H * (Q_NS + 1), QS_W2 = QS_B1 + Q_H,
+              QS_B2 = QS_W2 + Q_H * (Q_H + 1), QS_W3 = QS_B2 + Q_H, QS_B3 = QS_W3 + Q_H,
+              QS_SIZE = QS_B3 + 1;
+constexpr int QW_PER_T = (QW_SIZE + Q_NT - 1) / Q_NT;  // weights each thread fetches
+static_assert(QS_SIZE <= 4 * Q_CAP, "the weights fit in the key buffer");
+
+// shared-memory position of flat weight g
+__device__ __forceinline__ int q_wpos(int g) {
+  if (g < QW_B1) return QS_W1 + (g / Q_NS) * (Q_NS + 1) + g % Q_NS;
+  if (g < QW_W2) return QS_B1 + (g - QW_B1);
+  if (g < QW_B2) return QS_W2 + ((g - QW_W2) / Q_H) * (Q_H + 1) + (g - QW_W2) % Q_H;
+  if (g < QW_W3) return QS_B2 + (g - QW_B2);
+  if (g < QW_B3) return QS_W3 + (g - QW_W3);
+  return QS_B3;
+}
 
 struct QArgs {
   const float* feat;
@@ -65,7 +91,7 @@ __device__ uint32_t q_select(const float* __restrict__ feat, int64_t lo, int T, 
   uint32_t rank = (uint32_t)r;
   const int slot = q_slot(f);
   for (int shift = 24; shift >= 0; shift -= 8) {
-    hist[tid] = 0;
+    if (tid < 256) hist[tid] = 0;
     __syncthreads();
     for (int t = tid; t < T; t += Q_NT) {
       const uint32_t k = q_key(feat[(lo + t) * NFEAT + slot]);
@@ -107,7 +133,68 @@ __device__ uint32_t q_select(const float* __restrict__ feat, int64_t lo, int T, 
   return prefix;
 }
 
-__global__ void __launch_bounds__(Q_NT) qmlp_requests(const QArgs a) {
+// Ascending bitonic sort of the four columns col f = qs + (f << ln2) of n2 =
+// 2^ln2 keys each, n2 = 64 E (512 or 1,024), by the whole CTA: thread t
+// holds the E consecutive keys c0 .. c0 + E - 1 of one column (two warps per
+// column).  A compare-exchange stage of partner distance j runs in registers
+// for j < E, between the lanes of a warp (shfl.xor) for j < 32 E, and through
+// shared memory only for j = n2 / 2.
+template <int E>
+__device__ void q_bitonic(uint32_t* qs, int ln2) {
+  const int n2 = 1 << ln2, tid = threadIdx.x;
+  const int per_col = n2 / E;  // threads per column
+  const int c0 = (tid % per_col) * E;
+  uint32_t* col = qs + ((tid / per_col) << ln2);
+  uint32_t v[E];
+#pragma unroll
+  for (int e = 0; e < E; ++e) v[e] = col[c0 + e];
+  for (int k = 2; k <= n2; k <<= 1) {
+    for (int j = k >> 1; j >= E; j >>= 1) {
+      if (j >= 32 * E) {  // the other warp of the column
+        __syncthreads();
+#pragma unroll
+        for (int e = 0; e < E; ++e) col[c0 + e] = v[e];
+        __syncthreads();
+#pragma unroll
+        for (int e = 0; e < E; ++e) {
+          const int c = c0 + e;
+          const uint32_t p = col[c ^ j];
+          const bool keep_min = ((c & j) == 0) == ((c & k) == 0);
+          v[e] = keep_min ? min(v[e], p) : max(v[e], p);
+        }
+      } else {
+        const int lm = j / E;  // lane distance
+#pragma unroll
+        for (int e = 0; e < E; ++e) {
+          const int c = c0 + e;
+          const uint32_t p = __shfl_xor_sync(FULL, v[e], lm);
+          const bool keep_min = ((c & j) == 0) == ((c & k) == 0);
+          v[e] = keep_min ? min(v[e], p) : max(v[e], p);
+        }
+      }
+    }
+#pragma unroll
+    for (int jj = E / 2; jj >= 1; jj >>= 1) {  // inside the thread's keys
+      if (jj < k) {
+#pragma unroll
+        for (int e = 0; e < E; ++e) {
+          if ((e & jj) == 0) {
+            const uint32_t x = v[e], y = v[e + jj];
+            const bool up = ((c0 + e) & k) == 0;
+            const uint32_t lo = min(x, y), hi = max(x, y);
+            v[e] = up ? lo : hi;
+            v[e + jj] = up ? hi : lo;
+          }
+        }
+      }
+    }
+  }
+  __syncthreads();
+#pragma unroll
+  for (int e = 0; e < E; ++e) col[c0 + e] = v[e];
+}
+
+__global__ void __launch_bounds__(Q_NT, 3) qmlp_requests(const QArgs a) {
   extern __shared__ __align__(16) uint32_t qs[];  // [4][n2] keys (shared-memory path)
   __shared__ float qv[Q_NS];
   __shared__ float h1[Q_H], h2[Q_H];
@@ -126,6 +213,14 @@ __global__ void __launch_bounds__(Q_NT) qmlp_requests(const QArgs a) {
     return;
   }
   const int T = (int)(hi - lo);
+  // the MLP's weights, fetched now (coalesced) so that their latency overlaps
+  // the key loads and the sort
+  float wr[QW_PER_T];
+#pragma unroll
+  for (int i = 0; i < QW_PER_T; ++i) {
+    const int g = tid + i * Q_NT;
+    wr[i] = g < QW_SIZE ? __ldg(a.w + g) : 0.f;
+  }
   if (T == 0) {
     if (tid == 0) {
       a.score[r] = 0.f;
@@ -152,8 +247,64 @@ __global__ void __launch_bounds__(Q_NT) qmlp_requests(const QArgs a) {
     return;
   }
 
-  if (T <= Q_CAP) {
-    int ln2 = 0;  // n2 = 2^ln2 >= T
+  if (T <= Q_SMALL) {
+    uint4* q4 = reinterpret_cast<uint4*>(qs);  // row t: the keys of l, m, h, rho
+    __shared__ float sval[Q_NS];
+    uint4 mine = make_uint4(0u, 0u, 0u, 0u);
+    if (tid < T) {
+      const float* rec = a.feat + (lo + tid) * NFEAT;
+      mine = make_uint4(q_key(rec[q_slot(0)]), q_key(rec[q_slot(1)]), q_key(rec[q_slot(2)]),
+                        q_key(rec[q_slot(3)]));
+      q4[tid] = mine;
+    }
+    __syncthreads();
+    if (tid < T) {
+      // stable rank of each of the row's four keys
+      uint32_t r0 = 0, r1 = 0, r2 = 0, r3 = 0;
+      int j = 0;
+      for (; j < tid; ++j) {  // earlier rows: smaller or equal
+        const uint4 o = q4[j];
+        r0 += o.x <= mine.x;
+        r1 += o.y <= mine.y;
+        r2 += o.z <= mine.z;
+        r3 += o.w <= mine.w;
+      }
+      for (++j; j < T; ++j) {  // later rows: smaller only
+        const uint4 o = q4[j];
+        r0 += o.x < mine.x;
+        r1 += o.y < mine.y;
+        r2 += o.z < mine.z;
+        r3 += o.w < mine.w;
+      }
+      // hand over the needed order statistics (the lower one of a level to
+      // sval, the upper neighbour of an interpolated level to qv)
+      auto give = [&](int f, uint32_t r, uint32_t key) {
+        for (int lv = 0; lv < Q_NQ; ++lv) {
+          const uint32_t num = (uint32_t)q_level_a[lv] * (uint32_t)(T - 1);
+          const uint32_t b = (uint32_t)q_level_b[lv];
+          const uint32_t lo_i = num / b;
+          if (r == lo_i) sval[f * Q_NQ + lv] = q_unkey(key);
+          if (num != lo_i * b && r == lo_i + 1) qv[f * Q_NQ + lv] = q_unkey(key);
+        }
+      };
+      give(0, r0, mine.x);
+      give(1, r1, mine.y);
+      give(2, r2, mine.z);
+      give(3, r3, mine.w);
+    }
+    __syncthreads();
+    if (tid < Q_NS) {
+      const int f = tid / Q_NQ, lv = tid - f * Q_NQ;
+      const int64_t num = (int64_t)q_level_a[lv] * (T - 1);
+      const int b = q_level_b[lv];
+      const int lo_i = (int)(num / b), rem = (int)(num - (int64_t)lo_i * b);
+      const float xl = sval[tid];
+      float q = xl;
+      if (rem) q = xl + ((float)rem / (float)b) * (qv[tid] - xl);
+      qv[tid] = q;
+    }
+  } else if (T <= Q_CAP) {
+    int ln2 = 9;  // n2 = 2^ln2 >= T, at least 512
     while ((1 << ln2) < T) ++ln2;
     const int n2 = 1 << ln2;
     for (int i = tid; i < 4 * n2; i += Q_NT) {
@@ -161,25 +312,32 @@ __global__ void __launch_bounds__(Q_NT) qmlp_requests(const QArgs a) {
       qs[i] = t < T ? q_key(a.feat[(lo + t) * NFEAT + q_slot(f)]) : 0xffffffffu;
     }
     __syncthreads();
-    // bitonic sort of the four columns, ascending (powers of two: shifts, masks)
-    const int half = n2 >> 1, lh = ln2 - 1;
-    for (int k = 2; k <= n2; k <<= 1) {
-      for (int j = k >> 1; j > 0; j >>= 1) {
-        for (int idx = tid; idx < 4 * half; idx += Q_NT) {
-          const int f = idx >> lh, t = idx & (half - 1);
-          const int i = ((t & ~(j - 1)) << 1) | (t & (j - 1));
-          const int l = i + j;
-          uint32_t* col = qs + (f << ln2);
-          const uint32_t x = col[i], y = col[l];
-          const bool up = (i & k) == 0;
-          if ((x > y) == up) {
-            col[i] = y;
-            col[l] = x;
+    if (ln2 == 9) {
+      q_bitonic<8>(qs, 9);
+    } else if (ln2 == 10) {
+      q_bitonic<16>(qs, 10);
+    } else {  // 2,048 keys per column: shared-memory stages (32 keys per thread
+              // would take the registers that the other requests' CTAs need)
+      const int half = n2 >> 1, lh = ln2 - 1;
+      for (int k = 2; k <= n2; k <<= 1) {
+        for (int j = k >> 1; j > 0; j >>= 1) {
+          for (int idx = tid; idx < 4 * half; idx += Q_NT) {
+            const int f = idx >> lh, t = idx & (half - 1);
+            const int i = ((t & ~(j - 1)) << 1) | (t & (j - 1));
+            const int l = i + j;
+            uint32_t* col = qs + (f << ln2);
+            const uint32_t x = col[i], y = col[l];
+            const bool up = (i & k) == 0;
+            if ((x > y) == up) {
+              col[i] = y;
+              col[l] = x;
+            }
           }
+          __syncthreads();
         }
-        __syncthreads();
       }
     }
+    __syncthreads();
     if (tid < Q_NS) {
       const int f = tid / Q_NQ, j = tid - f * Q_NQ;
       const int64_t num = (int64_t)q_level_a[j] * (T - 1);
@@ -211,22 +369,28 @@ __global__ void __launch_bounds__(Q_NT) qmlp_requests(const QArgs a) {
   }
   __syncthreads();
 
-  // MLP 28 -> 64 -> 64 -> 1 (sums in input order)
-  const float* W = a.w;
+  // MLP 28 -> 64 -> 64 -> 1 (sums in input order), weights from shared memory
+  float* W = reinterpret_cast<float*>(qs);
+#pragma unroll
+  for (int i = 0; i < QW_PER_T; ++i) {
+    const int g = tid + i * Q_NT;
+    if (g < QW_SIZE) W[q_wpos(g)] = wr[i];
+  }
+  __syncthreads();
   if (tid < Q_H) {
-    float s = __ldg(W + QW_B1 + tid);
-    for (int i = 0; i < Q_NS; ++i) s = fmaf(__ldg(W + QW_W1 + tid * Q_NS + i), qv[i], s);
+    float s = W[QS_B1 + tid];
+    for (int i = 0; i < Q_NS; ++i) s = fmaf(W[QS_W1 + tid * (Q_NS + 1) + i], qv[i], s);
     h1[tid] = fmaxf(s, 0.f);
   }
   __syncthreads();
   if (tid < Q_H) {
-    float s = __ldg(W + QW_B2 + tid);
-    for (int i = 0; i < Q_H; ++i) s = fmaf(__ldg(W + QW_W2 + tid * Q_H + i), h1[i], s);
+    float s = W[QS_B2 + tid];
+    for (int i = 0; i < Q_H; ++i) s = fmaf(W[QS_W2 + tid * (Q_H + 1) + i], h1[i], s);
     h2[tid] = fmaxf(s, 0.f);
   }
   __syncthreads();
   if (warp < 2) {
-    float z = __ldg(W + QW_W3 + tid) * h2[tid];
+    float z = W[QS_W3 + tid] * h2[tid];
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) z += __shfl_xor_sync(FULL, z, o);
     if (lane == 0) zpart[warp] = z;
@@ -234,7 +398,7 @@ __global__ void __launch_bounds__(Q_NT) qmlp_requests(const QArgs a) {
   if (a.summary && tid < Q_NS) a.summary[r * Q_NS + tid] = qv[tid];
   __syncthreads();
   if (tid == 0) {
-    const float z = (zpart[0] + zpart[1]) + __ldg(W + QW_B3);
+    const float z = (zpart[0] + zpart[1]) + W[QS_B3];
     a.score[r] = 1.f / (1.f + expf(-z));
     a.ship[r] = (z >= a.zthr) ? 1 : 0;
     a.req_flags[r] = fl;
