@@ -149,3 +149,25 @@ def test_bounded_wait_runs_out_and_flags(B, ctx):
     check(B, ctx, 130, 128, 1000, seed=77)  # asserts the flag stays clear
     with pytest.raises(B.PRError):
         B.pr_selftest_wait(ctx, -1)
+
+
+def test_lmhead_exact_ties_across_splits(B, ctx):
+    """A weight row duplicated at two far indices (other tiles, splits and
+    column halves) and hidden states along it: the three logits are equal bit
+    for bit (same products in the same order), so the top-2 must be the two
+    lowest indices and the margin exactly 0, as in the oracle's (value desc,
+    index asc) order."""
+    n, d, V = 6, 256, 20000
+    h, w, chosen = make(n, d, V, seed=91)
+    w[7368] = w[17]  # column half 1 of its tile; 17 and 19999 are in half 0
+    w[19999] = w[17]
+    h[:3] = (w[17].float() * 4.0).to(torch.bfloat16)  # logit |w17|^2 * 4: far above the rest
+    feat, top2, rf = B.pr_lmhead_features(ctx, h.cuda(), w.cuda(), chosen.cuda(), 20)
+    torch.cuda.synchronize()
+    o = lmhead.features(bits(h), bits(w), chosen.numpy(), K=20)
+    assert_close(feat.cpu().numpy(), o["feat"], "features", rtol=TOL, atol=TOL)
+    tg = top2.cpu().numpy()
+    for r in range(3):
+        assert list(tg[r]) == [17, 7368], tg[r]
+        assert list(o["idx"][r]) == [17, 7368]
+        assert feat[r, 2].item() == 0.0  # margin p1 - p2
