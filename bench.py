@@ -342,6 +342,9 @@ def run_gb300(args):
         xs = W.to_oracle_array(x[lo:hi])
         cs = ch[lo:hi].cpu().numpy()
         o, dt, rows = oracle_sample(wl, xs, cs, 0, req_hi, cores)
+        # the same oracle on one core, on request 0 alone
+        hi1 = int(wl.offsets[1])
+        _, dt1, rows1 = oracle_sample(wl, xs[:hi1], cs[:hi1], 0, 1, 1)
         g_agg = agg[:req_hi].cpu().numpy().astype(np.float64)
         g_score = score[:req_hi].cpu().numpy().astype(np.float64)
         ok = bool(np.all(np.abs(g_agg - o["agg"]) <= 1e-5 + 1e-4 * np.abs(o["agg"])) and
@@ -370,6 +373,10 @@ def run_gb300(args):
             "cpu_baseline": {"value": rows / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
                              "sample": "requests 0..%d (%d rows), float64 C oracle, %d threads" % (
                                  req_hi - 1, rows, cores)},
+            "cpu_baseline_one_core": {"value": rows1 / dt1, "unit": UNIT, "cores": 1,
+                                      "kind": "oracle",
+                                      "sample": "request 0 (%d rows), float64 C oracle, 1 thread"
+                                                % rows1},
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d // world * world,
                     "d2h_bytes_per_step": d2h, "api": "pr_route_host (pinned host buffers)"},
             "gpu_launches": launches,
