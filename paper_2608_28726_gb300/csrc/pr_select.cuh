@@ -186,18 +186,20 @@ __global__ void __launch_bounds__(SEL_NT) sel_scan_digit(uint32_t* __restrict__ 
   if (tid == 0) total[blockIdx.x] = carry;
 }
 
-// Stable scatter of one tile by the digit at `shift`.  Warp w owns items
-// [w * 512, (w + 1) * 512) of the tile in 16 rounds of 32 consecutive items;
-// the lanes holding the same digit in a round are found with match.any and
-// ranked by lane, rounds in order, so the tile order of equal digits is
-// kept.  The tile is then laid out in shared memory in digit
-// order and written out in that order: each digit's run goes to consecutive
-// addresses.
+// Stable scatter of the tiles by the digit at `shift`.  Persistent: CTA b
+// takes tiles b, b + grid, b + 2 grid, ..., and loads the next tile's keys,
+// labels and offsets while it ranks and writes the current one.  Warp w owns
+// items [w * 256, (w + 1) * 256) of a tile in 8 rounds of 32 consecutive
+// items; the lanes holding the same digit in a round are found with
+// match.any and ranked by lane, rounds in order, so the tile order of equal
+// digits is kept.  The tile is then laid out in shared memory in digit order
+// and written out in that order: each digit's run goes to consecutive
+// addresses.  Indices are 32-bit (n < 2^31).
 __global__ void __launch_bounds__(SEL_NT) sel_scatter(const uint32_t* __restrict__ key_in,
                                                       const uint8_t* __restrict__ val_in,
-                                                      int64_t n, int shift,
+                                                      int64_t n64, int shift,
                                                       const uint32_t* __restrict__ counts,
-                                                      int64_t ntiles,
+                                                      int64_t ntiles64,
                                                       const uint32_t* __restrict__ total,
                                                       uint32_t* __restrict__ key_out,
                                                       uint8_t* __restrict__ val_out) {
@@ -209,90 +211,110 @@ __global__ void __launch_bounds__(SEL_NT) sel_scatter(const uint32_t* __restrict
   __shared__ uint32_t sk[SEL_TILE];
   __shared__ uint8_t sv[SEL_TILE];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  // this tile's offsets: loaded first, their latency overlaps the key loads
-  const uint32_t tv = total[tid];
-  const uint32_t before_tiles = counts[(int64_t)tid * ntiles + blockIdx.x];
-#pragma unroll
-  for (int w = 0; w < SEL_NT / 32; ++w) wcnt[w][tid] = 0;
-  __syncthreads();
+  const uint32_t n = (uint32_t)n64, ntiles = (uint32_t)ntiles64;
   constexpr int PER_WARP = SEL_TILE / (SEL_NT / 32);
-  const int64_t tile0 = (int64_t)blockIdx.x * SEL_TILE;
-  const int64_t base = tile0 + (int64_t)warp * PER_WARP;
-  const int64_t left = n - tile0;
-  const int nt = left < SEL_TILE ? (int)left : SEL_TILE;  // items in this tile
-  uint32_t k[SEL_IPT], pos[SEL_IPT];
-  uint8_t v[SEL_IPT];
   const unsigned lt = (1u << lane) - 1u;
+  const uint32_t tv = total[tid];
+  uint32_t k[SEL_IPT];
+  uint8_t v[SEL_IPT];
+  uint32_t bt = 0;  // items of digit tid in the tiles before the current one
+  auto fetch = [&](uint32_t t, uint32_t (&kk)[SEL_IPT], uint8_t (&vv)[SEL_IPT], uint32_t& b) {
+    const uint32_t base = t * (uint32_t)SEL_TILE + (uint32_t)warp * PER_WARP;
 #pragma unroll
-  for (int r = 0; r < SEL_IPT; ++r) {  // all loads first
-    const int64_t i = base + r * 32 + lane;
-    k[r] = i < n ? key_in[i] : 0u;
-    v[r] = i < n ? val_in[i] : 0;
-  }
-#pragma unroll
-  for (int r = 0; r < SEL_IPT; ++r) {
-    const bool ok = base + r * 32 + lane < n;
-    const uint32_t d = (k[r] >> shift) & 0xff;
-    const unsigned peers = __match_any_sync(FULL, ok ? d : SEL_RADIX);  // SEL_RADIX: no item
-    const uint32_t rank = __popc(peers & lt);
-    const uint32_t before = ok ? wcnt[warp][d] : 0u;
-    __syncwarp();
-    if (ok && rank == 0) wcnt[warp][d] = before + __popc(peers);
-    __syncwarp();
-    pos[r] = before + rank;
-  }
-  __syncthreads();
-  {
-    // per digit (thread tid = digit): exclusive prefix over the warps, and the
-    // tile's count of the digit
-    uint32_t run = 0;
-#pragma unroll
-    for (int w = 0; w < SEL_NT / 32; ++w) {
-      const uint32_t c = wcnt[w][tid];
-      wcnt[w][tid] = run;
-      run += c;
+    for (int r = 0; r < SEL_IPT; ++r) {
+      const uint32_t i = base + r * 32 + lane;
+      kk[r] = i < n ? key_in[i] : 0u;
+      vv[r] = i < n ? val_in[i] : 0;
     }
-    // exclusive scans over digits: of the tile's counts, and of the totals
-    uint32_t x = run, y = tv;
+    b = counts[(size_t)tid * ntiles + t];
+  };
+  uint32_t tile = blockIdx.x;
+  if (tile < ntiles) fetch(tile, k, v, bt);
+  for (; tile < ntiles; tile += gridDim.x) {
+    const uint32_t next = tile + gridDim.x;
+    uint32_t kn[SEL_IPT];
+    uint8_t vn[SEL_IPT];
+    uint32_t btn = 0;
+    if (next < ntiles) fetch(next, kn, vn, btn);  // in flight while this tile is done
 #pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const uint32_t xx = __shfl_up_sync(FULL, x, o), yy = __shfl_up_sync(FULL, y, o);
-      if (lane >= o) {
-        x += xx;
-        y += yy;
-      }
-    }
-    if (lane == 31) {
-      ws[warp] = x;
-      ws2[warp] = y;
+    for (int w = 0; w < SEL_NT / 32; ++w) wcnt[w][tid] = 0;
+    __syncthreads();
+    const uint32_t tile0 = tile * (uint32_t)SEL_TILE;
+    const uint32_t base = tile0 + (uint32_t)warp * PER_WARP;
+    const uint32_t nt = n - tile0 < (uint32_t)SEL_TILE ? n - tile0 : (uint32_t)SEL_TILE;
+    uint32_t pos[SEL_IPT];
+#pragma unroll
+    for (int r = 0; r < SEL_IPT; ++r) {
+      const bool ok = base + r * 32 + lane < n;
+      const uint32_t d = (k[r] >> shift) & 0xff;
+      const unsigned peers = __match_any_sync(FULL, ok ? d : SEL_RADIX);  // SEL_RADIX: no item
+      const uint32_t rank = __popc(peers & lt);
+      const uint32_t before = ok ? wcnt[warp][d] : 0u;
+      __syncwarp();
+      if (ok && rank == 0) wcnt[warp][d] = before + __popc(peers);
+      __syncwarp();
+      pos[r] = before + rank;
     }
     __syncthreads();
-    uint32_t xb = 0, yb = 0;
-    for (int w = 0; w < warp; ++w) {
-      xb += ws[w];
-      yb += ws2[w];
-    }
-    const uint32_t tile_off_d = xb + x - run;
-    toff[tid] = tile_off_d;
-    gbase[tid] = (yb + y - tv) + before_tiles - tile_off_d;
-  }
-  __syncthreads();
+    {
+      // per digit (thread tid = digit): exclusive prefix over the warps, and
+      // the tile's count of the digit
+      uint32_t run = 0;
 #pragma unroll
-  for (int r = 0; r < SEL_IPT; ++r) {
-    const int64_t i = base + r * 32 + lane;
-    if (i < n) {
-      const uint32_t d = (k[r] >> shift) & 0xff;
-      const uint32_t p = toff[d] + wcnt[warp][d] + pos[r];
-      sk[p] = k[r];
-      sv[p] = v[r];
+      for (int w = 0; w < SEL_NT / 32; ++w) {
+        const uint32_t c = wcnt[w][tid];
+        wcnt[w][tid] = run;
+        run += c;
+      }
+      // exclusive scans over digits: of the tile's counts, and of the totals
+      uint32_t x = run, y = tv;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t xx = __shfl_up_sync(FULL, x, o), yy = __shfl_up_sync(FULL, y, o);
+        if (lane >= o) {
+          x += xx;
+          y += yy;
+        }
+      }
+      if (lane == 31) {
+        ws[warp] = x;
+        ws2[warp] = y;
+      }
+      __syncthreads();
+      uint32_t xb = 0, yb = 0;
+      for (int w = 0; w < warp; ++w) {
+        xb += ws[w];
+        yb += ws2[w];
+      }
+      const uint32_t tile_off_d = xb + x - run;
+      toff[tid] = tile_off_d;
+      gbase[tid] = (yb + y - tv) + bt - tile_off_d;
     }
-  }
-  __syncthreads();
-  for (int j = tid; j < nt; j += SEL_NT) {
-    const uint32_t kk = sk[j];
-    const uint32_t o = gbase[(kk >> shift) & 0xff] + (uint32_t)j;
-    key_out[o] = kk;
-    val_out[o] = sv[j];
+    __syncthreads();
+#pragma unroll
+    for (int r = 0; r < SEL_IPT; ++r) {
+      const uint32_t i = base + r * 32 + lane;
+      if (i < n) {
+        const uint32_t d = (k[r] >> shift) & 0xff;
+        const uint32_t p = toff[d] + wcnt[warp][d] + pos[r];
+        sk[p] = k[r];
+        sv[p] = v[r];
+      }
+    }
+    __syncthreads();
+    for (uint32_t j = tid; j < nt; j += SEL_NT) {
+      const uint32_t kk = sk[j];
+      const uint32_t o = gbase[(kk >> shift) & 0xff] + j;
+      key_out[o] = kk;
+      val_out[o] = sv[j];
+    }
+    __syncthreads();  // sk, sv, gbase, toff and wcnt are free for the next tile
+#pragma unroll
+    for (int r = 0; r < SEL_IPT; ++r) {
+      k[r] = kn[r];
+      v[r] = vn[r];
+    }
+    bt = btn;
   }
 }
 

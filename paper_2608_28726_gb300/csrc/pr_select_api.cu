@@ -96,6 +96,15 @@ pr_status pr_selective_metrics(pr_ctx* c, const float* scores, const uint8_t* la
   prk::SelResult* res = reinterpret_cast<prk::SelResult*>(w + L.out);
   const int64_t ntiles = (n + prk::SEL_TILE - 1) / prk::SEL_TILE;
   const unsigned g_tiles = (unsigned)ntiles;
+  // the scatter is persistent: one wave of resident CTAs
+  static int scatter_bps = 0;
+  if (scatter_bps == 0) {
+    int b = 0;
+    PR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, prk::sel_scatter, prk::SEL_NT, 0));
+    scatter_bps = b > 0 ? b : 1;
+  }
+  const unsigned g_scatter =
+      (unsigned)std::min<int64_t>(ntiles, (int64_t)c->num_sms * scatter_bps);
   int launches = 0;
   // after each launch: count it, check it, and (PR_OPT_TIMING) record an event
   auto launched = [&]() -> pr_status {
@@ -118,8 +127,8 @@ pr_status pr_selective_metrics(pr_ctx* c, const float* scores, const uint8_t* la
     PR_LAUNCHED();
     prk::sel_scan_digit<<<prk::SEL_RADIX, prk::SEL_NT, 0, s>>>(counts, ntiles, total);
     PR_LAUNCHED();
-    prk::sel_scatter<<<g_tiles, prk::SEL_NT, 0, s>>>(key[cur], val[cur], n, 8 * pass, counts,
-                                                     ntiles, total, key[nxt], val[nxt]);
+    prk::sel_scatter<<<g_scatter, prk::SEL_NT, 0, s>>>(key[cur], val[cur], n, 8 * pass, counts,
+                                                       ntiles, total, key[nxt], val[nxt]);
     PR_LAUNCHED();
   }
   // four passes: the sorted arrays are back in key[0], val[0]
