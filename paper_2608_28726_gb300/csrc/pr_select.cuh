@@ -27,6 +27,8 @@ namespace prk {
 constexpr int SEL_NT = 256;                 // threads per CTA
 constexpr int SEL_IPT = 8;                  // items per thread
 constexpr int SEL_TILE = SEL_NT * SEL_IPT;  // items per tile
+constexpr int SR_IPT = 16;                  // items per thread in the radix passes: longer
+constexpr int SR_TILE = SEL_NT * SR_IPT;    // digit runs per tile, half the tile counts
 constexpr int SEL_RADIX = 256;
 constexpr uint32_t SEL_NONFINITE = 0xffffffffu;
 
@@ -104,9 +106,9 @@ __global__ void __launch_bounds__(SEL_NT) sel_hist(const uint32_t* __restrict__ 
 #pragma unroll
   for (int w = 0; w < SEL_NT / 32; ++w) h[w][threadIdx.x] = 0;
   __syncthreads();
-  const int64_t base = (int64_t)blockIdx.x * SEL_TILE;
+  const int64_t base = (int64_t)blockIdx.x * SR_TILE;
 #pragma unroll
-  for (int j = 0; j < SEL_IPT / 4; ++j) {
+  for (int j = 0; j < SR_IPT / 4; ++j) {
     const int64_t i = base + 4 * ((int64_t)j * SEL_NT + threadIdx.x);
     if (i + 3 < n) {
       const uint4 k = *reinterpret_cast<const uint4*>(key + i);
@@ -189,7 +191,7 @@ __global__ void __launch_bounds__(SEL_NT) sel_scan_digit(uint32_t* __restrict__ 
 // Stable scatter of the tiles by the digit at `shift`.  Persistent: CTA b
 // takes tiles b, b + grid, b + 2 grid, ..., and loads the next tile's keys,
 // labels and offsets while it ranks and writes the current one.  Warp w owns
-// items [w * 256, (w + 1) * 256) of a tile in 8 rounds of 32 consecutive
+// items [w * 512, (w + 1) * 512) of a tile in 16 rounds of 32 consecutive
 // items; the lanes holding the same digit in a round are found with
 // match.any and ranked by lane, rounds in order, so the tile order of equal
 // digits is kept.  The tile is then laid out in shared memory in digit order
@@ -208,20 +210,20 @@ __global__ void __launch_bounds__(SEL_NT) sel_scatter(const uint32_t* __restrict
                                          // minus the digit's offset inside the tile
   __shared__ uint32_t toff[SEL_RADIX];   // offset of digit d inside the tile
   __shared__ uint32_t ws[SEL_NT / 32], ws2[SEL_NT / 32];
-  __shared__ uint32_t sk[SEL_TILE];
-  __shared__ uint8_t sv[SEL_TILE];
+  __shared__ uint32_t sk[SR_TILE];
+  __shared__ uint8_t sv[SR_TILE];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const uint32_t n = (uint32_t)n64, ntiles = (uint32_t)ntiles64;
-  constexpr int PER_WARP = SEL_TILE / (SEL_NT / 32);
+  constexpr int PER_WARP = SR_TILE / (SEL_NT / 32);
   const unsigned lt = (1u << lane) - 1u;
   const uint32_t tv = total[tid];
-  uint32_t k[SEL_IPT];
-  uint8_t v[SEL_IPT];
+  uint32_t k[SR_IPT];
+  uint8_t v[SR_IPT];
   uint32_t bt = 0;  // items of digit tid in the tiles before the current one
-  auto fetch = [&](uint32_t t, uint32_t (&kk)[SEL_IPT], uint8_t (&vv)[SEL_IPT], uint32_t& b) {
-    const uint32_t base = t * (uint32_t)SEL_TILE + (uint32_t)warp * PER_WARP;
+  auto fetch = [&](uint32_t t, uint32_t (&kk)[SR_IPT], uint8_t (&vv)[SR_IPT], uint32_t& b) {
+    const uint32_t base = t * (uint32_t)SR_TILE + (uint32_t)warp * PER_WARP;
 #pragma unroll
-    for (int r = 0; r < SEL_IPT; ++r) {
+    for (int r = 0; r < SR_IPT; ++r) {
       const uint32_t i = base + r * 32 + lane;
       kk[r] = i < n ? key_in[i] : 0u;
       vv[r] = i < n ? val_in[i] : 0;
@@ -232,19 +234,19 @@ __global__ void __launch_bounds__(SEL_NT) sel_scatter(const uint32_t* __restrict
   if (tile < ntiles) fetch(tile, k, v, bt);
   for (; tile < ntiles; tile += gridDim.x) {
     const uint32_t next = tile + gridDim.x;
-    uint32_t kn[SEL_IPT];
-    uint8_t vn[SEL_IPT];
+    uint32_t kn[SR_IPT];
+    uint8_t vn[SR_IPT];
     uint32_t btn = 0;
     if (next < ntiles) fetch(next, kn, vn, btn);  // in flight while this tile is done
 #pragma unroll
     for (int w = 0; w < SEL_NT / 32; ++w) wcnt[w][tid] = 0;
     __syncthreads();
-    const uint32_t tile0 = tile * (uint32_t)SEL_TILE;
+    const uint32_t tile0 = tile * (uint32_t)SR_TILE;
     const uint32_t base = tile0 + (uint32_t)warp * PER_WARP;
-    const uint32_t nt = n - tile0 < (uint32_t)SEL_TILE ? n - tile0 : (uint32_t)SEL_TILE;
-    uint32_t pos[SEL_IPT];
+    const uint32_t nt = n - tile0 < (uint32_t)SR_TILE ? n - tile0 : (uint32_t)SR_TILE;
+    uint32_t pos[SR_IPT];
 #pragma unroll
-    for (int r = 0; r < SEL_IPT; ++r) {
+    for (int r = 0; r < SR_IPT; ++r) {
       const bool ok = base + r * 32 + lane < n;
       const uint32_t d = (k[r] >> shift) & 0xff;
       const unsigned peers = __match_any_sync(FULL, ok ? d : SEL_RADIX);  // SEL_RADIX: no item
@@ -292,7 +294,7 @@ __global__ void __launch_bounds__(SEL_NT) sel_scatter(const uint32_t* __restrict
     }
     __syncthreads();
 #pragma unroll
-    for (int r = 0; r < SEL_IPT; ++r) {
+    for (int r = 0; r < SR_IPT; ++r) {
       const uint32_t i = base + r * 32 + lane;
       if (i < n) {
         const uint32_t d = (k[r] >> shift) & 0xff;
@@ -310,7 +312,7 @@ __global__ void __launch_bounds__(SEL_NT) sel_scatter(const uint32_t* __restrict
     }
     __syncthreads();  // sk, sv, gbase, toff and wcnt are free for the next tile
 #pragma unroll
-    for (int r = 0; r < SEL_IPT; ++r) {
+    for (int r = 0; r < SR_IPT; ++r) {
       k[r] = kn[r];
       v[r] = vn[r];
     }

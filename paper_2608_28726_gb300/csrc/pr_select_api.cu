@@ -103,8 +103,9 @@ pr_status pr_selective_metrics(pr_ctx* c, const float* scores, const uint8_t* la
     PR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, prk::sel_scatter, prk::SEL_NT, 0));
     scatter_bps = b > 0 ? b : 1;
   }
+  const int64_t rtiles = (n + prk::SR_TILE - 1) / prk::SR_TILE;  // tiles of the radix passes
   const unsigned g_scatter =
-      (unsigned)std::min<int64_t>(ntiles, (int64_t)c->num_sms * scatter_bps);
+      (unsigned)std::min<int64_t>(rtiles, (int64_t)c->num_sms * scatter_bps);
   int launches = 0;
   // after each launch: count it, check it, and (PR_OPT_TIMING) record an event
   auto launched = [&]() -> pr_status {
@@ -123,12 +124,12 @@ pr_status pr_selective_metrics(pr_ctx* c, const float* scores, const uint8_t* la
   PR_LAUNCHED();
   for (int pass = 0; pass < 4; ++pass) {
     const int cur = pass & 1, nxt = cur ^ 1;
-    prk::sel_hist<<<g_tiles, prk::SEL_NT, 0, s>>>(key[cur], n, 8 * pass, counts, ntiles);
+    prk::sel_hist<<<(unsigned)rtiles, prk::SEL_NT, 0, s>>>(key[cur], n, 8 * pass, counts, rtiles);
     PR_LAUNCHED();
-    prk::sel_scan_digit<<<prk::SEL_RADIX, prk::SEL_NT, 0, s>>>(counts, ntiles, total);
+    prk::sel_scan_digit<<<prk::SEL_RADIX, prk::SEL_NT, 0, s>>>(counts, rtiles, total);
     PR_LAUNCHED();
     prk::sel_scatter<<<g_scatter, prk::SEL_NT, 0, s>>>(key[cur], val[cur], n, 8 * pass, counts,
-                                                       ntiles, total, key[nxt], val[nxt]);
+                                                       rtiles, total, key[nxt], val[nxt]);
     PR_LAUNCHED();
   }
   // four passes: the sorted arrays are back in key[0], val[0]

@@ -66,7 +66,7 @@ def check(g, s, y, q):
         assert (np.isnan(a) and np.isnan(b)) or abs(a - b) <= tol, (name, a, b)
 
 
-@pytest.mark.parametrize("n", [1, 2, 31, 2047, 2048, 2049, 4097, 12289, 100003])
+@pytest.mark.parametrize("n", [1, 2, 31, 2047, 2048, 2049, 4095, 4096, 4097, 12289, 100003])
 def test_selective_matches_oracle_sizes(B, ctx, n):
     # tile edges (2,048 items per tile) and ragged tails
     s, y = make(n, seed=n, levels=97, nan_frac=0.03)
