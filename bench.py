@@ -796,6 +796,10 @@ def run_lmhead_workload(args):
     # generated on the CPU (the oracle's child process draws the same values)
     hidden, weight, chosen = (t.to(dev) for t in W.lmhead_inputs(n, d, V, device="cpu"))
     off = torch.from_numpy(wl.offsets).to(dev)
+    if args.lm_rows > 0:  # the first rows only, as one request (e.g. one decode step's batch)
+        n = min(args.lm_rows, n)
+        hidden, chosen = hidden[:n].contiguous(), chosen[:n].contiguous()
+        off = torch.tensor([0, n], dtype=torch.int64, device=dev)
     ctx = B.pr_ctx_create(local, max_rows=n, max_requests=wl.n_req)
     stream = torch.cuda.current_stream(dev)
     feat = torch.empty(n, 8, device=dev)
@@ -909,8 +913,11 @@ def run_lmhead_workload(args):
             "value": n * world / (ms / 1e3), "unit": UNIT, "n_gpus": world, "steps": K,
             "warmup": max(3, args.warmup), "ms_per_step": ms, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": "LM head + row features: %d hidden states (the full-response "
-                                   "layout), d=%d, V=%d bf16 head (1.09 GB), seeded" % (n, d, V),
+            "config": {"workload": "LM head + row features: %d hidden states (%s), d=%d, V=%d "
+                                   "bf16 head (1.09 GB), seeded" % (
+                                       n, "the full-response layout" if args.lm_rows <= 0
+                                       else "the first rows of the full-response batch, one "
+                                            "request", d, V),
                        "l2": "inputs (1.15 GB) larger than L2 (129 MB), no flush"},
             "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak,
                          "unit": "TFLOP/s", "frac": achieved / peak,
@@ -1275,6 +1282,8 @@ def main():
     ap.add_argument("--sel-oracle-child", type=int, default=0, help=argparse.SUPPRESS)
     ap.add_argument("--qnt-oracle-child", action="store_true", help=argparse.SUPPRESS)
     ap.add_argument("--lm-oracle-child", type=int, default=0, help=argparse.SUPPRESS)
+    ap.add_argument("--lm-rows", type=int, default=0,
+                    help="lmhead workload: the first N hidden states only, as one request")
     args = ap.parse_args()
     if args.lm_oracle_child:
         return lm_oracle_child(args.lm_oracle_child)

@@ -539,22 +539,59 @@ __global__ void lm_wait_probe(uint32_t* err, uint64_t limit_ns, int32_t* complet
   *completed = lm_wait(&bar, 0u, &abort_flag, err, limit_ns) ? 1 : 0;
 }
 
-// one warp per row: merge the parts (splits x column halves) in order, then
-// the verifier's row finalisation (features, top-2 indices, flags)
+// wpr warps per row (1, 2, 4 or 8; 8 / wpr rows per CTA): warp w of a row
+// merges the row's parts (splits x column halves) w, w + wpr, ... in order,
+// the row's first warp then merges the wpr results in warp order (with wpr =
+// 1 simply all parts in order), then the verifier's row finalisation
+// (features, top-2 indices, flags).  Many parts per row (a small batch split
+// over many vocabulary splits) take more warps per row.
 __global__ void __launch_bounds__(256) lm_merge(const Args a, const LmPart* __restrict__ parts,
-                                                int nparts) {
-  const int lane = threadIdx.x & 31;
-  const int64_t row = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
-  if (row >= a.n_rows) return;
+                                                int nparts, int wpr) {
+  __shared__ float s_m[8], s_S[8], s_U[8], s_xy[8];
+  __shared__ uint32_t s_fl[8];  // bit 0: a non-finite logit, bit 1: holds the chosen token
+  __shared__ uint64_t s_top[8][32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int g = warp / wpr, w = warp - g * wpr;
+  const int64_t row = (int64_t)blockIdx.x * (8 / wpr) + g;
+  const bool live = row < a.n_rows;
   float m = M2_INIT, S = 0.f, U = 0.f, xy = NAN;
-  bool bad = false;
+  bool bad = false, has_y = false;
   uint64_t E = 0ull;
-  for (int s = 0; s < nparts; ++s) {
-    const LmPart& p = parts[(int64_t)s * a.n_rows + row];
-    lse_merge(m, S, U, p.m, p.S, p.U);
-    bad |= p.bad != 0u;
-    if (p.has_y) xy = p.xy;
-    E = warp_merge_desc<uint64_t>(E, p.top[lane], lane);
+  if (live)
+    for (int s = w; s < nparts; s += wpr) {
+      const LmPart& p = parts[(int64_t)s * a.n_rows + row];
+      lse_merge(m, S, U, p.m, p.S, p.U);
+      bad |= p.bad != 0u;
+      if (p.has_y) {
+        xy = p.xy;
+        has_y = true;
+      }
+      E = warp_merge_desc<uint64_t>(E, p.top[lane], lane);
+    }
+  if (wpr > 1) {
+    if (lane == 0) {
+      s_m[warp] = m;
+      s_S[warp] = S;
+      s_U[warp] = U;
+      s_xy[warp] = xy;
+      s_fl[warp] = (bad ? 1u : 0u) | (has_y ? 2u : 0u);
+    }
+    s_top[warp][lane] = E;
+    __syncthreads();
+    if (w != 0 || !live) return;
+    m = M2_INIT;
+    S = U = 0.f;
+    xy = NAN;
+    bad = false;
+    E = 0ull;
+    for (int v = warp; v < warp + wpr; ++v) {
+      lse_merge(m, S, U, s_m[v], s_S[v], s_U[v]);
+      bad |= (s_fl[v] & 1u) != 0u;
+      if (s_fl[v] & 2u) xy = s_xy[v];
+      E = warp_merge_desc<uint64_t>(E, s_top[v][lane], lane);
+    }
+  } else if (!live) {
+    return;
   }
   RowPre pre;
   pre.y = a.chosen[row];

@@ -82,8 +82,9 @@ pr_status pr_lmhead_features(pr_ctx* c, const void* hidden, const void* weight, 
   const int kc = topk > 2 ? topk : 2;
   const void* kern = kc <= 20 ? reinterpret_cast<const void*>(&prk::lm_fused<20>)
                               : reinterpret_cast<const void*>(&prk::lm_fused<32>);
-  // Launch shape: nsplit vocabulary splits (around 12; among those the count
-  // with the least idle tail in the last wave of one CTA per SM), CTA pairs of
+  // Launch shape: nsplit vocabulary splits (around 12, or for a small batch as
+  // many as fill one wave of one CTA per SM; among those the count with the
+  // least idle tail in the last wave), CTA pairs of
   // 256 rows ordered in bands of `band` row pairs, whose H rows (256 d bf16
   // each) fill about a quarter of L2: a wave then holds one band's H plus the
   // W tiles of a few splits, each read from DRAM about once per wave.
@@ -91,11 +92,13 @@ pr_status pr_lmhead_features(pr_ctx* c, const void* hidden, const void* weight, 
   int64_t nsplit = 1;
   {
     double best = 1e30;
-    for (int64_t ns = 8; ns <= 24 && ns <= ntiles; ++ns) {
+    const int64_t fill = std::max<int64_t>(1, c->num_sms / mt_pad);  // splits filling a wave
+    const double target = std::max<double>(12.0, (double)fill);
+    for (int64_t ns = 8; ns <= std::max<int64_t>(24, fill) && ns <= ntiles; ++ns) {
       const int64_t ctas = mt_pad * ns;
       const int64_t waves = (ctas + c->num_sms - 1) / c->num_sms;
       const double waste = (double)(waves * c->num_sms - ctas) / (double)(waves * c->num_sms);
-      const double score = waste + 0.002 * std::abs((double)ns - 12.0);
+      const double score = waste + 0.002 * std::abs((double)ns - target);
       if (score < best) {
         best = score;
         nsplit = ns;
@@ -172,7 +175,10 @@ pr_status pr_lmhead_features(pr_ctx* c, const void* hidden, const void* weight, 
   a.top2 = top2;
   a.row_flags = row_flags;
   a.ctx_flags = c->flags;
-  prk::lm_merge<<<(unsigned)((n_rows + 7) / 8), 256, 0, s>>>(a, la.parts, (int)nparts);
+  const int wpr = nparts >= 64 ? 8 : nparts >= 32 ? 4 : 1;  // warps per row of the merge
+  const int64_t rows_per_cta = 8 / wpr;
+  prk::lm_merge<<<(unsigned)((n_rows + rows_per_cta - 1) / rows_per_cta), 256, 0, s>>>(
+      a, la.parts, (int)nparts, wpr);
   PR_CUDA(cudaGetLastError());
   g_launches.fetch_add(2, std::memory_order_relaxed);
   return timing_mark(c, s);
