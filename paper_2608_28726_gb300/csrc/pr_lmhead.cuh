@@ -101,9 +101,6 @@ __device__ __forceinline__ void lm_mbar_expect(uint64_t* b, uint32_t bytes) {
                "r"(bytes)
                : "memory");
 }
-__device__ __forceinline__ void lm_mbar_arrive(uint64_t* b) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(lm_smem(b)) : "memory");
-}
 __device__ __forceinline__ bool lm_mbar_test(uint64_t* b, uint32_t parity) {
   uint32_t ok;
   asm volatile(
