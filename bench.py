@@ -869,6 +869,49 @@ def run_lmhead_workload(args):
     del logits
     sampler.stop()
 
+    # decode steps (with --lm-rows): the n rows as live slots, each step through
+    # pr_lmhead_decode_step, against cuBLAS logits + pr_decode_step
+    decode = None
+    if args.lm_rows > 0:
+        dctx = B.pr_ctx_create(local, max_rows=n, max_requests=n)
+        slot = torch.arange(n, dtype=torch.int32, device=dev)
+        eos0 = torch.zeros(n, dtype=torch.uint8, device=dev)
+        dw = torch.from_numpy(wl.w).to(dev)
+        dsc = torch.empty(n, device=dev)
+        dsh = torch.empty(n, dtype=torch.uint8, device=dev)
+        dfl = torch.empty(n, dtype=torch.int32, device=dev)
+        dlog = torch.empty(n, V, dtype=torch.bfloat16, device=dev)
+        KD = max(3, min(K, 200))
+
+        def dec_fused():
+            B.pr_lmhead_decode_step(dctx, hidden, weight, slot, chosen, eos0, dw, wl.b, wl.tau,
+                                    dsc, dsh, dfl, stream=stream)
+
+        def dec_unfused():
+            torch.matmul(hidden, weight.t(), out=dlog)
+            B.pr_decode_step(dctx, dlog, slot, chosen, eos0, dw, wl.b, wl.tau, dsc, dsh, dfl,
+                             stream=stream)
+
+        dres = {}
+        for name_, fn in (("fused", dec_fused), ("unfused", dec_unfused)):
+            B.pr_ctx_reset(dctx, stream=stream)
+            for _ in range(3):
+                fn()
+            torch.cuda.synchronize(dev)
+            d0, d1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            d0.record(stream)
+            for _ in range(KD):
+                fn()
+            d1.record(stream)
+            torch.cuda.synchronize(dev)
+            dres[name_] = d0.elapsed_time(d1) / KD
+        decode = {"slots": n, "steps": KD, "fused_ms_per_step": dres["fused"],
+                  "unfused_ms_per_step": dres["unfused"],
+                  "speedup_of_fused": dres["unfused"] / dres["fused"],
+                  "api": "pr_lmhead_decode_step vs cuBLAS logits + pr_decode_step"}
+        del dlog
+        B.pr_ctx_destroy(dctx)
+
     # e2e: the step's hidden states from pinned host memory, its records back
     hh = hidden.cpu().pin_memory()
     hfeat = torch.empty(n, 8).pin_memory()
@@ -931,6 +974,7 @@ def run_lmhead_workload(args):
                         "ms_per_step": gemm_ms + feat_ms,
                         "logit_bytes_written_and_read": n * V * 2,
                         "speedup_of_fused": (gemm_ms + feat_ms) / ms},
+            "decode_steps": decode,
             "cpu_baseline": {"value": n_sample / dd["seconds"], "unit": UNIT, "cores": 1,
                              "kind": "oracle",
                              "sample": "rows 0..%d: float64 product and features" % (n_sample - 1)},

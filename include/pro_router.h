@@ -337,6 +337,27 @@ pr_status pr_lmhead_features(pr_ctx* ctx, const void* hidden, const void* weight
                              uint32_t* row_flags, void* stream);
 
 /*
+ * pr_decode_step without logits in memory: row i's logits x = W h_i are
+ * computed from the hidden state of the token in slot[i] on the tensor cores
+ * (as pr_lmhead_features) and its Eq. 3 features are folded into that slot
+ * (as pr_decode_step: running count, compensated sums and minima in step
+ * order; at eos[i] the request's aggregates are scored and thresholded, the
+ * outputs at index slot[i] written and the slot cleared).
+ *   hidden   device bf16 [n_live][d], row-major, 16-byte aligned
+ *   weight   device bf16 [vocab][d], row-major, 16-byte aligned
+ *   d        a multiple of 8
+ *   slot, chosen, eos, w, b, tau, score_out, ship_out, slot_flags, agg_out:
+ *            as pr_decode_step (n_live <= the context's max_requests)
+ * Uses the context's PR_OPT_TOPK and PR_OPT_TOPK_RENORM.  Two launches on
+ * `stream`; the state buffer as pr_lmhead_features; PR_FLAG_TIMEOUT as there.
+ */
+pr_status pr_lmhead_decode_step(pr_ctx* ctx, const void* hidden, const void* weight,
+                                int32_t n_live, int64_t d, int64_t vocab, const int32_t* slot,
+                                const int32_t* chosen, const uint8_t* eos, const float* w,
+                                float b, float tau, float* score_out, uint8_t* ship_out,
+                                uint32_t* slot_flags, float* agg_out, void* stream);
+
+/*
  * Failure-detection self-test: runs the bounded device-side wait that
  * pr_lmhead_features' kernels use on an mbarrier that nothing completes, with
  * a limit of `limit_ns` nanoseconds (0 .. 2e9) instead of 2 s.  *completed (host)

@@ -32,7 +32,7 @@ EXPORTS = (
     "pr_state_export", "pr_state_import", "pr_status_string", "pr_last_cuda_error",
     "pr_launch_count", "pr_route_noalloc", "pr_head_param_count", "pr_head_score",
     "pr_ctx_kernel_times", "pr_selective_metrics", "pr_quantile_score", "pr_lmhead_features",
-    "pr_selftest_wait",
+    "pr_selftest_wait", "pr_lmhead_decode_step",
 )
 
 if not os.path.exists(LIB):
@@ -61,6 +61,8 @@ _SIGS = {
     "pr_ctx_kernel_times": [_P, _P, _I32, ctypes.POINTER(_I32)],
     "pr_lmhead_features": [_P, _P, _P, _I64, _I64, _I64, _P, _I32, _P, _I32, _P, _P, _P, _P],
     "pr_selftest_wait": [_P, _I64, ctypes.POINTER(_I32)],
+    "pr_lmhead_decode_step": [_P, _P, _P, _I32, _I64, _I64, _P, _P, _P, _P, _F32, _F32, _P, _P,
+                              _P, _P, _P],
     "pr_quantile_score": [_P, _P, _P, _I64, _P, _I32, _P, _F32, _P, _P, _P, _P, _P],
     "pr_selective_metrics": [_P, _P, _P, _I64, ctypes.c_double, _P, _P],
     "pr_head_score": [_P, _P, _P, _I64, _P, _I32, _P, _I32, _F32, _P, _P, _P, _P],
@@ -353,6 +355,23 @@ def pr_lmhead_features(ctx, hidden, weight, chosen, topk: int = 20, offsets=None
                                    int(topk), _ptr(offsets), n_req, _ptr(feat), _ptr(top2),
                                    _ptr(row_flags), _stream(stream)), "pr_lmhead_features")
     return feat, top2, row_flags
+
+
+def pr_lmhead_decode_step(ctx, hidden, weight, slot, chosen, eos, w, b: float, tau: float,
+                          score_out, ship_out, slot_flags, agg_out=None, stream=None):
+    """One decode step from the live slots' bf16 hidden states [n][d] and the
+    bf16 LM head [V][d]: the logits stay on chip, each row's features are
+    folded into its slot (outputs as pr_decode_step)."""
+    if hidden.dtype != torch.bfloat16 or weight.dtype != torch.bfloat16:
+        raise TypeError("hidden and weight must be bfloat16")
+    if not (hidden.is_contiguous() and weight.is_contiguous()) or hidden.size(1) != weight.size(1):
+        raise ValueError("hidden [n][d] and weight [V][d] must be contiguous with the same d")
+    n, d = hidden.shape
+    _check(_lib.pr_lmhead_decode_step(ctx, _ptr(hidden), _ptr(weight), n, d, weight.size(0),
+                                      _ptr(slot), _ptr(chosen), _ptr(eos), _ptr(w), float(b),
+                                      float(tau), _ptr(score_out), _ptr(ship_out),
+                                      _ptr(slot_flags), _ptr(agg_out), _stream(stream)),
+           "pr_lmhead_decode_step")
 
 
 def pr_selftest_wait(ctx, limit_ns: int) -> bool:

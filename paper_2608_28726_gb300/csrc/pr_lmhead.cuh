@@ -33,9 +33,9 @@
 //                       split, half) goes to a small buffer.
 //              A W block is read from L2 once per 256 rows, an H block once
 //              per 256 vocabulary columns.
-//   lm_merge   one warp per row: merges the parts' states in split order
-//              and writes the feature record with the verifier's own row
-//              finalisation (row_finish).
+//   lm_merge   merges each row's partial states in a fixed order and runs
+//              the verifier's own row finalisation (row_finish): the feature
+//              record, or the fold into the row's decode slot.
 // Every mbarrier wait is bounded (2 s of %globaltimer); a wait that runs out
 // sets an error flag and stops that role's loop; the roles of the other CTA
 // then run out of their own waits, the rank-0 producer waits (bounded) for
@@ -539,9 +539,11 @@ __global__ void lm_wait_probe(uint32_t* err, uint64_t limit_ns, int32_t* complet
 // wpr warps per row (1, 2, 4 or 8; 8 / wpr rows per CTA): warp w of a row
 // merges the row's parts (splits x column halves) w, w + wpr, ... in order,
 // the row's first warp then merges the wpr results in warp order (with wpr =
-// 1 simply all parts in order), then the verifier's row finalisation
-// (features, top-2 indices, flags).  Many parts per row (a small batch split
-// over many vocabulary splits) take more warps per row.
+// 1 simply all parts in order), then the verifier's row finalisation: the
+// feature record (MODE_FEATURES) or the fold into the row's decode slot
+// (MODE_DECODE).  Many parts per row (a small batch split over many
+// vocabulary splits) take more warps per row.
+template <int MODE>
 __global__ void __launch_bounds__(256) lm_merge(const Args a, const LmPart* __restrict__ parts,
                                                 int nparts, int wpr) {
   __shared__ float s_m[8], s_S[8], s_U[8], s_xy[8];
@@ -596,14 +598,17 @@ __global__ void __launch_bounds__(256) lm_merge(const Args a, const LmPart* __re
   pre.r = -1;
   pre.lo = pre.hi = 0;
   pre.eos = 0;
-  if (a.offsets) {
+  if (MODE == MODE_DECODE) {
+    pre.r = a.slot[row];
+    pre.eos = a.eos[row];
+  } else if (a.offsets) {
     pre.r = find_request(a.offsets, a.n_req, row, lane);
     if (pre.r >= 0) {
       pre.lo = __ldg(a.offsets + pre.r);
       pre.hi = __ldg(a.offsets + pre.r + 1);
     }
   }
-  row_finish<float, MODE_FEATURES>(a, row, m, S, U, bad, lane < a.kc ? E : 0ull, pre, lane);
+  row_finish<float, MODE>(a, row, m, S, U, bad, lane < a.kc ? E : 0ull, pre, lane);
 }
 
 }  // namespace prk

@@ -53,22 +53,12 @@ bool make_map(CUtensorMap* map, const void* base, int64_t rows, int64_t d, uint3
 
 }  // namespace
 
-extern "C" {
-
-pr_status pr_lmhead_features(pr_ctx* c, const void* hidden, const void* weight, int64_t n_rows,
-                             int64_t d, int64_t vocab, const int32_t* chosen, int32_t topk,
-                             const int64_t* offsets, int32_t n_req, float* feat, int32_t* top2,
-                             uint32_t* row_flags, void* stream) {
-  if (!c || n_rows < 0 || n_rows > 0x7fffffffLL || vocab <= 0 || vocab > 0x7fffffffLL)
-    return PR_ERR_INVALID_ARG;
-  if (d <= 0 || d % 8 != 0 || d > (int64_t)1 << 20) return PR_ERR_INVALID_ARG;
-  if (topk < 1 || topk > PR_MAX_TOPK || n_req < 0 || (offsets && n_req < 1))
-    return PR_ERR_INVALID_ARG;
-  if (n_rows == 0) return PR_OK;
-  if (!hidden || !weight || !chosen || !feat || !top2 || !row_flags) return PR_ERR_INVALID_ARG;
-  if (!aligned16(hidden) || !aligned16(weight)) return PR_ERR_INVALID_ARG;
-  pr_status st = set_device(c);
-  if (st != PR_OK) return st;
+// The first launch of both LM-head entry points: lm_fused over the batch into
+// the context's state buffer.  On return *nparts is the number of partial
+// states per row (splits x column halves).
+static pr_status launch_lm_fused(pr_ctx* c, const void* hidden, const void* weight, int64_t n_rows,
+                                 int64_t d, int64_t vocab, const int32_t* chosen, int kc,
+                                 cudaStream_t s, int64_t* nparts_out) {
   if (!c->lm_ready) {
     PR_CUDA(cudaFuncSetAttribute(prk::lm_fused<20>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)prk::LM_SMEM));
@@ -79,7 +69,6 @@ pr_status pr_lmhead_features(pr_ctx* c, const void* hidden, const void* weight, 
   const int64_t mtiles = (n_rows + prk::LM_BM - 1) / prk::LM_BM;
   const int64_t ntiles = (vocab + prk::LM_BN - 1) / prk::LM_BN;
   if (mtiles > 0x7fffffffLL) return PR_ERR_INVALID_ARG;
-  const int kc = topk > 2 ? topk : 2;
   const void* kern = kc <= 20 ? reinterpret_cast<const void*>(&prk::lm_fused<20>)
                               : reinterpret_cast<const void*>(&prk::lm_fused<32>);
   // Launch shape: nsplit vocabulary splits (around 12, or for a small batch as
@@ -125,8 +114,6 @@ pr_status pr_lmhead_features(pr_ctx* c, const void* hidden, const void* weight, 
     }
     c->lm_parts_bytes = part_bytes;
   }
-  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  if ((st = timing_begin(c, s)) != PR_OK) return st;
   prk::LmArgs la;
   memset(&la, 0, sizeof la);
   la.n_rows = n_rows;
@@ -160,6 +147,45 @@ pr_status pr_lmhead_features(pr_ctx* c, const void* hidden, const void* weight, 
   cfg.numAttrs = 1;
   void* kargs[] = {&ma, &mb, &la};
   PR_CUDA(cudaLaunchKernelExC(&cfg, kern, kargs));
+  *nparts_out = nparts;
+  return PR_OK;
+}
+
+// The merge launch: wpr warps per row, more for rows with many parts.
+static void launch_lm_merge(const prk::Args& a, pr_ctx* c, int64_t nparts, int mode,
+                            cudaStream_t s) {
+  const int wpr = nparts >= 64 ? 8 : nparts >= 32 ? 4 : 1;
+  const int64_t rows_per_cta = 8 / wpr;
+  const unsigned grid = (unsigned)((a.n_rows + rows_per_cta - 1) / rows_per_cta);
+  const prk::LmPart* parts = static_cast<const prk::LmPart*>(c->lm_parts);
+  if (mode == prk::MODE_DECODE)
+    prk::lm_merge<prk::MODE_DECODE><<<grid, 256, 0, s>>>(a, parts, (int)nparts, wpr);
+  else
+    prk::lm_merge<prk::MODE_FEATURES><<<grid, 256, 0, s>>>(a, parts, (int)nparts, wpr);
+}
+
+extern "C" {
+
+pr_status pr_lmhead_features(pr_ctx* c, const void* hidden, const void* weight, int64_t n_rows,
+                             int64_t d, int64_t vocab, const int32_t* chosen, int32_t topk,
+                             const int64_t* offsets, int32_t n_req, float* feat, int32_t* top2,
+                             uint32_t* row_flags, void* stream) {
+  if (!c || n_rows < 0 || n_rows > 0x7fffffffLL || vocab <= 0 || vocab > 0x7fffffffLL)
+    return PR_ERR_INVALID_ARG;
+  if (d <= 0 || d % 8 != 0 || d > (int64_t)1 << 20) return PR_ERR_INVALID_ARG;
+  if (topk < 1 || topk > PR_MAX_TOPK || n_req < 0 || (offsets && n_req < 1))
+    return PR_ERR_INVALID_ARG;
+  if (n_rows == 0) return PR_OK;
+  if (!hidden || !weight || !chosen || !feat || !top2 || !row_flags) return PR_ERR_INVALID_ARG;
+  if (!aligned16(hidden) || !aligned16(weight)) return PR_ERR_INVALID_ARG;
+  pr_status st = set_device(c);
+  if (st != PR_OK) return st;
+  const int kc = topk > 2 ? topk : 2;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if ((st = timing_begin(c, s)) != PR_OK) return st;
+  int64_t nparts = 0;
+  if ((st = launch_lm_fused(c, hidden, weight, n_rows, d, vocab, chosen, kc, s, &nparts)) != PR_OK)
+    return st;
   if ((st = timing_mark(c, s)) != PR_OK) return st;
   prk::Args a;
   memset(&a, 0, sizeof a);
@@ -175,10 +201,55 @@ pr_status pr_lmhead_features(pr_ctx* c, const void* hidden, const void* weight, 
   a.top2 = top2;
   a.row_flags = row_flags;
   a.ctx_flags = c->flags;
-  const int wpr = nparts >= 64 ? 8 : nparts >= 32 ? 4 : 1;  // warps per row of the merge
-  const int64_t rows_per_cta = 8 / wpr;
-  prk::lm_merge<<<(unsigned)((n_rows + rows_per_cta - 1) / rows_per_cta), 256, 0, s>>>(
-      a, la.parts, (int)nparts, wpr);
+  launch_lm_merge(a, c, nparts, prk::MODE_FEATURES, s);
+  PR_CUDA(cudaGetLastError());
+  g_launches.fetch_add(2, std::memory_order_relaxed);
+  return timing_mark(c, s);
+}
+
+pr_status pr_lmhead_decode_step(pr_ctx* c, const void* hidden, const void* weight, int32_t n_live,
+                                int64_t d, int64_t vocab, const int32_t* slot,
+                                const int32_t* chosen, const uint8_t* eos, const float* w, float b,
+                                float tau, float* score_out, uint8_t* ship_out,
+                                uint32_t* slot_flags, float* agg_out, void* stream) {
+  if (!c || n_live < 0 || vocab <= 0 || vocab > 0x7fffffffLL) return PR_ERR_INVALID_ARG;
+  if (d <= 0 || d % 8 != 0 || d > (int64_t)1 << 20) return PR_ERR_INVALID_ARG;
+  if (n_live > c->max_requests) return PR_ERR_INVALID_ARG;
+  if (n_live == 0) return PR_OK;
+  if (!hidden || !weight || !slot || !chosen || !eos || !w || !score_out || !ship_out ||
+      !slot_flags)
+    return PR_ERR_INVALID_ARG;
+  if (!aligned16(hidden) || !aligned16(weight)) return PR_ERR_INVALID_ARG;
+  pr_status st = set_device(c);
+  if (st != PR_OK) return st;
+  const int kc = c->topk > 2 ? c->topk : 2;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if ((st = timing_begin(c, s)) != PR_OK) return st;
+  int64_t nparts = 0;
+  if ((st = launch_lm_fused(c, hidden, weight, n_live, d, vocab, chosen, kc, s, &nparts)) != PR_OK)
+    return st;
+  if ((st = timing_mark(c, s)) != PR_OK) return st;
+  prk::Args a;
+  memset(&a, 0, sizeof a);
+  a.n_rows = n_live;
+  a.vocab = vocab;
+  a.chosen = chosen;
+  a.topk = c->topk;
+  a.kc = kc;
+  a.renorm = c->renorm;
+  a.slot = slot;
+  a.eos = eos;
+  a.acc = c->acc;
+  a.n_slots = c->max_requests;
+  a.w = w;
+  a.b = b;
+  a.zthr = zthreshold(tau);
+  a.score = score_out;
+  a.ship = ship_out;
+  a.req_flags = slot_flags;
+  a.agg = agg_out;
+  a.ctx_flags = c->flags;
+  launch_lm_merge(a, c, nparts, prk::MODE_DECODE, s);
   PR_CUDA(cudaGetLastError());
   g_launches.fetch_add(2, std::memory_order_relaxed);
   return timing_mark(c, s);

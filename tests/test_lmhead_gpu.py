@@ -171,3 +171,64 @@ def test_lmhead_exact_ties_across_splits(B, ctx):
         assert list(tg[r]) == [17, 7368], tg[r]
         assert list(o["idx"][r]) == [17, 7368]
         assert feat[r, 2].item() == 0.0  # margin p1 - p2
+
+
+def test_lmhead_decode_steps_match_oracle(B):
+    """pr_lmhead_decode_step over a 40-step trace of 6 slots (requests of 1..14
+    tokens, a new request when one ends): every finished request's
+    aggregates, score, ship decision and flags against the float64 oracle of
+    the request's rows (exact products of its hidden states and the head)."""
+    import oracle
+    n_slots, steps, d, V = 6, 40, 128, 3000
+    g = np.random.default_rng(21)
+    eos = np.zeros((steps, n_slots), np.uint8)
+    reqs = []
+    for s in range(n_slots):
+        t = 0
+        while t < steps:
+            L = int(g.integers(1, 15))
+            reqs.append((s, t, L))
+            if t + L - 1 < steps:
+                eos[t + L - 1, s] = 1
+            t += L
+    _, w_lm, _ = make(1, d, V, seed=301)
+    hs = [make(n_slots, d, 8, seed=400 + t)[0] for t in range(steps)]
+    ch = [torch.from_numpy(g.integers(0, V, n_slots).astype(np.int32)) for _ in range(steps)]
+    w = (g.standard_normal(11) * 0.1).astype(np.float32)
+    b = float(np.float32(g.standard_normal() * 0.1))
+    ctx = B.pr_ctx_create(0, max_rows=16, max_requests=n_slots)
+    try:
+        slot = torch.arange(n_slots, dtype=torch.int32, device="cuda")
+        dw, wd = torch.from_numpy(w).cuda(), w_lm.cuda()
+        score = torch.full((n_slots,), -1.0, device="cuda")
+        ship = torch.zeros(n_slots, dtype=torch.uint8, device="cuda")
+        fl = torch.zeros(n_slots, dtype=torch.int32, device="cuda")
+        agg = torch.zeros(n_slots, 11, device="cuda")
+        B.pr_ctx_reset(ctx)
+        ends = {}
+        for t in range(steps):
+            B.pr_lmhead_decode_step(ctx, hs[t].cuda(), wd, slot, ch[t].cuda(),
+                                    torch.from_numpy(eos[t]).cuda(), dw, b, 0.5, score, ship, fl,
+                                    agg_out=agg)
+            for s in np.nonzero(eos[t])[0]:
+                ends[(int(s), t)] = (score[s].item(), ship[s].item(), fl[s].item(),
+                                     agg[s].cpu().numpy().copy())
+        assert (B.pr_ctx_flags(ctx) & B.PR_FLAG_TIMEOUT) == 0
+    finally:
+        B.pr_ctx_destroy(ctx)
+    wb = bits(w_lm)
+    checked = 0
+    for (s, t0, L) in reqs:
+        if t0 + L > steps:
+            continue
+        hb = np.stack([bits(hs[t][s:s + 1])[0] for t in range(t0, t0 + L)])
+        X = lmhead.logits(hb, wb).astype(np.float32)  # rounded at the hand-over, as lmhead.features
+        C = np.array([int(ch[t][s]) for t in range(t0, t0 + L)], np.int32)
+        o = oracle.route(X, C, np.array([0, L]), w.astype(np.float64), b, 0.5)
+        sc, sh, f, ag = ends[(s, t0 + L - 1)]
+        assert f == o["req_flags"][0]
+        assert_close(ag, o["agg"][0], "decode agg", rtol=TOL, atol=TOL)
+        assert_close(sc, o["score"][0], "decode score", rtol=TOL, atol=TOL)
+        assert sh == o["ship"][0] or abs(o["score"][0] - 0.5) < 1e-4
+        checked += 1
+    assert checked >= 15
