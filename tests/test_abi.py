@@ -68,6 +68,19 @@ def test_null_context_is_rejected(lib):
     assert lib.pr_ctx_create(ctypes.byref(h), 0, -5, 1) == -1
     lib.pr_ctx_set_option.argtypes = [P, ctypes.c_int32, ctypes.c_int32]
     assert lib.pr_ctx_set_option(None, 0, 20) == -1
+    # the LM-head calls and the wait self-test check their arguments on the host
+    lib.pr_lmhead_features.argtypes = [P, P, P, ctypes.c_int64, ctypes.c_int64, ctypes.c_int64, P,
+                                       ctypes.c_int32, P, ctypes.c_int32, P, P, P, P]
+    assert lib.pr_lmhead_features(None, None, None, 8, 64, 256, None, 20, None, 0, None, None,
+                                  None, None) == -1
+    lib.pr_lmhead_decode_step.argtypes = [P, P, P, ctypes.c_int32, ctypes.c_int64, ctypes.c_int64,
+                                          P, P, P, P, ctypes.c_float, ctypes.c_float, P, P, P, P,
+                                          P]
+    assert lib.pr_lmhead_decode_step(None, None, None, 4, 64, 256, None, None, None, None, 0.0, 0.5,
+                                     None, None, None, None, None) == -1
+    lib.pr_selftest_wait.argtypes = [P, ctypes.c_int64, ctypes.POINTER(ctypes.c_int32)]
+    done = ctypes.c_int32(7)
+    assert lib.pr_selftest_wait(None, 1000, ctypes.byref(done)) == -1 and done.value == 7
     assert lib.pr_launch_count() == n0  # nothing was launched
 
 

@@ -232,3 +232,34 @@ def test_lmhead_decode_steps_match_oracle(B):
         assert sh == o["ship"][0] or abs(o["score"][0] - 0.5) < 1e-4
         checked += 1
     assert checked >= 15
+
+
+def test_lmhead_decode_step_arguments_and_bad_slot(B):
+    """Host checks (hidden size not a multiple of 8, more live rows than
+    slots) and a slot id outside the context flagged on the device."""
+    ctx = B.pr_ctx_create(0, max_rows=16, max_requests=4)
+    try:
+        w11 = torch.zeros(11, device="cuda")
+        out = (torch.zeros(4, device="cuda"), torch.zeros(4, dtype=torch.uint8, device="cuda"),
+               torch.zeros(4, dtype=torch.int32, device="cuda"))
+        h, w, chosen = make(2, 64, 300, seed=5)
+        slot = torch.tensor([0, 9], dtype=torch.int32, device="cuda")
+        eos = torch.ones(2, dtype=torch.uint8, device="cuda")
+        B.pr_ctx_flags(ctx, clear=True)
+        B.pr_lmhead_decode_step(ctx, h.cuda(), w.cuda(), slot, chosen.cuda(), eos, w11, 0.0, 0.5,
+                                *out)
+        torch.cuda.synchronize()
+        assert B.pr_ctx_flags(ctx, clear=True) & B.PR_FLAG_BAD_SLOT
+        h20 = torch.zeros(2, 20, dtype=torch.bfloat16, device="cuda")
+        w20 = torch.zeros(300, 20, dtype=torch.bfloat16, device="cuda")
+        with pytest.raises(B.PRError) as e:
+            B.pr_lmhead_decode_step(ctx, h20, w20, slot, chosen.cuda(), eos, w11, 0.0, 0.5, *out)
+        assert e.value.status == B.PR_ERR_INVALID_ARG
+        h6, _, c6 = make(6, 64, 300, seed=6)
+        with pytest.raises(B.PRError):
+            B.pr_lmhead_decode_step(ctx, h6.cuda(), w.cuda(),
+                                    torch.arange(6, dtype=torch.int32, device="cuda"), c6.cuda(),
+                                    torch.zeros(6, dtype=torch.uint8, device="cuda"), w11, 0.0,
+                                    0.5, *out)
+    finally:
+        B.pr_ctx_destroy(ctx)
