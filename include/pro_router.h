@@ -326,7 +326,7 @@ pr_status pr_head_score(pr_ctx* ctx, const float* feat, const uint32_t* row_flag
  * The record has pr_token_features' slots and conventions, computed from the
  * fp32 logits; uses the context's PR_OPT_TOPK_RENORM.  Two launches on
  * `stream` (the first in thread-block clusters of two CTAs sharing each
- * tcgen05 MMA); the context holds a state buffer of 576 bytes per row and
+ * tcgen05 MMA); the context holds a state buffer of 288 bytes per row and
  * vocabulary split (grown on demand; that call synchronises the device).  A
  * device-side wait that runs out (2 s) raises PR_FLAG_TIMEOUT in the context
  * flag word.

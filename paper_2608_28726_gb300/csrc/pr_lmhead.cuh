@@ -29,8 +29,10 @@
 //                       thread, folded into the row's online (max, sum of 2^t,
 //                       sum of t 2^t) state, an exact running top-KC list and
 //                       the chosen token's logit; each warp reports a read
-//                       accumulator to the rank-0 CTA; the state of each (row,
-//                       split, half) goes to a small buffer.
+//                       accumulator to the rank-0 CTA; at the end the two
+//                       halves' states of a row are merged (through the idle
+//                       stage ring) into one state per (row, split) in a small
+//                       buffer.
 //              A W block is read from L2 once per 256 rows, an H block once
 //              per 256 vocabulary columns.
 //   lm_merge   merges each row's partial states in a fixed order and runs
@@ -73,7 +75,7 @@ constexpr uint32_t LM_ERR_TIMEOUT = 32u;                 // PR_FLAG_TIMEOUT in t
 constexpr uint32_t LM_IDESC = (1u << 4) | (1u << 7) | (1u << 10) |
                               ((uint32_t)(LM_BN >> 3) << 17) | ((uint32_t)((2 * LM_BM) >> 4) << 24);
 
-struct LmPart {            // one row's state over one column half of one vocabulary split
+struct LmPart {            // one row's state over one vocabulary split
   float m, S, U, xy;       // base-2 (m, S, U); the chosen token's logit if in range
   uint32_t bad, has_y, pad0, pad1;
   uint64_t top[32];        // descending keys (value, lower index first); 0 = empty
@@ -86,7 +88,7 @@ struct LmArgs {
   int32_t nsplit, npairs;   // vocabulary splits; 256-row pairs (CTA pairs per split)
   int32_t band;             // row pairs per band of the launch order
   const int32_t* chosen;
-  LmPart* parts;           // [nsplit][LM_HALVES][n_rows]
+  LmPart* parts;           // [nsplit][n_rows]
   uint32_t* err;           // error word
 };
 
@@ -340,6 +342,31 @@ struct LmRow {
   }
 };
 
+// out = the merge of the two column halves' states of one row: the online
+// sums merged, the top-32 keys of the union (both lists descending, 0 =
+// empty), the chosen token's logit from the half that holds it
+__device__ __forceinline__ void lm_merge_halves(const LmPart& x, const LmPart& y, LmPart* out) {
+  float m = x.m, S = x.S, U = x.U;
+  lse_merge(m, S, U, y.m, y.S, y.U);
+  out->m = m;
+  out->S = S;
+  out->U = U;
+  out->xy = x.has_y ? x.xy : y.xy;
+  out->bad = x.bad | y.bad;
+  out->has_y = x.has_y | y.has_y;
+  int i0 = 0, i1 = 0;
+  for (int j = 0; j < 32; ++j) {
+    const uint64_t k0 = i0 < 32 ? x.top[i0] : 0ull, k1 = i1 < 32 ? y.top[i1] : 0ull;
+    if (k0 >= k1) {
+      out->top[j] = k0;
+      ++i0;
+    } else {
+      out->top[j] = k1;
+      ++i1;
+    }
+  }
+}
+
 template <int KC>
 __global__ void __launch_bounds__(LM_NT, 1)
     lm_fused(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
@@ -512,9 +539,20 @@ __global__ void __launch_bounds__(LM_NT, 1)
       __syncwarp();
       if (lane == 0) lm_arrive_remote(tempty0 + 8u * (uint32_t)b);
     }
-    if (live) st.store(a.parts + ((int64_t)split * LM_HALVES + hc) * a.n_rows + row);
+    // both column halves of each row go to shared memory (the stage ring is
+    // idle once the last tile has been read); after the barrier below the
+    // half-0 thread of the row merges them into the row's part of this split
+    st.store(reinterpret_cast<LmPart*>(sm) + hc * LM_BM + 32 * q + lane);
   }
   __syncthreads();
+  if (warp >= 2) {
+    const int q = warp & 3, hc = (warp - 2) >> 2, lr = 32 * q + lane;
+    const int64_t row = (int64_t)mt * LM_BM + lr;
+    if (hc == 0 && row < a.n_rows) {
+      const LmPart* ex = reinterpret_cast<const LmPart*>(sm);
+      lm_merge_halves(ex[lr], ex[LM_BM + lr], a.parts + (int64_t)split * a.n_rows + row);
+    }
+  }
   lm_cluster_sync();  // the MMAs into both TMEMs are complete; no remote arrival is pending
   if (warp == 1) {
     lm_fence_after();

@@ -100,7 +100,7 @@ static pr_status launch_lm_fused(pr_ctx* c, const void* hidden, const void* weig
   if (!make_map(&ma, hidden, n_rows, d, (uint32_t)prk::LM_BM) ||
       !make_map(&mb, weight, vocab, d, (uint32_t)(prk::LM_BN / 2)))
     return PR_ERR_UNSUPPORTED;
-  const int64_t nparts = nsplit * prk::LM_HALVES;
+  const int64_t nparts = nsplit;  // one state per (row, split)
   const size_t part_bytes = (size_t)nparts * (size_t)n_rows * sizeof(prk::LmPart);
   if (part_bytes > c->lm_parts_bytes) {
     PR_CUDA(cudaDeviceSynchronize());  // the old buffer may still be in use
