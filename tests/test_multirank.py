@@ -34,10 +34,13 @@ def _worker(rank, world, port, out):
 def test_max_over_ranks_with_gloo():
     world = 2
     port = _free_port()
-    mgr = mp.Manager()
-    out = mgr.dict()
-    mp.spawn(_worker, args=(world, port, out), nprocs=world, join=True)
-    assert out[0] == out[1] == 15.0
+    mgr = mp.get_context("spawn").Manager()  # no fork of this multi-threaded process
+    try:
+        out = mgr.dict()
+        mp.spawn(_worker, args=(world, port, out), nprocs=world, join=True)
+        assert out[0] == out[1] == 15.0
+    finally:
+        mgr.shutdown()
 
 
 def test_single_rank_needs_no_process_group():
