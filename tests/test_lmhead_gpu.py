@@ -70,6 +70,8 @@ def check(B, ctx, n, d, V, seed, topk=20, offsets=None, chosen_override=None):
             assert list(tg[r]) == list(o["idx"][r]), r
         else:
             assert x[r, tg[r, 0]] >= srt[r, 0] - 1e-3
+    if V == 1:
+        assert (tg[:, 1] == -1).all()
     return fg, o
 
 
@@ -100,8 +102,28 @@ def test_lmhead_flags_and_rho(B, ctx):
 
 
 def test_lmhead_large_vocab_and_hidden(B, ctx):
-    """d = 3,584 (the small model's hidden size) and V = 151,936 on a few rows."""
+    """d = 3,584 (the small model's hidden size) and V = 151,936 on a few rows
+    (on 152 SMs: 76 splits of 8 vocabulary tiles, the last split empty)."""
     check(B, ctx, 8, 3584, 151936, seed=7)
+
+
+def test_lmhead_splits_without_tiles(B, ctx):
+    """16 rows x V = 32,000: a small batch takes as many splits as fill one
+    wave (76 on 152 SMs) of 2 of the 125 vocabulary tiles each, so the last 13
+    splits hold no tile.  Their states stay empty and must leave the merge
+    unchanged."""
+    check(B, ctx, 16, 128, 32000, seed=21)
+
+
+@pytest.mark.parametrize("n,d,V", [(3, 64, 1), (5, 64, 5), (7, 128, 17)])
+def test_lmhead_vocab_below_k(B, ctx, n, d, V):
+    """V < K = 20: the top-K sums run over the whole vocabulary, so the
+    top-K entropy equals the full entropy; the lists' unused entries stay
+    empty; V = 1 gives i2 = -1 and a margin p1 - p2 of 1."""
+    fg, _ = check(B, ctx, n, d, V, seed=V)
+    assert np.allclose(-fg[:, 4], fg[:, 3], rtol=TOL, atol=TOL)
+    if V == 1:
+        assert np.allclose(fg[:, 1:3], 1.0, atol=TOL)
 
 
 def test_lmhead_is_deterministic(B, ctx):
