@@ -17,6 +17,7 @@ import argparse
 import hashlib
 import json
 import os
+import re
 import statistics
 import subprocess
 import sys
@@ -77,19 +78,26 @@ def algorithmic_bytes(wl) -> int:
     return wl.n_rows * per_row + wl.n_req * per_req
 
 
-def kernel_sha() -> str:
+def source_sha(files) -> str:
+    """Hash of the code of the given csrc files with comments and white space
+    left out: it identifies the compiled kernels, so a profile's counters stay
+    valid across comment edits and go stale with any change to the code."""
     h = hashlib.sha256()
-    for f in KERNEL_FILES:
-        with open(os.path.join(ROOT, "paper_2608_28726_gb300", "csrc", f), "rb") as fh:
-            h.update(fh.read())
+    for f in files:
+        with open(os.path.join(ROOT, "paper_2608_28726_gb300", "csrc", f)) as fh:
+            text = fh.read()
+        text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
+        text = re.sub(r"//[^\n]*", " ", text)
+        h.update(" ".join(text.split()).encode())
+        h.update(b"\0")
     return h.hexdigest()[:16]
 
 
-def profiled_traffic():
-    """DRAM bytes per launch from the committed ncu summary, if it was taken on
-    the current kernel source (else None)."""
+def profiled_file_traffic(path, files, key="dram_bytes_per_launch"):
+    """DRAM bytes per launch from a committed ncu summary, if its
+    `kernel_source_sha` is that of the current code of `files` (else None)."""
     try:
-        text = open(PROFILE).read()
+        text = open(path).read()
     except OSError:
         return None
     vals = {}
@@ -97,12 +105,17 @@ def profiled_traffic():
         if ":" in line and line.strip().startswith("- "):
             k, v = line.strip()[2:].split(":", 1)
             vals[k.strip()] = v.strip().strip("`")
-    if vals.get("kernel_source_sha") != kernel_sha():
+    if vals.get("kernel_source_sha") != source_sha(files):
         return None
     try:
-        return int(vals["dram_bytes_per_full_launch"])
+        return int(vals[key])
     except (KeyError, ValueError):
         return None
+
+
+def profiled_traffic():
+    """The verifier kernel's DRAM bytes per launch on the full-response batch."""
+    return profiled_file_traffic(PROFILE, KERNEL_FILES, key="dram_bytes_per_full_launch")
 
 
 class ClockSampler:
@@ -1138,30 +1151,6 @@ def run_quantile_workload(args):
         }))
     B.pr_ctx_destroy(ctx)
     return 0
-
-
-def profiled_file_traffic(path, files):
-    """DRAM bytes per launch from a committed ncu summary, if taken on the
-    current source of `files` (else None)."""
-    try:
-        text = open(path).read()
-    except OSError:
-        return None
-    vals = {}
-    for line in text.splitlines():
-        if ":" in line and line.strip().startswith("- "):
-            k, v = line.strip()[2:].split(":", 1)
-            vals[k.strip()] = v.strip().strip("`")
-    h = hashlib.sha256()
-    for f in files:
-        with open(os.path.join(ROOT, "paper_2608_28726_gb300", "csrc", f), "rb") as fh:
-            h.update(fh.read())
-    if vals.get("kernel_source_sha") != h.hexdigest()[:16]:
-        return None
-    try:
-        return int(vals["dram_bytes_per_launch"])
-    except (KeyError, ValueError):
-        return None
 
 
 SEL_FILES = ("pr_device.cuh", "pr_select.cuh", "pr_select_api.cu")

@@ -55,7 +55,8 @@ bool make_map(CUtensorMap* map, const void* base, int64_t rows, int64_t d, uint3
 
 // The first launch of both LM-head entry points: lm_fused over the batch into
 // the context's state buffer.  On return *nparts is the number of partial
-// states per row (splits x column halves).
+// states per row (one per vocabulary split; the kernel has already merged each
+// row's two column halves).
 static pr_status launch_lm_fused(pr_ctx* c, const void* hidden, const void* weight, int64_t n_rows,
                                  int64_t d, int64_t vocab, const int32_t* chosen, int kc,
                                  cudaStream_t s, int64_t* nparts_out) {
