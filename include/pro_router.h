@@ -224,7 +224,10 @@ pr_status pr_route(pr_ctx* ctx, const void* logits, pr_dtype dt, int64_t row_bas
  * double-buffered staging area owned by the context, overlapped with the
  * fused kernel, and score / ship / req_flags (and agg if not NULL) are copied
  * back to the host buffers.  Synchronous: returns when the host outputs are
- * written.  The first call allocates the staging area (2 * chunk_rows rows).
+ * written.  chunk_rows >= 1; a chunk larger than the batch is taken as the
+ * batch.  The staging area (2 chunks of rows and token ids) is allocated on
+ * the first call and again whenever a larger chunk or another row size is
+ * asked for (that call synchronises the device).
  */
 pr_status pr_route_host(pr_ctx* ctx, const void* logits, pr_dtype dt, int64_t n_rows,
                         int64_t vocab, int64_t row_stride, const int32_t* chosen,

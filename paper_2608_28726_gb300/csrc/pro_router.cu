@@ -311,6 +311,9 @@ pr_status pr_route_host(pr_ctx* c, const void* logits, pr_dtype dt, int64_t n_ro
   if ((st = set_device(c)) != PR_OK) return st;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   const size_t row_bytes = (size_t)row_stride * esize(dt);
+  // a chunk never holds more than the batch: the staging buffers are sized
+  // from it (and chunk_rows * row_bytes then stays within the host buffer)
+  chunk_rows = std::min<int64_t>(chunk_rows, std::max<int64_t>(n_rows, 1));
 
   // staging: two chunks of rows, token ids, the offsets, weights and outputs
   if (c->stage_rows < chunk_rows || c->stage_row_bytes != row_bytes) {
@@ -499,7 +502,9 @@ pr_status pr_route_noalloc(const void* logits, pr_dtype dt, int64_t n_rows, int6
   a.agg = agg;
   a.ctx_flags = reinterpret_cast<uint32_t*>(d->scratch + NA_OFF_FLAGS);
 
-  // CTAs per row as in pr_route's automatic choice
+  // CTAs per row (the cluster kernel only; no persistent-kernel set-up here):
+  // double C, up to MAXC, while the batch's CTAs stay under two waves of
+  // resident CTAs
   const int64_t slots = (int64_t)d->num_sms * d->bps[dt == PR_DTYPE_BF16 ? 1 : 0];
   int C = 1;
   while (C < prk::MAXC && n_rows * C < 2 * slots) C <<= 1;

@@ -290,7 +290,10 @@ def test_route_is_one_launch(ctx):
     assert B.launch_count() - n0 == 1
 
 
-def test_route_host_matches_route(ctx):
+@pytest.mark.parametrize("chunk_rows", [37, 1 << 40])
+def test_route_host_matches_route(ctx, chunk_rows):
+    # 37: several chunks through both staging buffers; 2^40: one chunk, the
+    # staging area sized by the batch, not by the requested chunk
     lengths = [50, 3, 0, 200, 11]
     x, ch, off, w, b = _batch(lengths, 4096, torch.bfloat16, seed=41)
     _set(ctx, split=1)  # the automatic split depends on the rows per call
@@ -301,7 +304,8 @@ def test_route_host_matches_route(ctx):
     hoff = torch.from_numpy(off)
     hw = torch.from_numpy(w)
     agg = torch.empty(len(lengths), 11)
-    score, ship, rf, _ = B.pr_route_host(ctx, hx, hc, hoff, hw, b, 0.5, chunk_rows=37, agg=agg)
+    score, ship, rf, _ = B.pr_route_host(ctx, hx, hc, hoff, hw, b, 0.5, chunk_rows=chunk_rows,
+                                         agg=agg)
     assert torch.equal(score.nan_to_num(3.0), ref[0].cpu().nan_to_num(3.0))
     assert torch.equal(ship, ref[1].cpu()) and torch.equal(rf, ref[2].cpu())
     assert torch.equal(agg.nan_to_num(3.0), ref[3].cpu().nan_to_num(3.0))
