@@ -314,6 +314,8 @@ pr_status pr_head_score(pr_ctx* ctx, const float* feat, const uint32_t* row_flag
 
 /* ---- LM head fused with the row reduction --------------------------------------------- */
 
+#define PR_LMHEAD_MAX_VOCAB 2147483392LL /* 2^31 - 256: largest vocab of the LM-head calls */
+
 /*
  * pr_token_features without logits in memory: the rows' logits x = W h are
  * computed on the tensor cores (tcgen05, bf16 inputs, fp32 accumulation) and
@@ -324,7 +326,9 @@ pr_status pr_head_score(pr_ctx* ctx, const float* feat, const uint32_t* row_flag
  *            hidden states of the small model)
  *   weight   device bf16 [vocab][d], row-major, 16-byte aligned (the LM head;
  *            x_v = sum_k weight[v][k] hidden[row][k])
- *   d        hidden size, a multiple of 8
+ *   vocab    1 <= V <= PR_LMHEAD_MAX_VOCAB (the kernel's 32-bit column
+ *            arithmetic runs up to the end of V's last 256-column tile)
+ *   d        hidden size, a multiple of 8, at most 2^20
  *   chosen, topk, offsets, n_req, feat, top2, row_flags: as pr_token_features
  * The record has pr_token_features' slots and conventions, computed from the
  * fp32 logits; uses the context's PR_OPT_TOPK_RENORM.  Two launches on
@@ -348,7 +352,8 @@ pr_status pr_lmhead_features(pr_ctx* ctx, const void* hidden, const void* weight
  * outputs at index slot[i] written and the slot cleared).
  *   hidden   device bf16 [n_live][d], row-major, 16-byte aligned
  *   weight   device bf16 [vocab][d], row-major, 16-byte aligned
- *   d        a multiple of 8
+ *   vocab    as pr_lmhead_features
+ *   d        a multiple of 8, at most 2^20
  *   slot, chosen, eos, w, b, tau, score_out, ship_out, slot_flags, agg_out:
  *            as pr_decode_step (n_live <= the context's max_requests)
  * Uses the context's PR_OPT_TOPK and PR_OPT_TOPK_RENORM.  Two launches on

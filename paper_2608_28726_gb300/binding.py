@@ -24,6 +24,7 @@ PR_OPT_TOPK, PR_OPT_TOPK_RENORM, PR_OPT_SPLIT, PR_OPT_OVERLAP, PR_OPT_TIMING = 0
 PR_NOALLOC_MAX_ROWS, PR_NOALLOC_MAX_REQUESTS = 16384, 1024
 PR_HEAD_D, PR_HEAD_HEADS, PR_HEAD_FF, PR_HEAD_MAX_LAYERS = 64, 4, 128, 8
 PR_QMLP_SUMMARY, PR_QMLP_PARAMS = 28, 6081
+PR_LMHEAD_MAX_VOCAB = (1 << 31) - 256
 
 # every symbol include/pro_router.h declares
 EXPORTS = (

@@ -13,6 +13,9 @@
 using namespace prh;
 
 static_assert(prk::LM_ERR_TIMEOUT == PR_FLAG_TIMEOUT, "flag bit");
+// the last tile's columns (and a chunk's end, col0 + 32) stay below 2^31
+static_assert((PR_LMHEAD_MAX_VOCAB + prk::LM_BN - 1) / prk::LM_BN * prk::LM_BN <= 0x7fffffffLL,
+              "vocabulary limit");
 
 namespace {
 
@@ -171,7 +174,7 @@ pr_status pr_lmhead_features(pr_ctx* c, const void* hidden, const void* weight, 
                              int64_t d, int64_t vocab, const int32_t* chosen, int32_t topk,
                              const int64_t* offsets, int32_t n_req, float* feat, int32_t* top2,
                              uint32_t* row_flags, void* stream) {
-  if (!c || n_rows < 0 || n_rows > 0x7fffffffLL || vocab <= 0 || vocab > 0x7fffffffLL)
+  if (!c || n_rows < 0 || n_rows > 0x7fffffffLL || vocab <= 0 || vocab > PR_LMHEAD_MAX_VOCAB)
     return PR_ERR_INVALID_ARG;
   if (d <= 0 || d % 8 != 0 || d > (int64_t)1 << 20) return PR_ERR_INVALID_ARG;
   if (topk < 1 || topk > PR_MAX_TOPK || n_req < 0 || (offsets && n_req < 1))
@@ -213,7 +216,7 @@ pr_status pr_lmhead_decode_step(pr_ctx* c, const void* hidden, const void* weigh
                                 const int32_t* chosen, const uint8_t* eos, const float* w, float b,
                                 float tau, float* score_out, uint8_t* ship_out,
                                 uint32_t* slot_flags, float* agg_out, void* stream) {
-  if (!c || n_live < 0 || vocab <= 0 || vocab > 0x7fffffffLL) return PR_ERR_INVALID_ARG;
+  if (!c || n_live < 0 || vocab <= 0 || vocab > PR_LMHEAD_MAX_VOCAB) return PR_ERR_INVALID_ARG;
   if (d <= 0 || d % 8 != 0 || d > (int64_t)1 << 20) return PR_ERR_INVALID_ARG;
   if (n_live > c->max_requests) return PR_ERR_INVALID_ARG;
   if (n_live == 0) return PR_OK;

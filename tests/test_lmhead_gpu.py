@@ -285,3 +285,30 @@ def test_lmhead_decode_step_arguments_and_bad_slot(B):
                                     0.5, *out)
     finally:
         B.pr_ctx_destroy(ctx)
+
+
+@pytest.mark.parametrize("vocab", [(1 << 31) - 255, (1 << 31) - 1])
+def test_lmhead_rejects_vocab_above_its_limit(B, ctx, vocab):
+    """A vocabulary above PR_LMHEAD_MAX_VOCAB (2^31 - 256, where the last
+    tile's 32-bit column arithmetic would pass 2^31) is refused by both calls
+    before anything is queued; the pointers are valid but never read."""
+    h, w, chosen = make(2, 64, 300, seed=3)
+    h, w, chosen = h.cuda(), w.cuda(), chosen.cuda()
+    feat = torch.zeros(2, 8, device="cuda")
+    top2 = torch.zeros(2, 2, dtype=torch.int32, device="cuda")
+    rf = torch.zeros(2, dtype=torch.int32, device="cuda")
+    n0 = B.launch_count()
+    st = B._lib.pr_lmhead_features(ctx, h.data_ptr(), w.data_ptr(), 2, 64, vocab,
+                                   chosen.data_ptr(), 20, None, 0, feat.data_ptr(),
+                                   top2.data_ptr(), rf.data_ptr(), None)
+    assert st == B.PR_ERR_INVALID_ARG
+    slot = torch.arange(2, dtype=torch.int32, device="cuda")
+    eos = torch.zeros(2, dtype=torch.uint8, device="cuda")
+    w11 = torch.zeros(11, device="cuda")
+    st = B._lib.pr_lmhead_decode_step(ctx, h.data_ptr(), w.data_ptr(), 2, 64, vocab,
+                                      slot.data_ptr(), chosen.data_ptr(), eos.data_ptr(),
+                                      w11.data_ptr(), 0.0, 0.5, feat.data_ptr(), eos.data_ptr(),
+                                      rf.data_ptr(), None, None)
+    assert st == B.PR_ERR_INVALID_ARG
+    assert B.launch_count() == n0
+    assert B.PR_LMHEAD_MAX_VOCAB == (1 << 31) - 256
