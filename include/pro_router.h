@@ -147,6 +147,15 @@ pr_status pr_ctx_set_option(pr_ctx* ctx, int32_t option, int32_t value);
 pr_status pr_ctx_flags(pr_ctx* ctx, void* stream, int32_t clear, uint32_t* flags);
 
 /*
+ * The same word without a stream: waits for all work on the context's device
+ * (cudaDeviceSynchronize), then stores in *flags the OR of every flag bit the
+ * context's calls have raised since the last clear or reset, leaving the word
+ * as it is.  For callers that issue work on several streams and want one
+ * check at the end of a batch.
+ */
+pr_status pr_last_error(pr_ctx* ctx, uint32_t* flags);
+
+/*
  * Per-kernel device times (milliseconds, launch order) of the last call made
  * with PR_OPT_TIMING = 1: for pr_head_score the embedding, the first QKV
  * projection, then per layer the attention and the row-local block, then the

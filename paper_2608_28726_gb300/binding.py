@@ -33,7 +33,7 @@ EXPORTS = (
     "pr_state_export", "pr_state_import", "pr_status_string", "pr_last_cuda_error",
     "pr_launch_count", "pr_route_noalloc", "pr_head_param_count", "pr_head_score",
     "pr_ctx_kernel_times", "pr_selective_metrics", "pr_quantile_score", "pr_lmhead_features",
-    "pr_selftest_wait", "pr_lmhead_decode_step",
+    "pr_selftest_wait", "pr_lmhead_decode_step", "pr_last_error",
 )
 
 if not os.path.exists(LIB):
@@ -48,6 +48,7 @@ _SIGS = {
     "pr_ctx_reset": [_P, _P],
     "pr_ctx_set_option": [_P, _I32, _I32],
     "pr_ctx_flags": [_P, _P, _I32, ctypes.POINTER(ctypes.c_uint32)],
+    "pr_last_error": [_P, ctypes.POINTER(ctypes.c_uint32)],
     "pr_token_features": [_P, _P, ctypes.c_int, _I64, _I64, _I64, _P, _I32, _P, _I32, _P, _P, _P,
                           _P],
     "pr_aggregate_score": [_P, _P, _P, _I64, _P, _I32, _P, _F32, _F32, _P, _P, _P, _P, _P],
@@ -173,6 +174,13 @@ def pr_ctx_flags(ctx, stream=None, clear: bool = False) -> int:
     v = ctypes.c_uint32(0)
     _check(_lib.pr_ctx_flags(ctx, _stream(stream), int(bool(clear)), ctypes.byref(v)),
            "pr_ctx_flags")
+    return int(v.value)
+
+
+def pr_last_error(ctx) -> int:
+    """The context's flag word after all work on its device has finished."""
+    v = ctypes.c_uint32(0)
+    _check(_lib.pr_last_error(ctx, ctypes.byref(v)), "pr_last_error")
     return int(v.value)
 
 

@@ -210,6 +210,14 @@ pr_status pr_ctx_flags(pr_ctx* c, void* stream, int32_t clear, uint32_t* flags) 
   return PR_OK;
 }
 
+pr_status pr_last_error(pr_ctx* c, uint32_t* flags) {
+  if (!c || !flags) return PR_ERR_INVALID_ARG;
+  pr_status st = set_device(c);
+  if (st != PR_OK) return st;
+  PR_CUDA(cudaDeviceSynchronize());
+  return pr_ctx_flags(c, nullptr, 0, flags);
+}
+
 pr_status pr_ctx_kernel_times(pr_ctx* c, float* ms, int32_t cap, int32_t* n) {
   if (!c || !n || cap < 0 || (cap > 0 && !ms)) return PR_ERR_INVALID_ARG;
   pr_status st = set_device(c);

@@ -81,6 +81,12 @@ def test_null_context_is_rejected(lib):
     lib.pr_selftest_wait.argtypes = [P, ctypes.c_int64, ctypes.POINTER(ctypes.c_int32)]
     done = ctypes.c_int32(7)
     assert lib.pr_selftest_wait(None, 1000, ctypes.byref(done)) == -1 and done.value == 7
+    # the flag word, with and without a stream
+    lib.pr_last_error.argtypes = [P, ctypes.POINTER(ctypes.c_uint32)]
+    word = ctypes.c_uint32(9)
+    assert lib.pr_last_error(None, ctypes.byref(word)) == -1 and word.value == 9
+    lib.pr_ctx_flags.argtypes = [P, P, ctypes.c_int32, ctypes.POINTER(ctypes.c_uint32)]
+    assert lib.pr_ctx_flags(None, None, 0, ctypes.byref(word)) == -1 and word.value == 9
     assert lib.pr_launch_count() == n0  # nothing was launched
 
 
