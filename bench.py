@@ -37,6 +37,7 @@ METRIC = "verified tokens/sec at V=151,936 bf16 and achieved HBM GB/s vs peak (1
 UNIT = "tokens/s"
 KERNEL_FILES = ("pr_device.cuh", "pr_kernels.cuh", "pro_router.cu")
 PROFILE = os.path.join(ROOT, "profiles", "verify_rows_ws_bf16_full_response.md")
+HBM_NOMINAL_GBS = 8000.0  # GB300 HBM3e nominal bandwidth, reported beside the measured copy peak
 
 
 def dist_env():
@@ -382,7 +383,9 @@ def run_gb300(args):
                          "avg_launch_ms": avg_launch_ms,
                          "isolated_launch_ms": isolated_ms,
                          "isolated_achieved": isolated_achieved,
-                         "isolated_frac": isolated_achieved / peak},
+                         "isolated_frac": isolated_achieved / peak,
+                         "nominal_peak": HBM_NOMINAL_GBS,
+                         "frac_of_nominal": achieved / HBM_NOMINAL_GBS},
             "cpu_baseline": {"value": rows / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
                              "sample": "requests 0..%d (%d rows), float64 C oracle, %d threads" % (
                                  req_hi - 1, rows, cores)},
