@@ -1,7 +1,10 @@
 """Host logic of bench.py that needs no GPU: the source hash that gates each
 committed ncu traffic figure follows the code, not its comments, and the
-traffic figure is read only while that hash matches."""
+traffic figure is read only while that hash matches; the algorithmic bytes
+and flops the roofline lines divide by."""
 import os
+
+import numpy as np
 
 import bench
 
@@ -31,3 +34,43 @@ def test_profiled_traffic_follows_the_source(tmp_path, monkeypatch):
     _tree(tmp_path, "int g() { return 4; }\n")
     assert bench.profiled_file_traffic(str(prof), ["k.cu"]) is None
     assert bench.profiled_file_traffic(os.path.join(str(tmp_path), "missing.md"), ["k.cu"]) is None
+
+
+def test_algorithmic_bytes_of_the_workloads():
+    """The bytes behind `roofline.achieved`: per row the logits, the token id
+    and the 36-byte record written and read back once (76 bytes beside the
+    logits); per request two offsets, 11 aggregates, score, ship and flags (69
+    bytes).  The seeded workload shapes give the per-launch figures the
+    roofline is quoted on."""
+    expect = {"full": (8847, 64, 151936, 2, 2689032372),
+              "tiny": (354, 8, 32000, 4, 45339456),
+              "wide": (147828, 512, 262144, 4, 155020163184)}
+    for name, (rows, reqs, V, eb, total) in expect.items():
+        wl = bench.W.make(name)
+        assert (wl.n_rows, wl.n_req, wl.vocab, wl.elem_bytes) == (rows, reqs, V, eb), name
+        assert bench.algorithmic_bytes(wl) == total, name
+        assert total == rows * (V * eb + 76) + reqs * 69, name
+
+
+def test_head_flops_follow_the_oracle_weight_shapes():
+    """The scorer head's algorithmic flops: per layer and token one multiply
+    and one add for every entry of the four projection matrices (taken from
+    the oracle's weight layout), and per layer, request and head the T x T
+    scores and the weighted sum of values over the head width."""
+    from oracle import head as oh
+    n_layers, lengths = 2, [1, 7, 40]
+    p = oh.unpack(np.zeros(oh.n_params(n_layers)), n_layers)
+    per_token = sum(2 * p["layers"][0][k].size for k in ("W_qkv", "W_o", "W_1", "W_2"))
+    attn = sum(oh.HEADS * 2 * (2 * T * T * oh.DH) for T in lengths)
+    step, one_attn = bench.head_flops(lengths, n_layers)
+    assert one_attn == attn
+    assert step == n_layers * (per_token * sum(lengths) + attn)
+
+
+def test_quantile_bytes_count_the_weights_of_the_oracle_mlp():
+    """One quantile-scorer launch reads each 32-byte record, the offsets and
+    the MLP's weights once, and writes score, ship and flags per request."""
+    from oracle import quantile as oq
+    n_rows, n_req = 1000, 7
+    assert bench.qnt_bytes(n_rows, n_req) == (32 * n_rows + 8 * (n_req + 1) + 4 * oq.n_params()
+                                              + (4 + 1 + 4) * n_req)
