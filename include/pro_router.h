@@ -56,7 +56,7 @@ extern "C" {
 typedef enum {
   PR_OK = 0,
   PR_ERR_INVALID_ARG = -1, /* a null, negative, out-of-range or misaligned argument */
-  PR_ERR_UNSUPPORTED = -2, /* a device or mode this build cannot run */
+  PR_ERR_UNSUPPORTED = -2, /* a device or mode this library cannot run */
   PR_ERR_CUDA = -3,        /* a CUDA runtime call failed; see pr_last_cuda_error */
   PR_ERR_NO_MEMORY = -4    /* a context allocation failed */
 } pr_status;
