@@ -5,7 +5,7 @@
  * The verifier reads, for every generated token t, the small model's logit row
  * x_t over the vocabulary (V entries) and reduces it to the per-token features
  * of Eq. 3:
- *     l_t   = log p_t(y_t)            log-probability of the emitted token y_t
+ *     l_t   = log p_t(y_t)            the emitted token's log-probability
  *     m_t   = max_v p_t(v)            maximum probability
  *     h_t   = -H_t^K,  H_t^K = -sum_{v in top-K} p_t(v) log p_t(v),  K = 20
  *     rho_t = t / T                   position fraction (t is 1-based)
@@ -329,8 +329,8 @@ pr_status pr_head_score(pr_ctx* ctx, const float* feat, const uint32_t* row_flag
  * pr_token_features without logits in memory: the rows' logits x = W h are
  * computed on the tensor cores (tcgen05, bf16 inputs, fp32 accumulation) and
  * reduced to the Eq. 3 row record in the GEMM's epilogue, so the [n_rows][V]
- * logit matrix is never written (Section 3.1: the features are a side product
- * of the small model's own decoding).
+ * logit matrix is never written (Section 3.1: the features need nothing the
+ * small model's decoding does not already compute).
  *   hidden   device bf16 [n_rows][d], row-major, 16-byte aligned (the final
  *            hidden states of the small model)
  *   weight   device bf16 [vocab][d], row-major, 16-byte aligned (the LM head;
@@ -432,7 +432,8 @@ typedef struct {
  * Calibrate the operating point on a validation pool and score the ranking
  * (Section 3.1: tau is fixed in advance on a validation pool; Section 4.1:
  * the coverage rule of selective prediction fixes a ship fraction q, and
- * AUROC / the area under the shipping-accuracy curve measure the ranking).
+ * AUROC and AUARC, the area under accuracy-of-what-ships against ship rate,
+ * measure the ranking).
  *   scores  device float [n], e.g. the score output of pr_route or
  *           pr_head_score; non-finite entries (flagged requests) never ship
  *           and are left out of the metrics

@@ -1,6 +1,6 @@
 """Float64 oracle of the LM head fused with the verifier's row features
-(Pro-Router, Section 3.1: the per-token features are a side product of the
-small model's own decoding; its logits are x = W h).
+(Pro-Router, Section 3.1: the per-token features need nothing beyond what the
+small model's decoding already computes; its logits are x = W h).
 
 TEST INFRASTRUCTURE ONLY: used by the tests and the benchmark's CPU baseline;
 the product path never imports it.  The definition written out: the logits of

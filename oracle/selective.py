@@ -14,8 +14,8 @@ written from the definitions in the text:
   never ship, so k is capped at the number of finite scores.
 * AUROC (Section 4.1): the probability that a randomly chosen correct answer
   scores above a randomly chosen incorrect one, a tie counting one half.
-* AUARC (Section 4.1): the area under the shipping-accuracy curve, accuracy
-  among the shipped requests as a function of the ship rate.  Reading: ship in
+* AUARC (Section 4.1): the area under the curve of the accuracy of what ships
+  against the fraction shipped.  Reading: ship in
   order of decreasing score; after k of the n requests the accuracy is
   C_k / k, where C_k is the number of correct answers among the k shipped;
   AUARC = (1/n) sum_{k=1..n} C_k / k.  Inside a group of tied scores the order
@@ -110,8 +110,8 @@ def auroc(scores, labels) -> float:
 
 
 def auarc_loop(scores, labels) -> float:
-    """Area under the shipping-accuracy curve with tie groups averaged, one
-    shipped request at a time."""
+    """AUARC with tie groups averaged, computed one shipped request at a
+    time."""
     s = np.asarray(scores, np.float64)
     y = np.asarray(labels).astype(np.float64)
     keep = np.isfinite(s)

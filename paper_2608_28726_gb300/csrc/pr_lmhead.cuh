@@ -1,5 +1,5 @@
 // LM head fused with the verifier's row reduction (Pro-Router, Section 3.1:
-// the features are a side product of the small model's own decoding): the
+// the features need nothing the small model's decoding does not compute): the
 // logits x = W h of a batch of hidden states are produced on the tensor cores
 // and reduced to the Eq. 3 row state in the epilogue, so they never reach
 // device memory.

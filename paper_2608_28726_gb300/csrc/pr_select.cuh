@@ -1,7 +1,7 @@
 // Operating-point calibration and selective-prediction metrics on the GPU
 // (Pro-Router, Section 3.1: tau fixed on a validation pool; Section 4.1: the
-// coverage rule with ship fraction q, AUROC and the area under the
-// shipping-accuracy curve).
+// coverage rule with ship fraction q, AUROC and AUARC, the area under the
+// accuracy of what ships against the fraction shipped).
 //
 // Everything follows from one ascending sort of the scores: a stable LSD radix
 // sort of 32-bit order-preserving keys carrying the 0/1 label, 8 bits per pass
