@@ -11,7 +11,8 @@ Readings where the paper is silent (its figure with the head's sizes is not
 available): d = 64, 4 heads, feed-forward width 128, post-norm encoder layers
 (residual, then LayerNorm with eps 1e-5), ReLU, sinusoidal positional encoding
 of the 0-based position t, L = 2 layers (1 and 4 in the paper's ablation).
-These sizes give 67,329 parameters for L = 2, close to the paper's count.
+These sizes give 67,329 parameters for L = 2, matching the paper's figure of
+about 67 thousand (Section 4.2).
 
 Weights are one flat float array in this order (y = x W^T + b convention):
   W_in[64][4] b_in[64]
