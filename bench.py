@@ -6,7 +6,14 @@ V = 151,936 bf16, 2.69 GB) and achieved HBM bandwidth of the fused kernel.
 
 A step is one fused verification of the whole batch (pr_route: row features,
 pooling, score, ship rule; one kernel launch) with the logits resident in HBM.
-The batch is larger than L2, so no flush is needed between steps.  Under
+The batch is larger than L2, so no flush is needed between steps.  The K-step
+timed loop is repeated until at least 1.5 s of device time is timed, and the
+median repeat is reported, so the clock record has many samples.  On one GPU
+the line also carries a `configs` object: the tiny (c1), decode-step (c3),
+large ragged (c4) and wide-vocabulary (c5) workloads, each generated in full,
+resident in HBM, timed the same way and checked against the oracle on sampled
+whole requests; and a `noalloc` record (the allocation-free call beside
+pr_route).  A value is printed only when its parity sample passes.  Under
 torchrun every rank verifies its own batch (weak scaling, no collective on
 the data path); rank 0 prints one JSON line.  ``--impl reference`` times the
 float64 CPU oracle on the host cores instead (a bounded sample per step).
@@ -228,6 +235,406 @@ def run_reference(args):
     return 0
 
 
+# ---- timing, parity and the per-configuration records of the verifier ------------------
+
+MIN_TIMED_S = 1.5  # each timed measurement repeats its K-step loop until this much device time
+TOL_RTOL, TOL_ATOL, SHIP_BAND = 1e-4, 1e-5, 1e-6  # the verifier's parity bar
+
+
+def measured_peak():
+    peaks_file = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(peaks_file):
+        return float(json.load(open(peaks_file))["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+def timed_repeats(step, K: int, stream, dev, world: int, B, min_s: float = MIN_TIMED_S):
+    """Time K back-to-back steps with CUDA events on `stream`, a barrier and a
+    synchronize on both sides (max over ranks), and repeat that K-step loop
+    until at least `min_s` seconds of device time are timed (at least three
+    repeats).  Returns (per-repeat ms per step, wall window, launches in all
+    timed repeats)."""
+    per, total_ms = [], 0.0
+    launches = 0
+    t_wall0 = time.time()
+    while len(per) < 3 or total_ms < min_s * 1e3:
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        barrier(world)
+        torch.cuda.synchronize(dev)
+        n0 = B.launch_count()
+        e0.record(stream)
+        for _ in range(K):
+            step()
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        barrier(world)
+        launches += B.launch_count() - n0
+        ms = reduce_max(e0.elapsed_time(e1), world, dev)
+        per.append(ms / K)
+        total_ms += ms
+    return per, (t_wall0, time.time()), launches
+
+
+def parity_ok(g_agg, g_score, g_ship, g_flags, o, tau):
+    """The verifier's parity bar on whole requests: aggregates and scores within
+    1e-5 + 1e-4 |oracle|, flags equal, ship equal except where the oracle's
+    score is within 1e-6 of tau.  `o` holds the oracle's agg, score, ship and
+    req_flags for the same requests, in the same order."""
+    ga = np.asarray(g_agg, np.float64)
+    gs = np.asarray(g_score, np.float64)
+    oa, os_ = np.asarray(o["agg"], np.float64), np.asarray(o["score"], np.float64)
+
+    def close(g, ref):
+        nan = np.isnan(g) & np.isnan(ref)
+        with np.errstate(invalid="ignore"):
+            return bool(np.all(nan | (np.abs(g - ref) <= TOL_ATOL + TOL_RTOL * np.abs(ref))))
+
+    ship_ok = np.all((np.asarray(g_ship) == np.asarray(o["ship"])) |
+                     (np.abs(os_ - tau) < SHIP_BAND))
+    flags_ok = np.array_equal(np.asarray(g_flags).astype(np.uint32),
+                              np.asarray(o["req_flags"]).astype(np.uint32))
+    return bool(close(ga, oa) and close(gs, os_) and ship_ok and flags_ok)
+
+
+def gate_on_parity(rec: dict) -> dict:
+    """Verified tokens/s count only for runs whose sampled outputs pass oracle
+    parity: a record whose parity failed keeps its timings but no value."""
+    if not rec.get("parity", {}).get("ok", False):
+        rec["value_withheld"] = "parity with the oracle failed on the sampled requests"
+        rec["value"] = None
+    return rec
+
+
+def oracle_on_requests(wl, x_rows_of, reqs, threads: int):
+    """The float64 oracle on whole requests `reqs`; x_rows_of(lo, hi) returns
+    the device rows [lo, hi) and their token ids.  Returns the oracle's agg,
+    score, ship and req_flags stacked in request order, the seconds it took
+    and the rows it covered."""
+    import oracle
+    outs, secs, rows = [], 0.0, 0
+    for r in reqs:
+        lo, hi = int(wl.offsets[r]), int(wl.offsets[r + 1])
+        x, ch = x_rows_of(lo, hi)
+        xs, cs = W.to_oracle_array(x), ch.cpu().numpy()
+        t0 = time.perf_counter()
+        outs.append(oracle.route(xs, cs, np.array([0, hi - lo], np.int64),
+                                 wl.w.astype(np.float64), wl.b, wl.tau, n_threads=threads))
+        secs += time.perf_counter() - t0
+        rows += hi - lo
+    stack = {k: np.concatenate([o[k] for o in outs]) for k in ("agg", "score", "ship",
+                                                                 "req_flags")}
+    return stack, secs, rows
+
+
+def _route_rec(wl, name, desc, timing, ms, iso_ms, stream_ms, bytes_per_step, rows_per_step,
+               world, clocks, launches, K, repeats, parity, graph=None):
+    peak, peak_src = measured_peak()
+    ach = bytes_per_step / (ms / 1e3) / 1e9
+    rec = {
+        "workload": desc, "value": rows_per_step * world / (ms / 1e3), "unit": UNIT,
+        "ms_per_step": ms, "steps": K, "repeats": repeats, "rows_per_step_per_gpu": rows_per_step,
+        "dtype": "f32" if wl.dtype == "f32" else "bf16", "timing": timing,
+        "roofline": {"bound": "hbm", "achieved": ach, "peak": peak, "unit": "GB/s",
+                     "frac": ach / peak, "traffic": None, "peak_source": peak_src,
+                     "kernel": ("verify_rows_ws" if rows_per_step > 1024 else "verify_rows")
+                               + "<%s, %s>" % ("f32" if wl.dtype == "f32" else "bf16",
+                                               "decode" if name == "decode" else "route"),
+                     "algorithmic_bytes_per_step": bytes_per_step,
+                     "stream_ms_per_step": stream_ms,
+                     "stream_frac": bytes_per_step / (stream_ms / 1e3) / 1e9 / peak,
+                     "isolated_ms_per_step": iso_ms,
+                     "isolated_frac": bytes_per_step / (iso_ms / 1e3) / 1e9 / peak},
+        "clocks": clocks, "gpu_launches": launches, "parity": parity,
+        "work_per_row": "Eq. 3 features of the row (Section 3.1), pooled, scored and thresholded "
+                        "per request",
+    }
+    if graph:
+        rec["graph"] = graph
+    return gate_on_parity(rec)
+
+
+def measure_route_config(name, B, dev, stream, K, warm, world, sampler, threads, log=None):
+    """One of the full-response-style verifier workloads (tiny, ragged, wide),
+    resident in HBM; a step is one verification of the whole batch (chunked
+    as the workload says).  Returns its record."""
+    t_gen = time.time()
+    wl = W.make(name)
+    copies = 8 if name == "tiny" else 1  # 8 x 45 MB rotated: more than L2 between reuses
+    need = copies * wl.n_rows * wl.vocab * wl.elem_bytes
+    free, _ = torch.cuda.mem_get_info(dev)
+    if need * 1.15 > free:
+        raise RuntimeError("%s workload needs %.1f GB, %.1f GB free" % (name, need / 1e9, free / 1e9))
+    xs, chs = [], []
+    for c in range(copies):
+        x = torch.empty(wl.n_rows, wl.vocab, dtype=wl.torch_dtype, device=dev)
+        ch = torch.empty(wl.n_rows, dtype=torch.int32, device=dev)
+        W.rows(wl, 0, wl.n_rows, device=dev, out=x, chosen_out=ch)
+        xs.append(x)
+        chs.append(ch)
+    torch.cuda.synchronize(dev)
+    gen_s = time.time() - t_gen
+    off = torch.from_numpy(wl.offsets).to(dev)
+    w = torch.from_numpy(wl.w).to(dev)
+    ctx = B.pr_ctx_create(dev.index, max_rows=wl.n_rows, max_requests=wl.n_req)
+    outs = [(torch.empty(wl.n_req, device=dev), torch.empty(wl.n_req, dtype=torch.uint8, device=dev),
+             torch.empty(wl.n_req, dtype=torch.int32, device=dev),
+             torch.empty(wl.n_req, 11, device=dev)) for _ in range(copies)]
+    chunk = wl.chunk_rows or wl.n_rows
+    state = {"c": 0}
+
+    def route_call(c, st):
+        for lo in range(0, wl.n_rows, chunk):
+            hi = min(wl.n_rows, lo + chunk)
+            o = outs[c]
+            B.pr_route(ctx, xs[c][lo:hi], chs[c][lo:hi], off, w, wl.b, wl.tau, row_base=lo,
+                       score=o[0], ship=o[1], req_flags=o[2], agg=o[3], stream=st)
+
+    def step():
+        c = state["c"] % copies
+        state["c"] += 1
+        route_call(c, stream)
+
+    def timed(overlap):
+        B.pr_ctx_set_option(ctx, B.PR_OPT_OVERLAP, overlap)
+        for _ in range(warm):
+            step()
+        torch.cuda.synchronize(dev)
+        return timed_repeats(step, K, stream, dev, world, B)
+
+    iso, _, _ = timed(0)
+    per, win, launches = timed(1)
+    stream_ms = statistics.median(per)
+    ms, reps, timing, graph = stream_ms, len(per), "stream of back-to-back calls", None
+    if name == "tiny":
+        # launch-bound: one step per rotated copy captured in a CUDA graph, replayed
+        gr = torch.cuda.CUDAGraph()
+        n0 = B.launch_count()
+        with torch.cuda.graph(gr, capture_error_mode="thread_local"):
+            gs = torch.cuda.current_stream(dev)
+            for c in range(copies):
+                route_call(c, gs)
+        nodes = B.launch_count() - n0
+        for _ in range(3):
+            gr.replay()
+        torch.cuda.synchronize(dev)
+        reps_per = max(1, -(-1000 // copies))
+        per_g, win, launches = timed_repeats(gr.replay, reps_per, torch.cuda.current_stream(dev),
+                                             dev, world, B)
+        ms = statistics.median(per_g) / copies
+        launches = nodes * reps_per * len(per_g)
+        reps = len(per_g)
+        timing = "CUDA graph replays (%d steps per graph, %d replays per repeat)" % (copies,
+                                                                                     reps_per)
+        graph = {"steps_per_graph": copies, "kernels_per_graph": nodes,
+                 "replays_per_repeat": reps_per}
+        del gr
+    B.pr_ctx_set_option(ctx, B.PR_OPT_OVERLAP, 0)
+    clocks = sampler.summary(*win)
+    # parity: the last timed outputs of copy 0 on sampled whole requests
+    route_call(0, stream)
+    torch.cuda.synchronize(dev)
+    if name == "tiny":
+        reqs = list(range(wl.n_req))
+    elif name == "ragged":
+        bounds = np.arange(wl.chunk_rows, wl.n_rows, wl.chunk_rows)
+        off_np = wl.offsets
+        crossing = [r for r in range(wl.n_req)
+                    if np.any((off_np[r] < bounds) & (bounds < off_np[r + 1]))]
+        reqs = crossing + [0, 511, 1023]
+    else:
+        reqs = [0, 1, 2, 200, 305, 400, 510, 511]
+    o, secs, rows = oracle_on_requests(wl, lambda lo, hi: (xs[0][lo:hi], chs[0][lo:hi]), reqs,
+                                       threads)
+    g = [t.cpu().numpy()[reqs] for t in outs[0]]
+    ok = parity_ok(g[3], g[0], g[1], g[2], o, wl.tau)
+    parity = {"requests_checked": len(reqs), "rows_checked": rows, "ok": ok,
+              "oracle_tokens_per_s": rows / secs if secs > 0 else None}
+    desc = {"tiny": "tiny full-response verify: 8 requests, T~U{16..64} (%d rows), V=%d fp32 "
+                    "2*N(0,1) + one spike U(0,8) per row; 8 rotated resident copies",
+            "ragged": "large ragged batch: 1,024 requests, lengths lognormal(ln 128, 0.8) "
+                      "clipped to [8,1024] (%d rows), V=%d bf16, 8,192-row chunks per step",
+            "wide": "wide vocabulary: 512 requests, T~U{64..512} (%d rows), V=%d fp32 "
+                    "2*Student-t(3), exact top-1 ties on 10%% of rows, one launch"}[name] % (
+                        wl.n_rows, wl.vocab)
+    rec = _route_rec(wl, name, desc, timing, ms, statistics.median(iso), stream_ms,
+                     algorithmic_bytes(wl) if name != "tiny" else algorithmic_bytes(wl),
+                     wl.n_rows, world, clocks, launches, K, reps, parity, graph)
+    rec["generation_s"] = gen_s
+    rec["l2"] = ("8 rotated copies (360 MB) larger than L2" if name == "tiny" else
+                 "inputs (%.1f GB) larger than L2 (129 MB), no flush" % (need / 1e9))
+    B.pr_ctx_destroy(ctx)
+    del xs, chs, outs
+    torch.cuda.empty_cache()
+    return rec
+
+
+def measure_decode_config(B, dev, stream, K, warm, world, sampler, threads):
+    """The incremental decode-step workload: 256 live slots for 1,000 steps,
+    V = 151,936 bf16, the whole trace resident (77.8 GB); a step is one
+    pr_decode_step of 256 rows.  Timed as isolated calls, back-to-back calls
+    and (headline) CUDA-graph replays of a context reset plus the whole trace.
+    Parity: every sampled request that finishes inside the trace against the
+    oracle on its rows."""
+    t_gen = time.time()
+    tr = W.decode_trace()
+    wl = tr.as_workload()
+    S, T = tr.n_slots, tr.n_steps
+    x_all = torch.empty(T * S, wl.vocab, dtype=wl.torch_dtype, device=dev)
+    ch_all = torch.empty(T * S, dtype=torch.int32, device=dev)
+    W.rows(wl, 0, T * S, device=dev, out=x_all, chosen_out=ch_all)
+    torch.cuda.synchronize(dev)
+    gen_s = time.time() - t_gen
+    eos = torch.from_numpy(tr.eos).to(dev)
+    slot = torch.arange(S, dtype=torch.int32, device=dev)
+    w = torch.from_numpy(tr.w).to(dev)
+    ctx = B.pr_ctx_create(dev.index, max_rows=S, max_requests=S)
+    outs = (torch.empty(S, device=dev), torch.empty(S, dtype=torch.uint8, device=dev),
+            torch.empty(S, dtype=torch.int32, device=dev), torch.empty(S, 11, device=dev))
+    state = {"t": 0}
+
+    def decode_call(t, st):
+        B.pr_decode_step(ctx, x_all[t * S:(t + 1) * S], slot, ch_all[t * S:(t + 1) * S], eos[t], w,
+                         tr.b, tr.tau, *outs[:3], agg_out=outs[3], stream=st)
+
+    def step():
+        t = state["t"]
+        if t == T:
+            B.pr_ctx_reset(ctx, stream=stream)
+            t = 0
+        decode_call(t, stream)
+        state["t"] = t + 1
+
+    def timed(overlap):
+        B.pr_ctx_set_option(ctx, B.PR_OPT_OVERLAP, overlap)
+        for _ in range(warm):
+            step()
+        torch.cuda.synchronize(dev)
+        return timed_repeats(step, max(K, 100), stream, dev, world, B)
+
+    iso, _, _ = timed(0)
+    per, _, _ = timed(1)
+    stream_ms = statistics.median(per)
+    gr = torch.cuda.CUDAGraph()
+    n0 = B.launch_count()
+    with torch.cuda.graph(gr, capture_error_mode="thread_local"):
+        gs = torch.cuda.current_stream(dev)
+        B.pr_ctx_reset(ctx, stream=gs)
+        for t in range(T):
+            decode_call(t, gs)
+    nodes = B.launch_count() - n0
+    for _ in range(2):
+        gr.replay()
+    torch.cuda.synchronize(dev)
+    per_g, win, _ = timed_repeats(gr.replay, 1, torch.cuda.current_stream(dev), dev, world, B)
+    ms = statistics.median(per_g) / T
+    launches = nodes * len(per_g)
+    B.pr_ctx_set_option(ctx, B.PR_OPT_OVERLAP, 0)
+    clocks = sampler.summary(*win)
+    del gr
+
+    # parity: one more pass over the trace, untimed, keeping every finished
+    # request's outputs (gathered on the device at its EOS step)
+    B.pr_ctx_reset(ctx, stream=stream)
+    ends = {}
+    keep = []
+    for t in range(T):
+        decode_call(t, stream)
+        done = np.nonzero(tr.eos[t])[0]
+        if done.size:
+            idx = torch.from_numpy(done.astype(np.int64)).to(dev)
+            keep.append((t, done, [o.index_select(0, idx) for o in outs]))
+    torch.cuda.synchronize(dev)
+    for t, done, vals in keep:
+        vals = [v.cpu().numpy() for v in vals]
+        for j, s in enumerate(done):
+            ends[(int(s), t)] = [v[j] for v in vals]
+    finished = [(s, t0, L) for (s, t0, L) in tr.requests if t0 + L <= T]
+    sample = finished[:12] + finished[-4:]
+    import oracle
+    g = {"agg": [], "score": [], "ship": [], "req_flags": []}
+    o_all = {"agg": [], "score": [], "ship": [], "req_flags": []}
+    secs, rows = 0.0, 0
+    for (s, t0, L) in sample:
+        idx = torch.tensor([(t0 + i) * S + s for i in range(L)], dtype=torch.int64, device=dev)
+        xs = W.to_oracle_array(x_all.index_select(0, idx))
+        cs = ch_all.index_select(0, idx).cpu().numpy()
+        c0 = time.perf_counter()
+        o = oracle.route(xs, cs, np.array([0, L], np.int64), tr.w.astype(np.float64), tr.b,
+                         tr.tau, n_threads=threads)
+        secs += time.perf_counter() - c0
+        rows += L
+        sc, sh, fl, ag = ends[(s, t0 + L - 1)]
+        g["score"].append(sc)
+        g["ship"].append(sh)
+        g["req_flags"].append(fl)
+        g["agg"].append(ag)
+        for k in o_all:
+            o_all[k].append(o[k][0])
+    ok = parity_ok(np.array(g["agg"]), np.array(g["score"]), np.array(g["ship"]),
+                   np.array(g["req_flags"]), {k: np.array(v) for k, v in o_all.items()}, tr.tau)
+    parity = {"requests_checked": len(sample), "rows_checked": rows, "ok": ok,
+              "oracle_tokens_per_s": rows / secs if secs > 0 else None}
+    bytes_per_step = S * (wl.vocab * 2 + 4 + 4 + 1) + S * 4
+    desc = ("incremental decode-step verify: 256 live slots x 1,000 steps (256,000 rows, "
+            "77.8 GB resident), V=%d bf16 as the full-response rows, lengths U{64..1000}, "
+            "one pr_decode_step of 256 rows per step" % wl.vocab)
+    rec = _route_rec(wl, "decode", desc, "CUDA graph replays (a context reset and the 1,000-step "
+                     "trace per graph)", ms, statistics.median(iso), stream_ms, bytes_per_step, S,
+                     world, clocks, launches, T, len(per_g), parity,
+                     {"steps_per_graph": T, "kernels_per_graph": nodes, "replays_per_repeat": 1})
+    rec["generation_s"] = gen_s
+    rec["l2"] = "a 77.8 GB trace: every step reads new rows from DRAM"
+    B.pr_ctx_destroy(ctx)
+    del x_all, ch_all
+    torch.cuda.empty_cache()
+    return rec
+
+
+def measure_noalloc(B, x, ch, wl, dev, stream, K, warm, world, n_req: int = 26):
+    """pr_route_noalloc (no context, fixed scratch) beside pr_route on the same
+    whole batch: the first `n_req` requests of the full-response workload
+    (3,994 rows of V = 151,936 bf16), each call one launch."""
+    hi = int(wl.offsets[n_req])
+    xs, cs = x[:hi], ch[:hi]
+    off = torch.from_numpy(wl.offsets[:n_req + 1].copy()).to(dev)
+    w = torch.from_numpy(wl.w).to(dev)
+    o_na = (torch.empty(n_req, device=dev), torch.empty(n_req, dtype=torch.uint8, device=dev),
+            torch.empty(n_req, dtype=torch.int32, device=dev), torch.empty(n_req, 11, device=dev))
+    o_rt = tuple(torch.empty_like(t) for t in o_na)
+    ctx = B.pr_ctx_create(dev.index, max_rows=hi, max_requests=n_req)
+
+    def na():
+        B.pr_route_noalloc(xs, cs, off, w, wl.b, wl.tau, *o_na[:3], agg=o_na[3], stream=stream)
+
+    def rt():
+        B.pr_route(ctx, xs, cs, off, w, wl.b, wl.tau, score=o_rt[0], ship=o_rt[1],
+                   req_flags=o_rt[2], agg=o_rt[3], stream=stream)
+
+    res = {}
+    for name, fn in (("pr_route_noalloc", na), ("pr_route", rt)):
+        for _ in range(warm):
+            fn()
+        torch.cuda.synchronize(dev)
+        per, _, _ = timed_repeats(fn, K, stream, dev, world, B, min_s=0.5)
+        res[name] = statistics.median(per)
+    torch.cuda.synchronize(dev)
+    same = (torch.equal(o_na[1], o_rt[1]) and torch.equal(o_na[2], o_rt[2]) and
+            bool(torch.all((o_na[0] - o_rt[0]).abs() <= 1e-5 + 1e-4 * o_rt[0].abs())))
+    B.pr_ctx_destroy(ctx)
+    abytes = hi * (wl.vocab * 2 + 76) + n_req * 69
+    peak, _ = measured_peak()
+    return {"workload": "full-response rows 0..%d (%d requests), V=%d bf16, one call" % (
+                hi - 1, n_req, wl.vocab),
+            "ms_per_call": res["pr_route_noalloc"], "pr_route_ms_per_call": res["pr_route"],
+            "tokens_per_s": hi / (res["pr_route_noalloc"] / 1e3),
+            "frac": abytes / (res["pr_route_noalloc"] / 1e3) / 1e9 / peak,
+            "pr_route_frac": abytes / (res["pr_route"] / 1e3) / 1e9 / peak,
+            "same_decisions_as_pr_route": bool(same)}
+
+
+CONFIG_NAMES = {"c1": "tiny", "c3": "decode", "c4": "ragged", "c5": "wide"}
+
+
 def run_gb300(args):
     rank, world, local = dist_env()
     if world > 1:
@@ -257,51 +664,33 @@ def run_gb300(args):
     sampler = ClockSampler(local)
     sampler.start()
     K = args.steps
+    warm = max(3, args.warmup)
+    min_s = 0.05 if args.skip_host else MIN_TIMED_S
 
-    # (1) isolated launches: one event pair per launch, no overlap between steps
+    # (1) isolated launches: one launch at a time (no overlap between steps)
     B.pr_ctx_set_option(ctx, B.PR_OPT_OVERLAP, 0)
-    for _ in range(max(3, args.warmup)):
+    for _ in range(warm):
         step()
     torch.cuda.synchronize(dev)
-    ev = [torch.cuda.Event(enable_timing=True) for _ in range(K + 1)]
-    barrier(world)
-    torch.cuda.synchronize(dev)
-    ev[0].record(stream)
-    for i in range(K):
-        step()
-        ev[i + 1].record(stream)
-    torch.cuda.synchronize(dev)
-    barrier(world)
-    per_launch = [ev[i].elapsed_time(ev[i + 1]) for i in range(K)]
-    isolated_ms = reduce_max(ev[0].elapsed_time(ev[K]), world, dev) / K
+    iso_per, _, _ = timed_repeats(step, K, stream, dev, world, B, min_s=min_s)
+    isolated_ms = statistics.median(iso_per)
 
     # (2) the headline: K back-to-back steps, each allowed to start while the
-    # previous one finishes (programmatic dependent launch; results identical)
+    # previous one finishes (programmatic dependent launch; results identical),
+    # the K-step loop repeated until enough time is timed; median over repeats
     B.pr_ctx_set_option(ctx, B.PR_OPT_OVERLAP, 1)
-    for _ in range(max(3, args.warmup)):
+    for _ in range(warm):
         step()
     torch.cuda.synchronize(dev)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    barrier(world)
-    torch.cuda.synchronize(dev)
-    n_launch0 = B.launch_count()
-    t_wall0 = time.time()
-    e0.record(stream)
-    for i in range(K):
-        step()
-    e1.record(stream)
-    torch.cuda.synchronize(dev)
-    barrier(world)
-    t_wall1 = time.time()
-    launches = B.launch_count() - n_launch0
-    total_ms = reduce_max(e0.elapsed_time(e1), world, dev)
+    per, (t_wall0, t_wall1), launches = timed_repeats(step, K, stream, dev, world, B, min_s=min_s)
+    ms_step = statistics.median(per)
     B.pr_ctx_set_option(ctx, B.PR_OPT_OVERLAP, 0)
     clocks = sampler.summary(t_wall0, t_wall1)
-    sampler.stop()  # nvidia-smi polling is not part of the host-memory leg
     if args.skip_host:
+        sampler.stop()
         if rank == 0:
             print(json.dumps({"profiling_case": True, "rows": wl.n_rows, "steps": K,
-                              "ms_per_step": total_ms / K, "gpu_launches": launches}))
+                              "ms_per_step": ms_step, "gpu_launches": launches}))
         B.pr_ctx_destroy(ctx)
         return 0
 
@@ -327,30 +716,29 @@ def run_gb300(args):
         e2e_step()
     barrier(world)
     e2e_s = reduce_max(time.perf_counter() - t0, world, dev)
+    B.pr_ctx_destroy(ctx_h)
+    del hx, hc
 
-    h2d = hx.numel() * hx.element_size() + hc.numel() * 4 + hoff.numel() * 8 + hw.numel() * 4
-    d2h = hs.numel() * 4 + hsh.numel() + hf.numel() * 4
+    h2d = wl.n_rows * wl.vocab * 2 + hc_bytes(wl)
+    d2h = wl.n_req * (4 + 1 + 4)
     rows_all = wl.n_rows * world
-    value = rows_all * K / (total_ms / 1e3)
+    value = rows_all / (ms_step / 1e3)
     e2e_value = rows_all * e2e_steps / e2e_s
 
-    avg_launch_ms = total_ms / K  # steady state: one launch per step
     abytes = algorithmic_bytes(wl)
-    achieved = abytes / (avg_launch_ms / 1e3) / 1e9
+    achieved = abytes / (ms_step / 1e3) / 1e9
     isolated_achieved = abytes / (isolated_ms / 1e3) / 1e9
-    peaks_file = os.path.join(ROOT, "MEASURED_PEAKS.json")
-    peak, peak_src = 6800.0, "fallback"
-    if os.path.exists(peaks_file):
-        peak = float(json.load(open(peaks_file))["hbm_gbs"])
-        peak_src = "measured"
+    peak, peak_src = measured_peak()
+    cores = os.cpu_count() or 1
 
     line = None
+    configs = {}
+    noalloc = None
     if rank == 0:
         # parity of the timed run's outputs on a sample of whole requests, and
         # the oracle's own speed on that sample (the CPU baseline)
         import oracle
         oracle.build()
-        cores = os.cpu_count() or 1
         req_hi = 8
         lo, hi = 0, int(wl.offsets[req_hi])
         xs = W.to_oracle_array(x[lo:hi])
@@ -359,28 +747,50 @@ def run_gb300(args):
         # the same oracle on one core, on request 0 alone
         hi1 = int(wl.offsets[1])
         _, dt1, rows1 = oracle_sample(wl, xs[:hi1], cs[:hi1], 0, 1, 1)
-        g_agg = agg[:req_hi].cpu().numpy().astype(np.float64)
-        g_score = score[:req_hi].cpu().numpy().astype(np.float64)
-        ok = bool(np.all(np.abs(g_agg - o["agg"]) <= 1e-5 + 1e-4 * np.abs(o["agg"])) and
-                  np.all(np.abs(g_score - o["score"]) <= 1e-5 + 1e-4 * np.abs(o["score"])) and
-                  np.all((ship[:req_hi].cpu().numpy() == o["ship"]) |
-                         (np.abs(o["score"] - wl.tau) < 1e-6)) and
-                  np.all(hsh[:req_hi].numpy() == ship[:req_hi].cpu().numpy()))
+        ok = (parity_ok(agg[:req_hi].cpu().numpy(), score[:req_hi].cpu().numpy(),
+                        ship[:req_hi].cpu().numpy(), rflags[:req_hi].cpu().numpy(), o, wl.tau)
+              and bool(np.all(hsh[:req_hi].numpy() == ship[:req_hi].cpu().numpy())))
+        if not args.requests:
+            noalloc = measure_noalloc(B, x, ch, wl, dev, stream, K, warm, world)
+    B.pr_ctx_destroy(ctx)
+    del x, ch
+    torch.cuda.empty_cache()
+
+    if rank == 0 and world == 1 and args.configs != "none":
+        for key in [k.strip() for k in args.configs.split(",") if k.strip()]:
+            name = CONFIG_NAMES[key]
+            try:
+                if name == "decode":
+                    configs[key] = measure_decode_config(B, dev, stream, K, warm, world, sampler,
+                                                         cores)
+                else:
+                    configs[key] = measure_route_config(name, B, dev, stream, K, warm, world,
+                                                        sampler, cores)
+            except (RuntimeError, torch.cuda.OutOfMemoryError) as e:
+                torch.cuda.empty_cache()
+                configs[key] = {"workload": name, "value": None, "error": str(e).splitlines()[0]}
+    sampler.stop()
+
+    if rank == 0:
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
-            "warmup": max(3, args.warmup), "ms_per_step": total_ms / K, "higher_is_better": True,
+            "warmup": warm, "ms_per_step": ms_step, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": {"workload": workload_desc(wl), "rows_per_step_per_gpu": wl.n_rows,
                        "logit_bytes_per_step_per_gpu": wl.n_rows * wl.vocab * 2,
                        "l2": "inputs (2.69 GB) larger than L2 (129 MB), no flush",
                        "overlap": "back-to-back steps may overlap (PR_OPT_OVERLAP: programmatic "
                                   "dependent launch); isolated launches reported in roofline",
+                       "timing": "the K-step loop repeated %d times (at least %.1f s of device "
+                                 "time); ms_per_step is the median repeat" % (len(per), min_s),
                        "parallelism": "dp%d (independent batches)" % world},
+            "repeats": len(per),
+            "ms_per_step_repeats": {"min": min(per), "median": ms_step, "max": max(per)},
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak, "traffic": profiled_traffic(),
                          "kernel": "verify_rows_ws<bf16, route>", "peak_source": peak_src,
                          "algorithmic_bytes_per_launch": abytes,
-                         "avg_launch_ms": avg_launch_ms,
+                         "avg_launch_ms": ms_step,
                          "isolated_launch_ms": isolated_ms,
                          "isolated_achieved": isolated_achieved,
                          "isolated_frac": isolated_achieved / peak,
@@ -393,24 +803,36 @@ def run_gb300(args):
                                       "kind": "oracle",
                                       "sample": "request 0 (%d rows), float64 C oracle, 1 thread"
                                                 % rows1},
-            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d // world * world,
+            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d * world,
                     "d2h_bytes_per_step": d2h, "api": "pr_route_host (pinned host buffers)"},
             "gpu_launches": launches,
+            "timed_steps_total": K * len(per),
             "clocks": clocks,
             "parity": {"requests_checked": req_hi, "rows_checked": rows, "ok": ok},
         }
+        if configs:
+            line["configs"] = configs
+        if noalloc:
+            line["noalloc"] = noalloc
+        line = gate_on_parity(line)
+        if line["value"] is None:
+            line["e2e"]["value"] = None
         print(json.dumps(line))
-    B.pr_ctx_destroy(ctx_h)
-    B.pr_ctx_destroy(ctx)
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
     return 0
 
+
+def hc_bytes(wl) -> int:
+    """Host-to-device bytes of one end-to-end step beside the logits: token
+    ids, offsets and scorer weights."""
+    return wl.n_rows * 4 + (wl.n_req + 1) * 8 + 11 * 4
+
+
 def run_other_workload(args):
-    """The four other workloads, timed the same way (CUDA events on the stream,
-    max over ranks); inputs resident in HBM.  Batches smaller than L2 are
-    rotated over distinct copies so every step reads from DRAM."""
+    """One of the four other verifier workloads on its own line, measured as
+    the default run's `configs` records are."""
     rank, world, local = dist_env()
     if world > 1:
         import torch.distributed as dist
@@ -421,165 +843,32 @@ def run_other_workload(args):
     prbuild.build()
     from paper_2608_28726_gb300 import binding as B
     stream = torch.cuda.current_stream(dev)
-    name = args.workload
-    launches0 = None
-
-    if name == "decode":
-        tr = W.decode_trace()
-        wl = tr.as_workload()
-        S, T = tr.n_slots, tr.n_steps
-        x_all = torch.empty(T * S, wl.vocab, dtype=wl.torch_dtype, device=dev)
-        ch_all = torch.empty(T * S, dtype=torch.int32, device=dev)
-        W.rows(wl, 0, T * S, device=dev, out=x_all, chosen_out=ch_all)
-        eos = torch.from_numpy(tr.eos).to(dev)
-        slot = torch.arange(S, dtype=torch.int32, device=dev)
-        w = torch.from_numpy(tr.w).to(dev)
-        ctx = B.pr_ctx_create(local, max_rows=S, max_requests=S)
-        outs = (torch.empty(S, device=dev), torch.empty(S, dtype=torch.uint8, device=dev),
-                torch.empty(S, dtype=torch.int32, device=dev))
-        state = {"t": 0}
-
-        def decode_call(t, st):
-            B.pr_decode_step(ctx, x_all[t * S:(t + 1) * S], slot, ch_all[t * S:(t + 1) * S], eos[t],
-                             w, tr.b, tr.tau, *outs, stream=st)
-
-        def step():
-            t = state["t"]
-            if t == T:
-                B.pr_ctx_reset(ctx, stream=stream)
-                t = 0
-            decode_call(t, stream)
-            state["t"] = t + 1
-
-        def graph_body(st):  # a context reset and the whole trace
-            B.pr_ctx_reset(ctx, stream=st)
-            for t in range(T):
-                decode_call(t, st)
-            return T
-
-        rows_per_step = S
-        bytes_per_step = S * (wl.vocab * 2 + 4 + 1 + 4) + S * 4
-        desc = ("decode steps: 256 live slots x 1,000 steps (%d rows resident), V=%d bf16, "
-                "lengths U{64..1000}, one pr_decode_step per step" % (T * S, wl.vocab))
-        dtype = "bf16"
+    sampler = ClockSampler(local)
+    sampler.start()
+    warm = max(3, args.warmup)
+    cores = os.cpu_count() or 1
+    if args.workload == "decode":
+        rec = measure_decode_config(B, dev, stream, args.steps, warm, world, sampler, cores)
     else:
-        wl = W.make(name)
-        copies = 1
-        if name == "tiny":
-            copies = 8  # 8 x 45 MB rotated: more than L2 between reuses
-        xs, chs = [], []
-        for c in range(copies):
-            x = torch.empty(wl.n_rows, wl.vocab, dtype=wl.torch_dtype, device=dev)
-            ch = torch.empty(wl.n_rows, dtype=torch.int32, device=dev)
-            W.rows(wl, 0, wl.n_rows, device=dev, out=x, chosen_out=ch)
-            xs.append(x)
-            chs.append(ch)
-        off = torch.from_numpy(wl.offsets).to(dev)
-        w = torch.from_numpy(wl.w).to(dev)
-        ctx = B.pr_ctx_create(local, max_rows=wl.n_rows, max_requests=wl.n_req)
-        outs = (torch.empty(wl.n_req, device=dev), torch.empty(wl.n_req, dtype=torch.uint8, device=dev),
-                torch.empty(wl.n_req, dtype=torch.int32, device=dev))
-        chunk = wl.chunk_rows or wl.n_rows
-        state = {"c": 0}
-
-        def route_call(c, st):
-            for lo in range(0, wl.n_rows, chunk):
-                hi = min(wl.n_rows, lo + chunk)
-                B.pr_route(ctx, xs[c][lo:hi], chs[c][lo:hi], off, w, wl.b, wl.tau, row_base=lo,
-                           score=outs[0], ship=outs[1], req_flags=outs[2], agg=None,
-                           stream=st, want_agg=False)
-
-        def step():
-            c = state["c"] % copies
-            state["c"] += 1
-            route_call(c, stream)
-
-        def graph_body(st):  # one step on each rotated copy
-            for c in range(copies):
-                route_call(c, st)
-            return copies
-
-        rows_per_step = wl.n_rows
-        bytes_per_step = algorithmic_bytes(wl)
-        desc = {"tiny": "tiny: 8 requests, T~U{16..64} (%d rows), V=%d fp32, 8 rotated copies",
-                "ragged": "ragged: 1,024 requests, lognormal lengths (%d rows), V=%d bf16, "
-                          "8,192-row chunks",
-                "wide": "wide vocabulary: 512 requests, T~U{64..512} (%d rows), V=%d fp32 "
-                        "Student-t(3), one launch"}[name] % (wl.n_rows, wl.vocab)
-        dtype = "f32" if wl.dtype == "f32" else "bf16"
-
-    K = args.steps
-
-    def timed(overlap: int):
-        B.pr_ctx_set_option(ctx, B.PR_OPT_OVERLAP, overlap)
-        for _ in range(max(3, args.warmup)):
-            step()
-        torch.cuda.synchronize(dev)
-        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        barrier(world)
-        torch.cuda.synchronize(dev)
-        n0 = B.launch_count()
-        ev0.record(stream)
-        for _ in range(K):
-            step()
-        ev1.record(stream)
-        torch.cuda.synchronize(dev)
-        barrier(world)
-        return reduce_max(ev0.elapsed_time(ev1), world, dev) / K, B.launch_count() - n0
-
-    isolated_ms, _ = timed(0)
-    ms, launches = timed(1)
-    stream_ms = ms
-    graph_info = None
-    if name in ("tiny", "decode"):
-        # launch-bound loops: the steps captured in one CUDA graph (tiny: one
-        # step per rotated copy; decode: a reset and the whole trace), replayed
-        gr = torch.cuda.CUDAGraph()
-        n0 = B.launch_count()
-        with torch.cuda.graph(gr, capture_error_mode="thread_local"):
-            per = graph_body(torch.cuda.current_stream(dev))
-        nodes = B.launch_count() - n0
-        gst = torch.cuda.current_stream(dev)
-        for _ in range(2):
-            gr.replay()
-        torch.cuda.synchronize(dev)
-        reps = max(3, -(-1000 // per))
-        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        barrier(world)
-        torch.cuda.synchronize(dev)
-        ev0.record(gst)
-        for _ in range(reps):
-            gr.replay()
-        ev1.record(gst)
-        torch.cuda.synchronize(dev)
-        barrier(world)
-        ms = reduce_max(ev0.elapsed_time(ev1), world, dev) / (reps * per)
-        launches = nodes * reps
-        K = reps * per
-        graph_info = {"steps_per_graph": per, "replays": reps, "kernels_per_graph": nodes}
-    B.pr_ctx_set_option(ctx, B.PR_OPT_OVERLAP, 0)
-    peaks_file = os.path.join(ROOT, "MEASURED_PEAKS.json")
-    peak = float(json.load(open(peaks_file))["hbm_gbs"]) if os.path.exists(peaks_file) else 6800.0
-    achieved = bytes_per_step / (ms / 1e3) / 1e9
+        rec = measure_route_config(args.workload, B, dev, stream, args.steps, warm, world,
+                                   sampler, cores)
+    sampler.stop()
     if rank == 0:
-        print(json.dumps({
-            "metric": "verified tokens/sec (%s workload)" % name,
-            "value": rows_per_step * world / (ms / 1e3), "unit": UNIT, "n_gpus": world, "steps": K,
-            "warmup": max(3, args.warmup), "ms_per_step": ms, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": dtype, "data": "synthetic",
-            "config": {"workload": desc, "rows_per_step_per_gpu": rows_per_step,
-                       "timing": ("CUDA graph replays (%d steps per graph, %d replays)" %
-                                  (graph_info["steps_per_graph"], graph_info["replays"])
-                                  if graph_info else "stream of back-to-back calls")},
-            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                         "frac": achieved / peak, "traffic": None,
-                         "algorithmic_bytes_per_step": bytes_per_step,
-                         "stream_ms_per_step": stream_ms,
-                         "isolated_ms_per_step": isolated_ms,
-                         "isolated_frac": bytes_per_step / (isolated_ms / 1e3) / 1e9 / peak},
-            "graph": graph_info,
-            "gpu_launches": launches}))
-    B.pr_ctx_destroy(ctx)
+        line = {"metric": "verified tokens/sec (%s workload)" % args.workload,
+                "value": rec["value"], "unit": UNIT, "n_gpus": world, "steps": rec["steps"],
+                "warmup": warm, "ms_per_step": rec["ms_per_step"], "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None, "dtype": rec["dtype"],
+                "data": "synthetic",
+                "config": {"workload": rec["workload"], "timing": rec["timing"],
+                           "rows_per_step_per_gpu": rec["rows_per_step_per_gpu"],
+                           "l2": rec["l2"]},
+                "roofline": rec["roofline"], "gpu_launches": rec["gpu_launches"],
+                "clocks": rec["clocks"], "parity": rec["parity"]}
+        if "graph" in rec:
+            line["graph"] = rec["graph"]
+        if "value_withheld" in rec:
+            line["value_withheld"] = rec["value_withheld"]
+        print(json.dumps(line))
     return 0
 
 
@@ -1309,6 +1598,9 @@ def main():
                          "workloads, head (the transformer scorer head), quantile (the "
                          "quantile-summary MLP), selective (calibration and ranking metrics) "
                          "or lmhead (the LM head fused with the row reduction)")
+    ap.add_argument("--configs", default="c1,c3,c4,c5",
+                    help="default run: the other workloads measured into the line's `configs` "
+                         "object (c1 tiny, c3 decode, c4 ragged, c5 wide; 'none' for none)")
     ap.add_argument("--requests", type=int, default=0,
                     help="profiling only: the first N requests of the workload")
     ap.add_argument("--skip-host", action="store_true",

@@ -391,7 +391,7 @@ pr_status pr_selftest_wait(pr_ctx* ctx, int64_t limit_ns, int32_t* completed);
 
 /*
  * The verifier-architecture ablation's alternative scorer (Section 4.2,
- * Table 2, "quantile summary + MLP").  Per request, for each feature x in
+ * Table 2): an MLP over quantiles pooled per request.  Per request, for each feature x in
  * (l, m, h, rho) (record slots LOGP, MAXP, TOPK, RHO of Eq. 3) over its T
  * rows, the quantiles at levels 0, 1/10, 1/4, 1/2, 3/4, 9/10, 1 by linear
  * interpolation between order statistics (x_(0) <= ... <= x_(T-1); level a/b:
@@ -474,12 +474,18 @@ pr_status pr_selective_metrics(pr_ctx* ctx, const float* scores, const uint8_t* 
  * exits.  Limits: 1 <= n_rows <= PR_NOALLOC_MAX_ROWS and
  * 1 <= n_req <= PR_NOALLOC_MAX_REQUESTS; larger batches are rejected with
  * PR_ERR_INVALID_ARG before anything is queued (use pr_route with a context
- * instead).  offsets[n_req] must not exceed n_rows (requests reaching past it
- * get PR_FLAG_BAD_OFFSETS).
+ * instead).  The offsets must cover the batch exactly, offsets[n_req] ==
+ * n_rows: there is no flag word the caller could read afterwards, so a
+ * request reaching past n_rows gets PR_FLAG_BAD_OFFSETS, and when
+ * offsets[n_req] < n_rows the last request is reported with
+ * PR_FLAG_BAD_OFFSETS and a NaN score while the rows after offsets[n_req],
+ * which belong to no request, are not verified.
  *
  * The first call on a device looks up the scratch array's device address and
  * the launch shape, once, with that device current; make that first call
- * before any stream capture.  Every call clears the counters it needs on
+ * before any stream capture.  The address is kept for the life of the
+ * process: after cudaDeviceReset (which unloads the library's device code)
+ * this call must not be used on that device again.  Every call clears the counters it needs on
  * `stream` and then reuses the same array, which keeps the previous call's
  * contents: two calls whose work overlaps on the GPU (different streams, no
  * ordering between them) race on the scratch and give undefined results.

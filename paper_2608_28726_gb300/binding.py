@@ -86,10 +86,12 @@ _lib.pr_head_param_count.restype = _I64
 
 
 class PRError(RuntimeError):
-    def __init__(self, status: int, call: str):
+    def __init__(self, status: int, call: str, detail: str | None = None):
         msg = _lib.pr_status_string(status).decode()
         if status == PR_ERR_CUDA:
             msg += " (" + _lib.pr_last_cuda_error().decode() + ")"
+        if detail:
+            msg += " (" + detail + ")"
         super().__init__("%s: %s" % (call, msg))
         self.status = status
 
@@ -97,6 +99,69 @@ class PRError(RuntimeError):
 def _check(st: int, call: str):
     if st != PR_OK:
         raise PRError(st, call)
+
+
+# ---- argument checks before any pointer reaches the library -------------------------
+#
+# The C ABI cannot tell a host pointer from a device pointer, nor a buffer's
+# size, without a driver query per call; a CPU tensor, a tensor on another GPU
+# or a short output buffer would reach a kernel as a bad address.  So every
+# tensor meant for device memory is checked here: a CUDA tensor on the
+# device of the context (or the current device for the context-free call),
+# of the expected dtype, contiguous, and at least as large as the call needs.
+
+_CTX_DEVICE = {}  # context handle value -> CUDA device index
+
+_I32_T = (torch.int32,)
+_U8_T = (torch.uint8, torch.bool)
+_F32_T = (torch.float32,)
+_I64_T = (torch.int64,)
+
+
+def _ctx_device(ctx) -> int:
+    h = getattr(ctx, "value", ctx)
+    if h in _CTX_DEVICE:
+        return _CTX_DEVICE[h]
+    return torch.cuda.current_device() if torch.cuda.is_available() else 0
+
+
+def _dev(call: str, dev: int, name: str, t, dtypes=None, numel: int | None = None,
+         optional: bool = False, contiguous: bool = True):
+    if t is None:
+        if optional:
+            return
+        raise PRError(PR_ERR_INVALID_ARG, call, "%s is required" % name)
+    if not isinstance(t, torch.Tensor) or not t.is_cuda or t.device.index != dev:
+        where = t.device if isinstance(t, torch.Tensor) else type(t).__name__
+        raise PRError(PR_ERR_INVALID_ARG, call,
+                      "%s must be a CUDA tensor on cuda:%d, got %s" % (name, dev, where))
+    if dtypes is not None and t.dtype not in dtypes:
+        raise PRError(PR_ERR_INVALID_ARG, call, "%s has dtype %s, expected %s" % (
+            name, t.dtype, " or ".join(str(d) for d in dtypes)))
+    if contiguous and not t.is_contiguous():
+        raise PRError(PR_ERR_INVALID_ARG, call, "%s must be contiguous" % name)
+    if numel is not None and t.numel() < numel:
+        raise PRError(PR_ERR_INVALID_ARG, call, "%s holds %d elements, the call needs %d" % (
+            name, t.numel(), numel))
+
+
+def _host(call: str, name: str, t, optional: bool = False):
+    if t is None:
+        if optional:
+            return
+        raise PRError(PR_ERR_INVALID_ARG, call, "%s is required" % name)
+    if isinstance(t, torch.Tensor):
+        if t.is_cuda:
+            raise PRError(PR_ERR_INVALID_ARG, call, "%s must be in host memory" % name)
+        if not t.is_contiguous():
+            raise PRError(PR_ERR_INVALID_ARG, call, "%s must be contiguous" % name)
+    elif not isinstance(t, np.ndarray):
+        raise PRError(PR_ERR_INVALID_ARG, call, "%s must be a host tensor" % name)
+
+
+def _logits(call: str, dev: int, logits):
+    if not isinstance(logits, torch.Tensor) or not logits.is_cuda or logits.device.index != dev:
+        _dev(call, dev, "logits", logits)
 
 
 def _ptr(t):
@@ -147,11 +212,13 @@ def pr_ctx_create(device: int = 0, max_rows: int = 0, max_requests: int = 0):
     h = ctypes.c_void_p()
     _check(_lib.pr_ctx_create(ctypes.byref(h), int(device), int(max_rows), int(max_requests)),
            "pr_ctx_create")
+    _CTX_DEVICE[h.value] = int(device)
     return h
 
 
 def pr_ctx_destroy(ctx):
     _check(_lib.pr_ctx_destroy(ctx), "pr_ctx_destroy")
+    _CTX_DEVICE.pop(getattr(ctx, "value", ctx), None)
 
 
 def pr_ctx_reset(ctx, stream=None):
@@ -186,94 +253,156 @@ def pr_last_error(ctx) -> int:
 
 # ---- verifier calls ------------------------------------------------------------------
 
+_FLAG_T = (torch.int32,) + ((torch.uint32,) if hasattr(torch, "uint32") else ())
+
+
 def pr_token_features(ctx, logits, chosen, topk: int = 20, offsets=None, feat=None, top2=None,
                       row_flags=None, vocab=None, stream=None):
+    call = "pr_token_features"
+    dev = _ctx_device(ctx)
+    _logits(call, dev, logits)
     n = logits.size(0)
     V, stride = _rows(logits, vocab)
-    dev = logits.device
-    feat = torch.empty(n, PR_NFEAT, dtype=torch.float32, device=dev) if feat is None else feat
-    top2 = torch.empty(n, 2, dtype=torch.int32, device=dev) if top2 is None else top2
-    row_flags = torch.empty(n, dtype=torch.int32, device=dev) if row_flags is None else row_flags
+    d = logits.device
+    feat = torch.empty(n, PR_NFEAT, dtype=torch.float32, device=d) if feat is None else feat
+    top2 = torch.empty(n, 2, dtype=torch.int32, device=d) if top2 is None else top2
+    row_flags = torch.empty(n, dtype=torch.int32, device=d) if row_flags is None else row_flags
     n_req = 0 if offsets is None else offsets.numel() - 1
+    _dev(call, dev, "chosen", chosen, _I32_T, n)
+    _dev(call, dev, "offsets", offsets, _I64_T, optional=True)
+    _dev(call, dev, "feat", feat, _F32_T, n * PR_NFEAT)
+    _dev(call, dev, "top2", top2, _I32_T, 2 * n)
+    _dev(call, dev, "row_flags", row_flags, _FLAG_T, n)
     _check(_lib.pr_token_features(ctx, _ptr(logits), _dtype(logits), n, V, stride, _ptr(chosen),
                                   int(topk), _ptr(offsets), n_req, _ptr(feat), _ptr(top2),
-                                  _ptr(row_flags), _stream(stream)), "pr_token_features")
+                                  _ptr(row_flags), _stream(stream)), call)
     return feat, top2, row_flags
+
+
+def _request_outputs(call, dev, n_req, score, ship, req_flags, agg=None, want_agg=False):
+    d = torch.device("cuda", dev)
+    score = torch.empty(n_req, dtype=torch.float32, device=d) if score is None else score
+    ship = torch.empty(n_req, dtype=torch.uint8, device=d) if ship is None else ship
+    req_flags = torch.empty(n_req, dtype=torch.int32, device=d) if req_flags is None else req_flags
+    if agg is None and want_agg:
+        agg = torch.empty(n_req, PR_NAGG, dtype=torch.float32, device=d)
+    _dev(call, dev, "score", score, _F32_T, n_req)
+    _dev(call, dev, "ship", ship, _U8_T, n_req)
+    _dev(call, dev, "req_flags", req_flags, _FLAG_T, n_req)
+    _dev(call, dev, "agg", agg, _F32_T, n_req * PR_NAGG, optional=True)
+    return score, ship, req_flags, agg
+
+
+def _offsets_and_w(call, dev, offsets, w, n_w=PR_NAGG):
+    _dev(call, dev, "offsets", offsets, _I64_T)
+    _dev(call, dev, "w", w, _F32_T, n_w)
+    return offsets.numel() - 1
 
 
 def pr_aggregate_score(ctx, feat, offsets, w, b: float, tau: float, row_flags=None, agg=None,
                        score=None, ship=None, req_flags=None, stream=None):
-    n_req = offsets.numel() - 1
-    dev = feat.device
-    agg = torch.empty(n_req, PR_NAGG, dtype=torch.float32, device=dev) if agg is None else agg
-    score = torch.empty(n_req, dtype=torch.float32, device=dev) if score is None else score
-    ship = torch.empty(n_req, dtype=torch.uint8, device=dev) if ship is None else ship
-    req_flags = torch.empty(n_req, dtype=torch.int32, device=dev) if req_flags is None else req_flags
-    _check(_lib.pr_aggregate_score(ctx, _ptr(feat), _ptr(row_flags), feat.size(0), _ptr(offsets),
+    call = "pr_aggregate_score"
+    dev = _ctx_device(ctx)
+    n_req = _offsets_and_w(call, dev, offsets, w)
+    _dev(call, dev, "feat", feat, _F32_T)
+    n_rows = feat.size(0) if feat.dim() > 0 else 0
+    _dev(call, dev, "feat", feat, _F32_T, n_rows * PR_NFEAT)
+    _dev(call, dev, "row_flags", row_flags, _FLAG_T, n_rows, optional=True)
+    score, ship, req_flags, agg = _request_outputs(call, dev, n_req, score, ship, req_flags, agg,
+                                                   want_agg=True)
+    _check(_lib.pr_aggregate_score(ctx, _ptr(feat), _ptr(row_flags), n_rows, _ptr(offsets),
                                    n_req, _ptr(w), float(b), float(tau), _ptr(agg), _ptr(score),
-                                   _ptr(ship), _ptr(req_flags), _stream(stream)),
-           "pr_aggregate_score")
+                                   _ptr(ship), _ptr(req_flags), _stream(stream)), call)
     return agg, score, ship, req_flags
 
 
 def pr_route(ctx, logits, chosen, offsets, w, b: float, tau: float, row_base: int = 0, score=None,
              ship=None, req_flags=None, agg=None, vocab=None, stream=None, want_agg: bool = True):
+    call = "pr_route"
+    dev = _ctx_device(ctx)
+    _logits(call, dev, logits)
     n = logits.size(0)
     V, stride = _rows(logits, vocab)
-    n_req = offsets.numel() - 1
-    dev = logits.device
-    score = torch.empty(n_req, dtype=torch.float32, device=dev) if score is None else score
-    ship = torch.empty(n_req, dtype=torch.uint8, device=dev) if ship is None else ship
-    req_flags = torch.empty(n_req, dtype=torch.int32, device=dev) if req_flags is None else req_flags
-    if agg is None and want_agg:
-        agg = torch.empty(n_req, PR_NAGG, dtype=torch.float32, device=dev)
+    n_req = _offsets_and_w(call, dev, offsets, w)
+    _dev(call, dev, "chosen", chosen, _I32_T, n)
+    score, ship, req_flags, agg = _request_outputs(call, dev, n_req, score, ship, req_flags, agg,
+                                                   want_agg)
     _check(_lib.pr_route(ctx, _ptr(logits), _dtype(logits), int(row_base), n, V, stride,
                          _ptr(chosen), _ptr(offsets), n_req, _ptr(w), float(b), float(tau),
                          _ptr(score), _ptr(ship), _ptr(req_flags), _ptr(agg), _stream(stream)),
-           "pr_route")
+           call)
     return score, ship, req_flags, agg
 
 
 def pr_route_host(ctx, logits, chosen, offsets, w, b: float, tau: float, chunk_rows: int = 8192,
                   score=None, ship=None, req_flags=None, agg=None, vocab=None, stream=None):
     """Host tensors in, host tensors out (pinned host memory copies fastest)."""
+    call = "pr_route_host"
+    _host(call, "logits", logits)
     n = logits.size(0)
     V, stride = _rows(logits, vocab)
     n_req = offsets.numel() - 1
     score = torch.empty(n_req, dtype=torch.float32) if score is None else score
     ship = torch.empty(n_req, dtype=torch.uint8) if ship is None else ship
     req_flags = torch.empty(n_req, dtype=torch.int32) if req_flags is None else req_flags
+    for name, t in (("chosen", chosen), ("offsets", offsets), ("w", w), ("score", score),
+                    ("ship", ship), ("req_flags", req_flags)):
+        _host(call, name, t)
+    _host(call, "agg", agg, optional=True)
     _check(_lib.pr_route_host(ctx, _ptr(logits), _dtype(logits), n, V, stride, _ptr(chosen),
                               _ptr(offsets), n_req, _ptr(w), float(b), float(tau), int(chunk_rows),
                               _ptr(score), _ptr(ship), _ptr(req_flags), _ptr(agg),
-                              _stream(stream)), "pr_route_host")
+                              _stream(stream)), call)
     return score, ship, req_flags, agg
 
 
 def pr_route_noalloc(logits, chosen, offsets, w, b: float, tau: float, score, ship, req_flags,
                      agg=None, vocab=None, stream=None):
     """pr_route for callers that cannot allocate: no context, the library's
-    fixed scratch, every output buffer supplied by the caller (device tensors on
-    the current device).  Batches above PR_NOALLOC_MAX_ROWS rows or
-    PR_NOALLOC_MAX_REQUESTS requests raise PRError (invalid argument)."""
+    fixed scratch, every output buffer supplied by the caller (CUDA tensors on
+    the current device; anything else raises PRError before the library is
+    called).  Batches above PR_NOALLOC_MAX_ROWS rows or PR_NOALLOC_MAX_REQUESTS
+    requests raise PRError (invalid argument).  The offsets must cover the
+    batch: when offsets[n_req] < n_rows the last request is reported with
+    PR_FLAG_BAD_OFFSETS and a NaN score, and the rows after offsets[n_req] are
+    not verified."""
+    call = "pr_route_noalloc"
+    if not torch.cuda.is_available():
+        raise PRError(PR_ERR_UNSUPPORTED, call, "no CUDA device")
+    dev = torch.cuda.current_device()
+    _logits(call, dev, logits)
     n = logits.size(0)
     V, stride = _rows(logits, vocab)
-    n_req = offsets.numel() - 1
+    n_req = _offsets_and_w(call, dev, offsets, w)
+    _dev(call, dev, "chosen", chosen, _I32_T, n)
+    _request_outputs(call, dev, n_req, score, ship, req_flags, agg)
     _check(_lib.pr_route_noalloc(_ptr(logits), _dtype(logits), n, V, stride, _ptr(chosen),
                                  _ptr(offsets), n_req, _ptr(w), float(b), float(tau), _ptr(score),
-                                 _ptr(ship), _ptr(req_flags), _ptr(agg), _stream(stream)),
-           "pr_route_noalloc")
+                                 _ptr(ship), _ptr(req_flags), _ptr(agg), _stream(stream)), call)
     return score, ship, req_flags, agg
 
 
 def pr_decode_step(ctx, logits, slot, chosen, eos, w, b: float, tau: float, score_out, ship_out,
                    slot_flags, agg_out=None, vocab=None, stream=None):
+    """One decode step: row i belongs to slot[i].  The outputs are indexed by
+    slot, so they must hold an entry for every slot index passed."""
+    call = "pr_decode_step"
+    dev = _ctx_device(ctx)
+    _logits(call, dev, logits)
     n = logits.size(0)
     V, stride = _rows(logits, vocab)
+    _dev(call, dev, "slot", slot, _I32_T, n)
+    _dev(call, dev, "chosen", chosen, _I32_T, n)
+    _dev(call, dev, "eos", eos, _U8_T, n)
+    _dev(call, dev, "w", w, _F32_T, PR_NAGG)
+    _dev(call, dev, "score_out", score_out, _F32_T)
+    _dev(call, dev, "ship_out", ship_out, _U8_T)
+    _dev(call, dev, "slot_flags", slot_flags, _FLAG_T)
+    _dev(call, dev, "agg_out", agg_out, _F32_T, optional=True)
     _check(_lib.pr_decode_step(ctx, _ptr(logits), _dtype(logits), n, V, stride, _ptr(slot),
                                _ptr(chosen), _ptr(eos), _ptr(w), float(b), float(tau),
                                _ptr(score_out), _ptr(ship_out), _ptr(slot_flags), _ptr(agg_out),
-                               _stream(stream)), "pr_decode_step")
+                               _stream(stream)), call)
 
 
 def pr_state_export(ctx) -> bytes:
@@ -297,14 +426,18 @@ def pr_head_param_count(n_layers: int) -> int:
 
 def pr_head_score(ctx, feat, offsets, w, n_layers: int, tau: float, row_flags=None, score=None,
                   ship=None, req_flags=None, stream=None):
-    n_req = offsets.numel() - 1
-    dev = feat.device
-    score = torch.empty(n_req, dtype=torch.float32, device=dev) if score is None else score
-    ship = torch.empty(n_req, dtype=torch.uint8, device=dev) if ship is None else ship
-    req_flags = torch.empty(n_req, dtype=torch.int32, device=dev) if req_flags is None else req_flags
-    _check(_lib.pr_head_score(ctx, _ptr(feat), _ptr(row_flags), feat.size(0), _ptr(offsets), n_req,
+    call = "pr_head_score"
+    dev = _ctx_device(ctx)
+    n_w = pr_head_param_count(n_layers)
+    n_req = _offsets_and_w(call, dev, offsets, w, max(n_w, 0))
+    _dev(call, dev, "feat", feat, _F32_T)
+    n_rows = feat.size(0) if feat.dim() > 0 else 0
+    _dev(call, dev, "feat", feat, _F32_T, n_rows * PR_NFEAT)
+    _dev(call, dev, "row_flags", row_flags, _FLAG_T, n_rows, optional=True)
+    score, ship, req_flags, _ = _request_outputs(call, dev, n_req, score, ship, req_flags)
+    _check(_lib.pr_head_score(ctx, _ptr(feat), _ptr(row_flags), n_rows, _ptr(offsets), n_req,
                               _ptr(w), int(n_layers), float(tau), _ptr(score), _ptr(ship),
-                              _ptr(req_flags), _stream(stream)), "pr_head_score")
+                              _ptr(req_flags), _stream(stream)), call)
     return score, ship, req_flags
 
 
@@ -319,6 +452,10 @@ class PrSelective(ctypes.Structure):
 def pr_selective_metrics(ctx, scores, q: float, labels=None, stream=None) -> dict:
     """Calibrate tau for ship fraction q on device scores; with device labels
     (uint8, non-zero = correct) also AUROC, AUARC and the shipped accuracy."""
+    call = "pr_selective_metrics"
+    dev = _ctx_device(ctx)
+    _dev(call, dev, "scores", scores, _F32_T)
+    _dev(call, dev, "labels", labels, _U8_T, scores.numel(), optional=True)
     res = PrSelective()
     _check(_lib.pr_selective_metrics(ctx, _ptr(scores), _ptr(labels), scores.numel(), float(q),
                                      ctypes.byref(res), _stream(stream)), "pr_selective_metrics")
@@ -329,17 +466,20 @@ def pr_selective_metrics(ctx, scores, q: float, labels=None, stream=None) -> dic
 
 def pr_quantile_score(ctx, feat, offsets, w, tau: float, row_flags=None, summary=None, score=None,
                       ship=None, req_flags=None, want_summary: bool = True, stream=None):
-    n_req = offsets.numel() - 1
-    dev = feat.device
+    call = "pr_quantile_score"
+    dev = _ctx_device(ctx)
+    n_req = _offsets_and_w(call, dev, offsets, w, PR_QMLP_PARAMS)
+    _dev(call, dev, "feat", feat, _F32_T)
+    n_rows = feat.size(0) if feat.dim() > 0 else 0
+    _dev(call, dev, "feat", feat, _F32_T, n_rows * PR_NFEAT)
+    _dev(call, dev, "row_flags", row_flags, _FLAG_T, n_rows, optional=True)
     if summary is None and want_summary:
-        summary = torch.empty(n_req, PR_QMLP_SUMMARY, dtype=torch.float32, device=dev)
-    score = torch.empty(n_req, dtype=torch.float32, device=dev) if score is None else score
-    ship = torch.empty(n_req, dtype=torch.uint8, device=dev) if ship is None else ship
-    req_flags = torch.empty(n_req, dtype=torch.int32, device=dev) if req_flags is None else req_flags
-    _check(_lib.pr_quantile_score(ctx, _ptr(feat), _ptr(row_flags), feat.size(0), _ptr(offsets),
+        summary = torch.empty(n_req, PR_QMLP_SUMMARY, dtype=torch.float32, device=feat.device)
+    _dev(call, dev, "summary", summary, _F32_T, n_req * PR_QMLP_SUMMARY, optional=True)
+    score, ship, req_flags, _ = _request_outputs(call, dev, n_req, score, ship, req_flags)
+    _check(_lib.pr_quantile_score(ctx, _ptr(feat), _ptr(row_flags), n_rows, _ptr(offsets),
                                   n_req, _ptr(w), float(tau), _ptr(summary), _ptr(score),
-                                  _ptr(ship), _ptr(req_flags), _stream(stream)),
-           "pr_quantile_score")
+                                  _ptr(ship), _ptr(req_flags), _stream(stream)), call)
     return score, ship, req_flags, summary
 
 
@@ -353,13 +493,22 @@ def pr_lmhead_features(ctx, hidden, weight, chosen, topk: int = 20, offsets=None
         raise TypeError("hidden and weight must be bfloat16")
     if not (hidden.is_contiguous() and weight.is_contiguous()) or hidden.size(1) != weight.size(1):
         raise ValueError("hidden [n][d] and weight [V][d] must be contiguous with the same d")
+    call = "pr_lmhead_features"
+    dev = _ctx_device(ctx)
+    _dev(call, dev, "hidden", hidden)
+    _dev(call, dev, "weight", weight)
     n, d = hidden.shape
     V = weight.size(0)
-    dev = hidden.device
-    feat = torch.empty(n, PR_NFEAT, dtype=torch.float32, device=dev) if feat is None else feat
-    top2 = torch.empty(n, 2, dtype=torch.int32, device=dev) if top2 is None else top2
-    row_flags = torch.empty(n, dtype=torch.int32, device=dev) if row_flags is None else row_flags
+    feat = torch.empty(n, PR_NFEAT, dtype=torch.float32, device=hidden.device) if feat is None else feat
+    top2 = torch.empty(n, 2, dtype=torch.int32, device=hidden.device) if top2 is None else top2
+    row_flags = (torch.empty(n, dtype=torch.int32, device=hidden.device) if row_flags is None
+                 else row_flags)
     n_req = 0 if offsets is None else offsets.numel() - 1
+    _dev(call, dev, "chosen", chosen, _I32_T, n)
+    _dev(call, dev, "offsets", offsets, _I64_T, optional=True)
+    _dev(call, dev, "feat", feat, _F32_T, n * PR_NFEAT)
+    _dev(call, dev, "top2", top2, _I32_T, 2 * n)
+    _dev(call, dev, "row_flags", row_flags, _FLAG_T, n)
     _check(_lib.pr_lmhead_features(ctx, _ptr(hidden), _ptr(weight), n, d, V, _ptr(chosen),
                                    int(topk), _ptr(offsets), n_req, _ptr(feat), _ptr(top2),
                                    _ptr(row_flags), _stream(stream)), "pr_lmhead_features")
@@ -375,7 +524,19 @@ def pr_lmhead_decode_step(ctx, hidden, weight, slot, chosen, eos, w, b: float, t
         raise TypeError("hidden and weight must be bfloat16")
     if not (hidden.is_contiguous() and weight.is_contiguous()) or hidden.size(1) != weight.size(1):
         raise ValueError("hidden [n][d] and weight [V][d] must be contiguous with the same d")
+    call = "pr_lmhead_decode_step"
+    dev = _ctx_device(ctx)
+    _dev(call, dev, "hidden", hidden)
+    _dev(call, dev, "weight", weight)
     n, d = hidden.shape
+    _dev(call, dev, "slot", slot, _I32_T, n)
+    _dev(call, dev, "chosen", chosen, _I32_T, n)
+    _dev(call, dev, "eos", eos, _U8_T, n)
+    _dev(call, dev, "w", w, _F32_T, PR_NAGG)
+    _dev(call, dev, "score_out", score_out, _F32_T)
+    _dev(call, dev, "ship_out", ship_out, _U8_T)
+    _dev(call, dev, "slot_flags", slot_flags, _FLAG_T)
+    _dev(call, dev, "agg_out", agg_out, _F32_T, optional=True)
     _check(_lib.pr_lmhead_decode_step(ctx, _ptr(hidden), _ptr(weight), n, d, weight.size(0),
                                       _ptr(slot), _ptr(chosen), _ptr(eos), _ptr(w), float(b),
                                       float(tau), _ptr(score_out), _ptr(ship_out),

@@ -90,6 +90,9 @@ struct Args {
   const uint8_t* eos;
   float* acc;
   int32_t n_slots;
+  // route, whole batch per call: offsets[n_req] must equal n_rows, else the
+  // last request is reported as inconsistent (rows past it have no request)
+  int32_t whole;
   uint32_t* ctx_flags;
 };
 

@@ -121,6 +121,14 @@ __device__ __forceinline__ int32_t find_request(const int64_t* off, int32_t n_re
   return (a <= gr && gr < c) ? (int32_t)lo : -1;
 }
 
+// Route mode: whether request r's rows [lo, hi) are inconsistent with the
+// batch.  A whole-batch call also needs the last request to end at the last row.
+__device__ __forceinline__ bool route_bad_request(const Args& a, int64_t r, int64_t lo,
+                                                  int64_t hi) {
+  return lo < 0 || hi < lo || hi > a.max_rows ||
+         (a.whole && r == (int64_t)a.n_req - 1 && hi != a.max_rows);
+}
+
 // Route mode: the results of empty requests touching this launch's row range
 // and of requests whose offsets are inconsistent (requests start, start +
 // stride, ...).  Written by every launch; idempotent.
@@ -128,7 +136,7 @@ __device__ __forceinline__ void route_special_requests(const Args& a, int64_t st
                                                        int64_t stride) {
   for (int64_t r = start; r < a.n_req; r += stride) {
     const int64_t lo = a.offsets[r], hi = a.offsets[r + 1];
-    if (lo < 0 || hi < lo || hi > a.max_rows) {
+    if (route_bad_request(a, r, lo, hi)) {
       write_special(r, NAN, FLAG_BAD_OFFSETS, a.agg, a.score, a.ship, a.req_flags);
       atomicOr(a.ctx_flags, FLAG_BAD_OFFSETS);
     } else if (lo == hi && lo >= a.row_base && lo <= a.row_base + a.n_rows) {
@@ -322,7 +330,7 @@ __device__ __forceinline__ void row_finish(const Args& a, int64_t row, float m, 
     const int64_t gr = a.row_base + row;
     const int32_t r = pre.r;
     const int64_t lo = pre.lo, hi = pre.hi;
-    if (r < 0 || lo < 0 || hi > a.max_rows) {
+    if (r < 0 || route_bad_request(a, r, lo, hi)) {
       if (lane == 0) atomicOr(a.ctx_flags, FLAG_BAD_OFFSETS);
       return;
     }

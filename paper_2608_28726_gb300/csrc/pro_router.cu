@@ -501,6 +501,7 @@ pr_status pr_route_noalloc(const void* logits, pr_dtype dt, int64_t n_rows, int6
   a.req_flags = req_flags;
   a.agg = agg;
   a.ctx_flags = reinterpret_cast<uint32_t*>(d->scratch + NA_OFF_FLAGS);
+  a.whole = 1;  // no flag word the caller can read: report short offsets in the last request
 
   // CTAs per row (the cluster kernel only; no persistent-kernel set-up here):
   // double C, up to MAXC, while the batch's CTAs stay under two waves of

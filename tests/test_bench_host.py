@@ -74,3 +74,40 @@ def test_quantile_bytes_count_the_weights_of_the_oracle_mlp():
     n_rows, n_req = 1000, 7
     assert bench.qnt_bytes(n_rows, n_req) == (32 * n_rows + 8 * (n_req + 1) + 4 * oq.n_params()
                                               + (4 + 1 + 4) * n_req)
+
+
+def _oracle_stub(n=3, tau=0.5):
+    rng = np.random.Generator(np.random.PCG64(7))
+    agg = rng.normal(size=(n, 11))
+    score = 1.0 / (1.0 + np.exp(-rng.normal(size=n)))
+    return {"agg": agg, "score": score, "ship": (score >= tau).astype(np.uint8),
+            "req_flags": np.zeros(n, np.uint32)}
+
+
+def test_parity_bar_and_value_gate():
+    """A stubbed oracle result: outputs equal to it pass; a score off by more
+    than 1e-5 + 1e-4 |oracle|, a flipped ship bit outside the 1e-6 band or a
+    flag bit fails, and a failing record prints no value."""
+    o = _oracle_stub()
+    g = {k: v.copy() for k, v in o.items()}
+    assert bench.parity_ok(g["agg"], g["score"].astype(np.float32), g["ship"], g["req_flags"],
+                           o, 0.5)
+    bad = g["score"].copy()
+    bad[1] += 2e-5 + 1e-4 * abs(bad[1])
+    assert not bench.parity_ok(g["agg"], bad, g["ship"], g["req_flags"], o, 0.5)
+    ship = g["ship"].copy()
+    ship[0] ^= 1
+    assert not bench.parity_ok(g["agg"], g["score"], ship, g["req_flags"], o, 0.5)
+    fl = g["req_flags"].copy()
+    fl[2] = 1
+    assert not bench.parity_ok(g["agg"], g["score"], g["ship"], fl, o, 0.5)
+    # a score within 1e-6 of tau may go either way
+    o2 = _oracle_stub()
+    o2["score"][0] = 0.5 + 5e-7
+    o2["ship"][0] = 1
+    assert bench.parity_ok(o2["agg"], o2["score"], np.array([0, *o2["ship"][1:]]),
+                           o2["req_flags"], o2, 0.5)
+    rec = bench.gate_on_parity({"value": 123.0, "parity": {"ok": False}})
+    assert rec["value"] is None and "parity" in rec["value_withheld"]
+    rec = bench.gate_on_parity({"value": 123.0, "parity": {"ok": True}})
+    assert rec["value"] == 123.0 and "value_withheld" not in rec

@@ -468,6 +468,48 @@ def test_decode_bad_slot_flagged(ctx):
     B.pr_ctx_reset(ctx)
 
 
+def test_last_error_reads_the_flag_word_after_the_device_finishes(ctx):
+    """pr_last_error waits for all work on the context's device, not one
+    stream: a flagged decode step queued on a side stream (never synchronised
+    by the test) shows up in its answer.  The word is left as it is, so a
+    second read gives the same bits, until pr_ctx_flags clears it."""
+    B.pr_ctx_reset(ctx)
+    B.pr_ctx_flags(ctx, clear=True)
+    assert B.pr_last_error(ctx) == 0
+    side = torch.cuda.Stream()
+    x, ch = random_rows(3, 5000, torch.bfloat16, seed=4)
+    slot = torch.tensor([0, 4096, 1], dtype=torch.int32, device="cuda")
+    eos = torch.zeros(3, dtype=torch.uint8, device="cuda")
+    out = torch.zeros(1024, device="cuda")
+    ship = torch.zeros(1024, dtype=torch.uint8, device="cuda")
+    fl = torch.zeros(1024, dtype=torch.int32, device="cuda")
+    torch.cuda.synchronize()
+    with torch.cuda.stream(side):
+        # a long chain of work first, so the flagged step is still queued when
+        # the host asks
+        big = torch.randn(4096, 4096, device="cuda")
+        for _ in range(8):
+            big = big @ big
+            big /= big.norm()
+        B.pr_decode_step(ctx, x, slot, ch, eos, torch.zeros(11, device="cuda"), 0.0, 0.5, out,
+                         ship, fl, stream=side)
+    word = B.pr_last_error(ctx)
+    assert word == B.PR_FLAG_BAD_SLOT, word
+    assert B.pr_last_error(ctx) == word  # read only
+    assert B.pr_ctx_flags(ctx, clear=True) == word
+    assert B.pr_last_error(ctx) == 0
+    # a route call whose request reaches past the context's rows raises
+    # PR_FLAG_BAD_OFFSETS in the same word
+    off = torch.tensor([0, 2, (1 << 16) + 5], dtype=torch.int64, device="cuda")
+    x2, ch2 = random_rows(2, 300, torch.float32, seed=5)
+    score, sh, rf, _ = B.pr_route(ctx, x2, ch2, off, torch.zeros(11, device="cuda"), 0.0, 0.5)
+    assert B.pr_last_error(ctx) == B.PR_FLAG_BAD_OFFSETS
+    assert rf[1].item() == B.PR_FLAG_BAD_OFFSETS and np.isnan(score[1].item())
+    assert rf[0].item() == 0 and score[0].item() == 0.5
+    B.pr_ctx_flags(ctx, clear=True)
+    B.pr_ctx_reset(ctx)
+
+
 def test_overlap_option_changes_nothing_but_timing(ctx):
     """With PR_OPT_OVERLAP a call may start while the previous one finishes;
     back-to-back route calls and decode steps give bit-identical results."""
