@@ -127,6 +127,17 @@ def _ctx_device(ctx) -> int:
 
 def _dev(call: str, dev: int, name: str, t, dtypes=None, numel: int | None = None,
          optional: bool = False, contiguous: bool = True):
+    # the common case in one expression (this runs on every call of a hot loop)
+    try:
+        if (t.is_cuda and t.get_device() == dev and (dtypes is None or t.dtype in dtypes)
+                and (not contiguous or t.is_contiguous()) and (numel is None or t.numel() >= numel)):
+            return
+    except AttributeError:
+        pass
+    _dev_refuse(call, dev, name, t, dtypes, numel, optional, contiguous)
+
+
+def _dev_refuse(call, dev, name, t, dtypes, numel, optional, contiguous):
     if t is None:
         if optional:
             return
@@ -168,7 +179,7 @@ def _ptr(t):
     if t is None:
         return None
     if isinstance(t, torch.Tensor):
-        return ctypes.c_void_p(t.data_ptr())
+        return t.data_ptr()  # an int: ctypes converts it for a c_void_p argument
     if isinstance(t, np.ndarray):
         return t.ctypes.data_as(ctypes.c_void_p)
     raise TypeError(type(t))
