@@ -41,6 +41,7 @@ constexpr int NT = 256;            // threads per CTA
 constexpr int NWARP = NT / 32;     // warps per CTA
 constexpr int UNR = 4;             // 16-byte groups per thread per tile
 constexpr int TILE = NT * UNR;     // groups per CTA tile
+constexpr int PF_TILES = 2;        // one CTA per row: tiles prefetched into L2 ahead of the loads
 constexpr int MAX_SLOTS = 24;      // stored tile maxima per thread (tiles are merged beyond)
 constexpr int CCAP = 256;          // candidate super-groups
 constexpr int ECAP = 512;          // candidate elements
@@ -110,6 +111,11 @@ __device__ __forceinline__ uint4 ld_stream(const void* p) {
                : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
                : "l"(p));
   return r;
+}
+
+// bulk prefetch of [p, p + bytes) into L2 (16-byte aligned, a multiple of 16 bytes)
+__device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
 }
 
 __device__ __forceinline__ uint32_t hmax2(uint32_t a, uint32_t b) {

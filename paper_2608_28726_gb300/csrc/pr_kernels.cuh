@@ -463,6 +463,20 @@ __global__ void __launch_bounds__(NT) verify_rows(const Args a) {
     auto load = [&](int32_t gi) -> uint4 {
       return ALIGNED ? ld_stream(vp + g0 + gi) : Tr::load_elems(rowp, (int64_t)(g0 + gi));
     };
+    // one CTA per row: one thread keeps the tiles PF_TILES ahead on their way
+    // into L2 (bulk prefetches need no registers, so the CTA has more bytes in
+    // flight than its two register tiles; measured on 256-row decode steps:
+    // 24.9 us isolated and 11.2 us in a CUDA graph against 27.0 and 12.8 us
+    // without; with clusters, whose CTAs already keep HBM busy, it slowed
+    // the step)
+    auto prefetch_tile = [&](int32_t t) {
+      if (PF_TILES > 0 && ALIGNED && C == 1 && tid == 0 && t < ntiles) {
+        const int32_t gs = t * TILE;
+        prefetch_l2(vp + g0 + gs, (uint32_t)min(TILE, ng - gs) * 16u);
+      }
+    };
+#pragma unroll
+    for (int32_t p = 1; p <= PF_TILES; ++p) prefetch_tile(p);
     uint4 cur[UNR], nxt[UNR];
     if (nfull > 0) {
 #pragma unroll
@@ -473,6 +487,7 @@ __global__ void __launch_bounds__(NT) verify_rows(const Args a) {
     }
     for (int32_t t = 0; t < ntiles; ++t) {
       const int32_t nb = (t + 1) * TILE;
+      prefetch_tile(t + 1 + PF_TILES);
       if (t + 1 < nfull) {
 #pragma unroll
         for (int k = 0; k < UNR; ++k) nxt[k] = load(nb + k * NT + tid);
