@@ -83,12 +83,13 @@ pr_status ws_setup(pr_ctx* c, pr_dtype dt, int mode, bool aligned, int* bps) {
 // Launch shape of a batch: CTAs per row (C) and whether the persistent
 // kernel runs it.
 //  * the forced option: split 1 is the persistent kernel, 2 / 4 / 8 clusters;
-//  * a batch with at least one row per SM whose one-CTA-per-row launch fills
-//    at most half the resident CTA slots (a decode step of 256 rows): one CTA
-//    per row, without a cluster.  Two such launches fit on the GPU at once, so
-//    back-to-back calls overlap one launch's per-row selection with the next
-//    one's stream (measured on 256 x 151,936 bf16: 12.8 us per step in a CUDA
-//    graph against 15.6 us with two-CTA clusters, which fill 84% of the slots);
+//  * a batch with at least one row per SM that fits one wave of resident
+//    CTAs: one CTA per row, without a cluster.  Such a launch leaves room for
+//    the next one, so back-to-back calls overlap one launch's per-row
+//    selection with the next one's stream (measured in CUDA graphs: 256 x
+//    151,936 bf16 decode steps 12.8 us per step against 15.6 us with two-CTA
+//    clusters, which fill 84% of the slots; 354 x 32,000 fp32 batches 12.0 us
+//    against 13.9 us with the persistent kernel);
 //  * fewer rows: the largest split (<= 8) whose CTAs still fit in one wave;
 //  * more rows: the persistent kernel.
 struct LaunchShape {
@@ -100,7 +101,7 @@ LaunchShape choose_launch(pr_ctx* c, pr_dtype dt, int mode, int64_t n_rows) {
   if (c->split == 1) return {1, true};
   if (c->split == 2 || c->split == 4 || c->split == 8) return {c->split, false};
   const int64_t slots = (int64_t)c->num_sms * blocks_per_sm(c, dt, mode);
-  if (n_rows >= c->num_sms && n_rows * 2 <= slots) return {1, false};
+  if (n_rows >= c->num_sms && n_rows <= slots) return {1, false};
   int s = 1;
   while (s < prk::MAXC && n_rows * (s * 2) <= slots) s <<= 1;
   return {s, s == 1};

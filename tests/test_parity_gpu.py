@@ -454,6 +454,50 @@ def test_decode_checkpoint_resume(ctx):
     B.pr_ctx_reset(ctx)
 
 
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+def test_decode_and_route_agree_on_the_same_requests(ctx, dtype):
+    """The incremental mode and the full-response mode on the same requests.
+    Route pools a request's records with a fixed-order lane-strided sum;
+    a decode slot keeps a compensated running sum in step order.  So the
+    minima and the mean position fraction are bit-identical between the
+    modes, and the five means agree within the parity tolerance, with each
+    other and with the oracle; the decisions are equal outside the band
+    around tau.  Both modes run the same launch shape (8 CTAs per row), so
+    each row's features are computed identically."""
+    _set(ctx, split=8)
+    lengths = [1, 2, 7, 33, 64, 129, 300, 1000]
+    x, ch, off, w, b = _batch(lengths, 4097, dtype, seed=77)
+    dw, doff = torch.from_numpy(w).cuda(), torch.from_numpy(off).cuda()
+    n = len(lengths)
+    r_score, r_ship, r_flags, r_agg = B.pr_route(ctx, x, ch, doff, dw, b, 0.5)
+    # decode: request r in slot r, one row per step while it is live
+    B.pr_ctx_reset(ctx)
+    d_score = torch.zeros(1024, device="cuda")
+    d_ship = torch.zeros(1024, dtype=torch.uint8, device="cuda")
+    d_flags = torch.zeros(1024, dtype=torch.int32, device="cuda")
+    d_agg = torch.zeros(1024, 11, device="cuda")
+    for t in range(max(lengths)):
+        live = [r for r in range(n) if lengths[r] > t]
+        rows = torch.tensor([int(off[r]) + t for r in live], dtype=torch.int64, device="cuda")
+        slot = torch.tensor(live, dtype=torch.int32, device="cuda")
+        eos = torch.tensor([1 if lengths[r] == t + 1 else 0 for r in live], dtype=torch.uint8,
+                           device="cuda")
+        B.pr_decode_step(ctx, x.index_select(0, rows), slot, ch.index_select(0, rows).contiguous(),
+                         eos, dw, b, 0.5, d_score, d_ship, d_flags, agg_out=d_agg)
+    torch.cuda.synchronize()
+    ra, da = r_agg.cpu().numpy(), d_agg[:n].cpu().numpy()
+    mins_and_rho = [1, 3, 5, 7, 9, 10]
+    assert np.array_equal(ra[:, mins_and_rho], da[:, mins_and_rho])
+    assert_close(da, ra, "decode vs route agg")
+    assert_close(d_score[:n].cpu().numpy(), r_score.cpu().numpy(), "decode vs route score")
+    assert np.array_equal(d_flags[:n].cpu().numpy(), r_flags.cpu().numpy())
+    o = oracle.route(as_oracle(x), ch.cpu().numpy(), off, w.astype(np.float64), b, 0.5)
+    _check_requests(d_score[:n], d_ship[:n], d_flags[:n], d_agg[:n], o, 0.5, "decode")
+    _check_requests(r_score, r_ship, r_flags, r_agg, o, 0.5, "route")
+    B.pr_ctx_reset(ctx)
+    _set(ctx)
+
+
 def test_decode_bad_slot_flagged(ctx):
     B.pr_ctx_reset(ctx)
     x, ch = random_rows(2, 300, torch.float32, seed=1)
