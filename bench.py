@@ -248,12 +248,14 @@ def measured_peak():
     return 6800.0, "fallback"
 
 
-def timed_repeats(step, K: int, stream, dev, world: int, B, min_s: float = MIN_TIMED_S):
+def timed_repeats(step, K: int, stream, dev, world: int, B, min_s: float | None = None):
     """Time K back-to-back steps with CUDA events on `stream`, a barrier and a
     synchronize on both sides (max over ranks), and repeat that K-step loop
     until at least `min_s` seconds of device time are timed (at least three
     repeats).  Returns (per-repeat ms per step, wall window, launches in all
     timed repeats)."""
+    if min_s is None:
+        min_s = MIN_TIMED_S
     per, total_ms = [], 0.0
     launches = 0
     t_wall0 = time.time()
@@ -468,7 +470,7 @@ def measure_route_config(name, B, dev, stream, K, warm, world, sampler, threads,
     return rec
 
 
-def measure_decode_config(B, dev, stream, K, warm, world, sampler, threads):
+def measure_decode_config(B, dev, stream, K, warm, world, sampler, threads, n_steps: int = 1000):
     """The incremental decode-step workload: 256 live slots for 1,000 steps,
     V = 151,936 bf16, the whole trace resident (77.8 GB); a step is one
     pr_decode_step of 256 rows.  Timed as isolated calls, back-to-back calls
@@ -476,7 +478,7 @@ def measure_decode_config(B, dev, stream, K, warm, world, sampler, threads):
     Parity: every sampled request that finishes inside the trace against the
     oracle on its rows."""
     t_gen = time.time()
-    tr = W.decode_trace()
+    tr = W.decode_trace(n_steps=n_steps)
     wl = tr.as_workload()
     S, T = tr.n_slots, tr.n_steps
     x_all = torch.empty(T * S, wl.vocab, dtype=wl.torch_dtype, device=dev)
@@ -575,15 +577,18 @@ def measure_decode_config(B, dev, stream, K, warm, world, sampler, threads):
     parity = {"requests_checked": len(sample), "rows_checked": rows, "ok": ok,
               "oracle_tokens_per_s": rows / secs if secs > 0 else None}
     bytes_per_step = S * (wl.vocab * 2 + 4 + 4 + 1) + S * 4
-    desc = ("incremental decode-step verify: 256 live slots x 1,000 steps (256,000 rows, "
-            "77.8 GB resident), V=%d bf16 as the full-response rows, lengths U{64..1000}, "
-            "one pr_decode_step of 256 rows per step" % wl.vocab)
-    rec = _route_rec(wl, "decode", desc, "CUDA graph replays (a context reset and the 1,000-step "
-                     "trace per graph)", ms, statistics.median(iso), stream_ms, bytes_per_step, S,
+    desc = ("incremental decode-step verify: 256 live slots x %d steps (%d rows, "
+            "%.1f GB resident), V=%d bf16 as the full-response rows, lengths U{64..1000}, "
+            "one pr_decode_step of 256 rows per step" % (T, T * S, T * S * wl.vocab * 2 / 1e9,
+                                                       wl.vocab))
+    rec = _route_rec(wl, "decode", desc, "CUDA graph replays (a context reset and the %d-step trace per "
+                     "graph)" % T, ms, statistics.median(iso), stream_ms, bytes_per_step, S,
                      world, clocks, launches, T, len(per_g), parity,
                      {"steps_per_graph": T, "kernels_per_graph": nodes, "replays_per_repeat": 1})
     rec["generation_s"] = gen_s
-    rec["l2"] = "a 77.8 GB trace: every step reads new rows from DRAM"
+    rec["l2"] = "a %.1f GB trace: every step reads new rows from DRAM" % (T * S * wl.vocab * 2 / 1e9)
+    if T != 1000:
+        rec["profiling_case"] = "a %d-step trace instead of the 1,000-step one" % T
     B.pr_ctx_destroy(ctx)
     del x_all, ch_all
     torch.cuda.empty_cache()
@@ -665,7 +670,7 @@ def run_gb300(args):
     sampler.start()
     K = args.steps
     warm = max(3, args.warmup)
-    min_s = 0.05 if args.skip_host else MIN_TIMED_S
+    min_s = min(0.05, MIN_TIMED_S) if args.skip_host else MIN_TIMED_S
 
     # (1) isolated launches: one launch at a time (no overlap between steps)
     B.pr_ctx_set_option(ctx, B.PR_OPT_OVERLAP, 0)
@@ -851,7 +856,8 @@ def run_other_workload(args):
     warm = max(3, args.warmup)
     cores = os.cpu_count() or 1
     if args.workload == "decode":
-        rec = measure_decode_config(B, dev, stream, args.steps, warm, world, sampler, cores)
+        rec = measure_decode_config(B, dev, stream, args.steps, warm, world, sampler, cores,
+                                    n_steps=args.decode_steps)
     else:
         rec = measure_route_config(args.workload, B, dev, stream, args.steps, warm, world,
                                    sampler, cores)
@@ -871,6 +877,8 @@ def run_other_workload(args):
             line["graph"] = rec["graph"]
         if "value_withheld" in rec:
             line["value_withheld"] = rec["value_withheld"]
+        if "profiling_case" in rec:
+            line["profiling_case"] = rec["profiling_case"]
         print(json.dumps(line))
     return 0
 
@@ -1606,6 +1614,10 @@ def main():
                          "object (c1 tiny, c3 decode, c4 ragged, c5 wide; 'none' for none)")
     ap.add_argument("--requests", type=int, default=0,
                     help="profiling only: the first N requests of the workload")
+    ap.add_argument("--timed-seconds", type=float, default=MIN_TIMED_S,
+                    help="device time each timed measurement repeats its K-step loop for")
+    ap.add_argument("--decode-steps", type=int, default=1000,
+                    help="profiling only: the decode workload's first N steps (resident trace)")
     ap.add_argument("--skip-host", action="store_true",
                     help="profiling only: skip the host-memory and oracle legs")
     ap.add_argument("--head-oracle-sample", type=int, default=0, help=argparse.SUPPRESS)
@@ -1616,6 +1628,7 @@ def main():
     ap.add_argument("--lm-rows", type=int, default=0,
                     help="lmhead workload: the first N hidden states only, as one request")
     args = ap.parse_args()
+    globals()["MIN_TIMED_S"] = args.timed_seconds
     if args.lm_oracle_child:
         return lm_oracle_child(args.lm_oracle_child)
     if args.qnt_oracle_child:
