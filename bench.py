@@ -1318,9 +1318,12 @@ def qnt_bytes(n_rows: int, n_req: int) -> int:
     return 32 * n_rows + 8 * (n_req + 1) + 4 * 6081 + 9 * n_req
 
 
-def qnt_oracle_child():
+Q_LAYOUTS = {"ragged": "ragged", "full": "full"}  # request layout -> workload it is taken from
+
+
+def qnt_oracle_child(layout: str = "ragged"):
     from oracle import quantile as oq
-    wl = W.make("ragged")
+    wl = W.make(Q_LAYOUTS[layout])
     feat, offsets = W.head_features(wl.lengths, seed=4001)
     w = W.qmlp_weights()
     t0 = time.perf_counter()
@@ -1333,7 +1336,8 @@ def qnt_oracle_child():
 
 def run_quantile_workload(args):
     """The quantile-summary + MLP aggregator on the ragged request layout
-    (1,024 requests, lognormal lengths, 181,659 rows)."""
+    (1,024 requests, lognormal lengths, 181,659 rows) or, with --q-layout
+    full, the full-response layout (64 requests, T ~ U{32..256}, 8,847 rows)."""
     rank, world, local = dist_env()
     if world > 1:
         import torch.distributed as dist
@@ -1343,7 +1347,7 @@ def run_quantile_workload(args):
     from paper_2608_28726_gb300 import build as prbuild
     prbuild.build()
     from paper_2608_28726_gb300 import binding as B
-    wl = W.make("ragged")
+    wl = W.make(Q_LAYOUTS[args.q_layout])
     feat_h, offsets = W.head_features(wl.lengths, seed=4001)
     w_h = W.qmlp_weights()
     feat, off = torch.from_numpy(feat_h).to(dev), torch.from_numpy(offsets).to(dev)
@@ -1383,6 +1387,25 @@ def run_quantile_workload(args):
     ms = reduce_max(sum(a.elapsed_time(b) for a, b in ev), world, dev) / K
     clocks = sampler.summary(t_wall0, t_wall1)
     sampler.stop()
+    # back-to-back launches without the flush (the features stay in L2, as
+    # they would right after the verifier wrote them): about the kernel's own
+    # duration per launch
+    b2b, _, _ = timed_repeats(step, K, stream, dev, world, B, min_s=0.2)
+    b2b_ms = statistics.median(b2b)
+    # the same launches replayed from a CUDA graph (no host cost between them)
+    gr = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(gr, capture_error_mode="thread_local"):
+        gs = torch.cuda.current_stream(dev)
+        for _ in range(20):
+            B.pr_quantile_score(ctx, feat, off, w, wl.tau, score=score, ship=ship,
+                                req_flags=rflags, want_summary=False, stream=gs)
+    for _ in range(3):
+        gr.replay()
+    torch.cuda.synchronize(dev)
+    g_per, _, _ = timed_repeats(gr.replay, 10, torch.cuda.current_stream(dev), dev, world, B,
+                                min_s=0.2)
+    graph_ms = statistics.median(g_per) / 20
+    del gr
 
     hf, ho = torch.from_numpy(feat_h).pin_memory(), torch.from_numpy(offsets).pin_memory()
     hs = torch.empty(n_req).pin_memory()
@@ -1414,7 +1437,8 @@ def run_quantile_workload(args):
     peak = float(json.load(open(peaks_file))["hbm_gbs"]) if os.path.exists(peaks_file) else 6800.0
     achieved = qbytes / (ms / 1e3) / 1e9
     if rank == 0:
-        out = subprocess.run([sys.executable, os.path.abspath(__file__), "--qnt-oracle-child"],
+        out = subprocess.run([sys.executable, os.path.abspath(__file__), "--qnt-oracle-child",
+                              "--q-layout", args.q_layout],
                              env=dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1",
                                       MKL_NUM_THREADS="1"),
                              capture_output=True, text=True, check=True)
@@ -1424,13 +1448,16 @@ def run_quantile_workload(args):
         ok = bool(np.all(np.abs(g - so) <= 1e-5) and
                   np.all((ship.cpu().numpy() == po) | (np.abs(so - wl.tau) < 1e-6)))
         print(json.dumps({
-            "metric": "scored tokens/sec (quantile summary + MLP, 1,024-request ragged layout)",
+            "metric": "scored tokens/sec (quantile summary + MLP, %s)" % (
+                "1,024-request ragged layout" if args.q_layout == "ragged" else
+                "64-request full-response layout"),
             "value": n_rows * world / (ms / 1e3), "unit": UNIT, "n_gpus": world, "steps": K,
             "warmup": max(3, args.warmup), "ms_per_step": ms, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-            "config": {"workload": "quantile summary + MLP: %d requests, lognormal lengths "
-                                   "(median 128, 8..1,024; %d rows), seeded feature records and "
-                                   "weights (6,081 floats)" % (n_req, n_rows),
+            "config": {"workload": "quantile summary + MLP: %d requests, %s (%d rows), seeded "
+                                   "feature records and weights (6,081 floats)" % (
+                                       n_req, "lognormal lengths (median 128, 8..1,024)"
+                                       if args.q_layout == "ragged" else "T~U{32..256}", n_rows),
                        "l2": "256 MB written between timed steps (flush)"},
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak,
                          "unit": "GB/s", "frac": achieved / peak,
@@ -1440,7 +1467,9 @@ def run_quantile_workload(args):
                          "note": "latency-bound: one CTA per request, 2.25 waves; the "
                                  "per-request chains (loads, rank or sort, MLP), not bandwidth, "
                                  "set the time",
-                         "algorithmic_bytes_per_launch": qbytes, "avg_launch_ms": ms},
+                         "algorithmic_bytes_per_launch": qbytes, "avg_launch_ms": ms,
+                         "back_to_back_launch_ms": b2b_ms,
+                         "graph_launch_ms": graph_ms},
             "cpu_baseline": {"value": n_rows / d["seconds"], "unit": UNIT, "cores": 1,
                              "kind": "oracle",
                              "sample": "the whole %d-row workload, float64 numpy oracle" % n_rows},
@@ -1624,6 +1653,8 @@ def main():
     ap.add_argument("--head-layers", type=int, default=2, help=argparse.SUPPRESS)
     ap.add_argument("--sel-oracle-child", type=int, default=0, help=argparse.SUPPRESS)
     ap.add_argument("--qnt-oracle-child", action="store_true", help=argparse.SUPPRESS)
+    ap.add_argument("--q-layout", default="ragged", choices=sorted(Q_LAYOUTS),
+                    help="quantile workload: the ragged (default) or full-response request layout")
     ap.add_argument("--lm-oracle-child", type=int, default=0, help=argparse.SUPPRESS)
     ap.add_argument("--lm-rows", type=int, default=0,
                     help="lmhead workload: the first N hidden states only, as one request")
@@ -1632,7 +1663,7 @@ def main():
     if args.lm_oracle_child:
         return lm_oracle_child(args.lm_oracle_child)
     if args.qnt_oracle_child:
-        return qnt_oracle_child()
+        return qnt_oracle_child(args.q_layout)
     if args.head_oracle_sample:
         return head_oracle_child(args.head_oracle_sample, args.head_layers)
     if args.sel_oracle_child:

@@ -405,9 +405,11 @@ pr_status pr_selftest_wait(pr_ctx* ctx, int64_t limit_ns, int32_t* completed);
  *   summary    device float [n_req][PR_QMLP_SUMMARY] or NULL: the quantiles,
  *              feature-major (written for requests that are scored)
  *   score, ship, req_flags   device [n_req]                     (outputs)
- * One launch, one CTA per request; requests of up to 2,048 rows are sorted in
- * shared memory, longer ones use radix selection over global memory (exact,
- * slower).  fp32, fixed-order sums.  n_rows < 2^31.
+ * One launch, one CTA per request; requests of up to 256 rows are sorted in
+ * registers (one warp per feature), up to 2,048 rows in shared memory, longer
+ * ones use radix selection over global memory (exact, slower).  fp32,
+ * fixed-order sums.  n_rows < 2^31; feat must be 16-byte aligned
+ * (PR_ERR_INVALID_ARG otherwise).
  */
 pr_status pr_quantile_score(pr_ctx* ctx, const float* feat, const uint32_t* row_flags,
                             int64_t n_rows, const int64_t* offsets, int32_t n_req, const float* w,

@@ -5,18 +5,18 @@
 // interpolation between order statistics), a 28-number summary, then a
 // 28 -> 64 -> 64 -> 1 ReLU MLP and a sigmoid.
 //
-// One CTA per request.  Up to Q_SMALL rows each thread takes one row and
-// computes the exact stable rank of its four keys (order-preserving 32-bit
-// keys, one 16-byte word per row in shared memory, read by all threads at
-// once): the count of smaller keys plus equal keys of earlier rows; the row
-// whose rank is a needed index hands its value over.  Up to Q_CAP rows the
+// One CTA per request.  Up to Q_SMALL rows two warps per feature sort its
+// column's order-preserving 32-bit keys (padded to 256) in registers, four
+// per lane (a bitonic network inside the lanes, across them by shfl.xor, and
+// one stage between the two warps).  Up to Q_CAP rows the
 // four columns are bitonic-sorted together: up to 1,024 rows each thread
 // holds a run of keys in registers (register and warp-shuffle stages, one
 // stage through shared memory), above that in shared memory; longer requests
 // find each needed order statistic by radix selection (four 8-bit passes of
 // shared histograms over the request's rows in global memory).  All three
 // give the exact order statistics.  The MLP runs in the same CTA with
-// fixed-order sums.
+// fixed-order sums (four threads per hidden unit, quarters added in a fixed
+// butterfly).
 #pragma once
 
 #include "pr_device.cuh"
@@ -45,6 +45,9 @@ constexpr int QS_W1 = 0, QS_B1 = Q_H * (Q_NS + 1), QS_W2 = QS_B1 + Q_H,
               QS_SIZE = QS_B3 + 1;
 constexpr int QW_PER_T = (QW_SIZE + Q_NT - 1) / Q_NT;  // weights each thread fetches
 static_assert(QS_SIZE <= 4 * Q_CAP, "the weights fit in the key buffer");
+static_assert(4 * Q_SMALL + QS_SIZE <= 4 * Q_CAP, "beside the keys of a short request too");
+static_assert(Q_SMALL == 256 && Q_NT == 256, "two warps per column sort 256 keys");
+static_assert(Q_NT == 4 * Q_H && Q_NS % 4 == 0 && Q_H % 4 == 0, "four threads per hidden unit");
 
 // shared-memory position of flat weight g
 __device__ __forceinline__ int q_wpos(int g) {
@@ -133,6 +136,51 @@ __device__ uint32_t q_select(const float* __restrict__ feat, int64_t lo, int T, 
   return prefix;
 }
 
+// Ascending bitonic sort of the 256 keys of one column held by two warps:
+// lane l of warp `half` holds keys c = 128 half + 4 l .. + 3 in v.  Stages of
+// partner distance below 4 run inside the lane's registers, 4..64 between
+// lanes (shfl.xor), 128 between the two warps through xbuf (128 keys per
+// warp) and the named barrier `bar` of the pair's 64 threads.
+__device__ __forceinline__ void q_sort256_pair(uint32_t (&v)[4], int half, int lane,
+                                               uint32_t* xbuf, int bar) {
+#pragma unroll
+  for (int k = 2; k <= 256; k <<= 1) {
+    if (k == 256) {  // partner distance 128: the other warp
+#pragma unroll
+      for (int e = 0; e < 4; ++e) xbuf[half * 128 + lane * 4 + e] = v[e];
+      asm volatile("bar.sync %0, 64;" ::"r"(bar) : "memory");
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const uint32_t p = xbuf[(half ^ 1) * 128 + lane * 4 + e];
+        v[e] = half == 0 ? min(v[e], p) : max(v[e], p);  // one ascending block
+      }
+    }
+#pragma unroll
+    for (int j = (k >> 1) < 64 ? (k >> 1) : 64; j >= 4; j >>= 1) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int c = half * 128 + lane * 4 + e;
+        const uint32_t p = __shfl_xor_sync(FULL, v[e], j >> 2);
+        const bool keep_min = ((c & j) == 0) == ((c & k) == 0);
+        v[e] = keep_min ? min(v[e], p) : max(v[e], p);
+      }
+    }
+#pragma unroll
+    for (int j = (k >> 1) < 2 ? (k >> 1) : 2; j >= 1; j >>= 1) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        if ((e & j) == 0) {
+          const uint32_t x = v[e], y = v[e + j];
+          const bool up = ((half * 128 + lane * 4 + e) & k) == 0;
+          const uint32_t lo = min(x, y), hi = max(x, y);
+          v[e] = up ? lo : hi;
+          v[e + j] = up ? hi : lo;
+        }
+      }
+    }
+  }
+}
+
 // Ascending bitonic sort of the four columns col f = qs + (f << ln2) of n2 =
 // 2^ln2 keys each, n2 = 64 E (512 or 1,024), by the whole CTA: thread t
 // holds the E consecutive keys c0 .. c0 + E - 1 of one column (two warps per
@@ -199,6 +247,7 @@ __global__ void __launch_bounds__(Q_NT, 3) qmlp_requests(const QArgs a) {
   __shared__ float qv[Q_NS];
   __shared__ float h1[Q_H], h2[Q_H];
   __shared__ uint32_t hist[256], bcast[2], wfl[Q_NT / 32];
+  __shared__ uint32_t qx[4][Q_SMALL];  // exchange between the two warps of a column
   __shared__ float zpart[2];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int64_t r = blockIdx.x;
@@ -229,87 +278,72 @@ __global__ void __launch_bounds__(Q_NT, 3) qmlp_requests(const QArgs a) {
     }
     return;
   }
+  // the rows' flags: read now, decided after the order statistics (a flagged
+  // request is rare, and its loads then overlap the key loads)
   uint32_t fl = 0;
   if (a.row_flags)
     for (int t = tid; t < T; t += Q_NT) fl |= a.row_flags[lo + t];
   fl = __reduce_or_sync(FULL, fl);
   if (lane == 0) wfl[warp] = fl;
-  __syncthreads();
-  fl = 0;
-#pragma unroll
-  for (int w2 = 0; w2 < Q_NT / 32; ++w2) fl |= wfl[w2];
-  if (fl & (FLAG_NONFINITE | FLAG_BAD_CHOSEN)) {
-    if (tid == 0) {
-      a.score[r] = NAN;
-      a.ship[r] = 0;
-      a.req_flags[r] = fl;
-    }
-    return;
-  }
 
+  float* W = reinterpret_cast<float*>(qs);  // the MLP's weights in shared memory
   if (T <= Q_SMALL) {
-    uint4* q4 = reinterpret_cast<uint4*>(qs);  // row t: the keys of l, m, h, rho
-    __shared__ float sval[Q_NS];
-    uint4 mine = make_uint4(0u, 0u, 0u, 0u);
-    if (tid < T) {
-      const float* rec = a.feat + (lo + tid) * NFEAT;
-      mine = make_uint4(q_key(rec[q_slot(0)]), q_key(rec[q_slot(1)]), q_key(rec[q_slot(2)]),
-                        q_key(rec[q_slot(3)]));
-      q4[tid] = mine;
+    // the weights go beside the keys at once (their loads were issued at the
+    // top), so that staging them is off the request's critical path
+    W = reinterpret_cast<float*>(qs + 4 * Q_SMALL);
+#pragma unroll
+    for (int i = 0; i < QW_PER_T; ++i) {
+      const int g = tid + i * Q_NT;
+      if (g < QW_SIZE) W[q_wpos(g)] = wr[i];
     }
-    __syncthreads();
-    if (tid < T) {
-      // stable rank of each of the row's four keys
-      uint32_t r0 = 0, r1 = 0, r2 = 0, r3 = 0;
-      int j = 0;
-      for (; j < tid; ++j) {  // earlier rows: smaller or equal
-        const uint4 o = q4[j];
-        r0 += o.x <= mine.x;
-        r1 += o.y <= mine.y;
-        r2 += o.z <= mine.z;
-        r3 += o.w <= mine.w;
+    // two warps per feature column: its keys (padded with the largest key to
+    // 256) sorted in registers, then stored in order for the interpolation
+    {
+      const int f = warp >> 1, half = warp & 1;
+      const int slot = q_slot(f);
+      uint32_t v[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int t = half * 128 + lane * 4 + e;
+        v[e] = t < T ? q_key(__ldg(a.feat + (lo + t) * NFEAT + slot)) : 0xffffffffu;
       }
-      for (++j; j < T; ++j) {  // later rows: smaller only
-        const uint4 o = q4[j];
-        r0 += o.x < mine.x;
-        r1 += o.y < mine.y;
-        r2 += o.z < mine.z;
-        r3 += o.w < mine.w;
-      }
-      // hand over the needed order statistics (the lower one of a level to
-      // sval, the upper neighbour of an interpolated level to qv)
-      auto give = [&](int f, uint32_t r, uint32_t key) {
-        for (int lv = 0; lv < Q_NQ; ++lv) {
-          const uint32_t num = (uint32_t)q_level_a[lv] * (uint32_t)(T - 1);
-          const uint32_t b = (uint32_t)q_level_b[lv];
-          const uint32_t lo_i = num / b;
-          if (r == lo_i) sval[f * Q_NQ + lv] = q_unkey(key);
-          if (num != lo_i * b && r == lo_i + 1) qv[f * Q_NQ + lv] = q_unkey(key);
-        }
-      };
-      give(0, r0, mine.x);
-      give(1, r1, mine.y);
-      give(2, r2, mine.z);
-      give(3, r3, mine.w);
+      q_sort256_pair(v, half, lane, qx[f], 1 + f);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) qs[f * Q_SMALL + half * 128 + lane * 4 + e] = v[e];
     }
     __syncthreads();
     if (tid < Q_NS) {
       const int f = tid / Q_NQ, lv = tid - f * Q_NQ;
-      const int64_t num = (int64_t)q_level_a[lv] * (T - 1);
-      const int b = q_level_b[lv];
-      const int lo_i = (int)(num / b), rem = (int)(num - (int64_t)lo_i * b);
-      const float xl = sval[tid];
+      const uint32_t num = (uint32_t)q_level_a[lv] * (uint32_t)(T - 1);  // T <= 256
+      const uint32_t b = (uint32_t)q_level_b[lv];
+      const uint32_t lo_i = num / b, rem = num - lo_i * b;
+      const uint32_t* col = qs + f * Q_SMALL;
+      const float xl = q_unkey(col[lo_i]);
       float q = xl;
-      if (rem) q = xl + ((float)rem / (float)b) * (qv[tid] - xl);
+      if (rem) q = xl + ((float)rem / (float)b) * (q_unkey(col[lo_i + 1]) - xl);
       qv[tid] = q;
     }
   } else if (T <= Q_CAP) {
     int ln2 = 9;  // n2 = 2^ln2 >= T, at least 512
     while ((1 << ln2) < T) ++ln2;
     const int n2 = 1 << ln2;
-    for (int i = tid; i < 4 * n2; i += Q_NT) {
-      const int f = i >> ln2, t = i & (n2 - 1);
-      qs[i] = t < T ? q_key(a.feat[(lo + t) * NFEAT + q_slot(f)]) : 0xffffffffu;
+    // each thread reads whole records (two 16-byte loads give the four
+    // features), several rows in flight at once
+#pragma unroll 4
+    for (int t = tid; t < n2; t += Q_NT) {
+      uint32_t k0 = 0xffffffffu, k1 = 0xffffffffu, k2 = 0xffffffffu, k3 = 0xffffffffu;
+      if (t < T) {
+        const float4* rec = reinterpret_cast<const float4*>(a.feat + (lo + t) * NFEAT);
+        const float4 r0 = __ldg(rec), r1 = __ldg(rec + 1);
+        k0 = q_key(r0.x);  // l
+        k1 = q_key(r0.y);  // m
+        k2 = q_key(r1.x);  // h
+        k3 = q_key(r1.y);  // rho
+      }
+      qs[t] = k0;
+      qs[n2 + t] = k1;
+      qs[2 * n2 + t] = k2;
+      qs[3 * n2 + t] = k3;
     }
     __syncthreads();
     if (ln2 == 9) {
@@ -369,24 +403,48 @@ __global__ void __launch_bounds__(Q_NT, 3) qmlp_requests(const QArgs a) {
   }
   __syncthreads();
 
-  // MLP 28 -> 64 -> 64 -> 1 (sums in input order), weights from shared memory
-  float* W = reinterpret_cast<float*>(qs);
+  fl = 0;
 #pragma unroll
-  for (int i = 0; i < QW_PER_T; ++i) {
-    const int g = tid + i * Q_NT;
-    if (g < QW_SIZE) W[q_wpos(g)] = wr[i];
+  for (int w2 = 0; w2 < Q_NT / 32; ++w2) fl |= wfl[w2];
+  if (fl & (FLAG_NONFINITE | FLAG_BAD_CHOSEN)) {
+    if (tid == 0) {
+      a.score[r] = NAN;
+      a.ship[r] = 0;
+      a.req_flags[r] = fl;
+    }
+    return;
+  }
+
+  // MLP 28 -> 64 -> 64 -> 1, weights from shared memory (longer requests
+  // stage them now, in the key buffer)
+  if (T > Q_SMALL) {
+#pragma unroll
+    for (int i = 0; i < QW_PER_T; ++i) {
+      const int g = tid + i * Q_NT;
+      if (g < QW_SIZE) W[q_wpos(g)] = wr[i];
+    }
   }
   __syncthreads();
-  if (tid < Q_H) {
-    float s = W[QS_B1 + tid];
-    for (int i = 0; i < Q_NS; ++i) s = fmaf(W[QS_W1 + tid * (Q_NS + 1) + i], qv[i], s);
-    h1[tid] = fmaxf(s, 0.f);
-  }
-  __syncthreads();
-  if (tid < Q_H) {
-    float s = W[QS_B2 + tid];
-    for (int i = 0; i < Q_H; ++i) s = fmaf(W[QS_W2 + tid * (Q_H + 1) + i], h1[i], s);
-    h2[tid] = fmaxf(s, 0.f);
+  // four threads per hidden unit: each sums a quarter of the inputs in order,
+  // then the quarters are added in a fixed butterfly (lanes 4o .. 4o + 3)
+  {
+    const int o = tid >> 2, part = tid & 3;
+    constexpr int P1 = Q_NS / 4, P2 = Q_H / 4;
+    float s1 = 0.f;
+#pragma unroll
+    for (int i = 0; i < P1; ++i)
+      s1 = fmaf(W[QS_W1 + o * (Q_NS + 1) + part * P1 + i], qv[part * P1 + i], s1);
+    s1 += __shfl_xor_sync(FULL, s1, 1);
+    s1 += __shfl_xor_sync(FULL, s1, 2);
+    if (part == 0) h1[o] = fmaxf(s1 + W[QS_B1 + o], 0.f);
+    __syncthreads();
+    float s2 = 0.f;
+#pragma unroll
+    for (int i = 0; i < P2; ++i)
+      s2 = fmaf(W[QS_W2 + o * (Q_H + 1) + part * P2 + i], h1[part * P2 + i], s2);
+    s2 += __shfl_xor_sync(FULL, s2, 1);
+    s2 += __shfl_xor_sync(FULL, s2, 2);
+    if (part == 0) h2[o] = fmaxf(s2 + W[QS_B2 + o], 0.f);
   }
   __syncthreads();
   if (warp < 2) {

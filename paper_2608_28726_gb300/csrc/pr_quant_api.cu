@@ -21,6 +21,7 @@ pr_status pr_quantile_score(pr_ctx* c, const float* feat, const uint32_t* row_fl
   if (n_req == 0) return PR_OK;
   if (!offsets || !w || !score || !ship || !req_flags) return PR_ERR_INVALID_ARG;
   if (n_rows > 0 && !feat) return PR_ERR_INVALID_ARG;
+  if (!aligned16(feat)) return PR_ERR_INVALID_ARG;  // records are read as 16-byte words
   pr_status st = set_device(c);
   if (st != PR_OK) return st;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
