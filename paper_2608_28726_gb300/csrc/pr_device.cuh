@@ -340,6 +340,7 @@ struct Smem {
   float fm, fS, fU;
   int fbad;
   uint64_t flist[32];
+  uint64_t top[32];           // the CTA's top-32 keys, ranked by counting
   int careful, fallback;
 };
 

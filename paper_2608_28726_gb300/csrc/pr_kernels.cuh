@@ -548,9 +548,29 @@ __global__ void __launch_bounds__(NT) verify_rows(const Args a) {
     if (lane == 0) {
       sm.theta1 = th1;
       sm.fallback = !(th1 > -INFINITY);
+      // a masked (-inf), NaN or infinite logit made the CTA's fast
+      // accumulators non-finite: it re-streams its range with guards (the
+      // row's merged state is non-finite exactly when a CTA's is)
+      sm.careful = (!bad && !(isfinite(S) && isfinite(U))) ? 1 : 0;
     }
   }
+  if (tid < 32) sm.top[tid] = 0ull;
   __syncthreads();
+  if (sm.careful) {
+    float cm = M2_INIT, cS = 0.f, cU = 0.f;
+    bool cbad = false;
+    const int64_t e1 = (int64_t)g1 * VEC;
+    for (int64_t v = (int64_t)g0 * VEC + tid; v < e1; v += NT)
+      careful_add(Tr::elem(rowp, v), cm, cS, cU, cbad);
+    if (has_tail && rank == 0)
+      for (int64_t v = (int64_t)gfull * VEC + tid; v < V; v += NT)
+        careful_add(Tr::elem(rowp, v), cm, cS, cU, cbad);
+    block_reduce_state(sm, cm, cS, cU, cbad, warp, lane);  // warp 0 holds the CTA's state
+    m = cm;
+    S = cS;
+    U = cU;
+    bad = cbad;
+  }
 
   // ---- candidate super-groups: stored tile maxima >= theta1
   const float th1 = sm.theta1;
@@ -575,32 +595,16 @@ __global__ void __launch_bounds__(NT) verify_rows(const Args a) {
   }
   __syncthreads();
 
-  // ---- theta: the exact kc-th largest candidate value (warp 0)
-  if (warp == 0 && !sm.fallback) {
-    const int n = sm.ncand;
-    if (n > CCAP) {
-      if (lane == 0) sm.fallback = 1;
-    } else {
-      uint32_t L = 0u;
-      for (int b0 = 0; b0 < n; b0 += 32) {
-        uint32_t k = b0 + lane < n ? ord(sm.cand_v[b0 + lane]) : 0u;
-        k = warp_sort_desc<uint32_t>(k, lane);
-        L = warp_merge_desc<uint32_t>(L, k, lane);
-      }
-      const float th = unord(__shfl_sync(FULL, L, kc - 1));
-      if (lane == 0) sm.theta = th;
-    }
-  }
-  __syncthreads();
-
-  // ---- re-read the candidates >= theta; elements >= theta become keys
-  if (!sm.fallback) {
-    const float th = sm.theta;
-    const int n = sm.ncand;
+  // ---- re-read the candidates; their elements >= theta1 become keys (kc
+  // distinct elements reach theta1, so the CTA's top kc are among them)
+  const int ncand = sm.ncand;
+  const bool fb_cand = sm.fallback || ncand > CCAP;
+  if (!fb_cand) {
+    const float th = th1;
+    const int n = ncand;
     const int gpc = UNR << shift;  // groups per super-group
     for (int i = tid; i < n * gpc; i += NT) {
       const int c = i / gpc, j = i - c * gpc;
-      if (!(sm.cand_v[c] >= th)) continue;
       const uint32_t id = sm.cand_id[c];
       if (id == TAIL_ID) {
         if (j != 0) continue;
@@ -630,11 +634,39 @@ __global__ void __launch_bounds__(NT) verify_rows(const Args a) {
   }
   __syncthreads();
 
-  // ---- the CTA's exact top-32 elements (warp 0)
+  // ---- what the row's epilogue needs besides the reduction (cluster rank 0,
+  // warp 0), fetched now so that its latency overlaps the selection
+  RowPre pre;
+  if (rank == 0 && warp == 0) {
+    pre = load_pre<T, MODE>(a, row, rowp, lane);
+    if (C == 1) {
+      pdl_wait();
+      if (MODE == MODE_DECODE && lane == 0 && pre.r >= 0 && pre.r < a.n_slots) {
+        const float* A = a.acc + (int64_t)pre.r * ACC_WORDS;  // into L1 for row_finish
+        asm volatile("prefetch.global.L1 [%0];" ::"l"(A));
+        asm volatile("prefetch.global.L1 [%0];" ::"l"(A + 16));
+      }
+    }
+  }
+
+  // ---- the CTA's exact top-32 elements: up to NT candidate keys are ranked
+  // by counting (keys are distinct: the index is part of the key), more by
+  // warp 0's sorting network; the exact scan when the buffers overflowed
   uint64_t E = 0ull;
-  if (warp == 0) {
-    const int n = sm.nelem;
-    if (!sm.fallback && n <= ECAP) {
+  const int ne = sm.nelem;
+  const bool fb = fb_cand || ne > ECAP;
+  if (!fb && ne <= NT) {
+    if (tid < ne) {
+      const uint64_t key = sm.ebuf[tid];
+      int rk = 0;
+      for (int q = 0; q < ne; ++q) rk += sm.ebuf[q] > key ? 1 : 0;
+      if (rk < 32) sm.top[rk] = key;
+    }
+    __syncthreads();
+    if (warp == 0) E = sm.top[lane];
+  } else if (warp == 0) {
+    const int n = ne;
+    if (!fb) {
       for (int b0 = 0; b0 < n; b0 += 32) {
         uint64_t k = b0 + lane < n ? sm.ebuf[b0 + lane] : 0ull;
         k = warp_sort_desc<uint64_t>(k, lane);
@@ -703,22 +735,8 @@ __global__ void __launch_bounds__(NT) verify_rows(const Args a) {
     if (rank != 0) return;
   }
 
-  // ---- rows that made the fast accumulators non-finite: re-stream with guards
-  if (warp == 0 && lane == 0) sm.careful = (!bad && !(isfinite(S) && isfinite(U))) ? 1 : 0;
-  __syncthreads();
-  if (sm.careful) {
-    float cm = M2_INIT, cS = 0.f, cU = 0.f;
-    bool cbad = false;
-    for (int64_t v = tid; v < V; v += NT) careful_add(Tr::elem(rowp, v), cm, cS, cU, cbad);
-    block_reduce_state(sm, cm, cS, cU, cbad, warp, lane);
-    m = cm;
-    S = cS;
-    U = cU;
-    bad = cbad;
-  }
   if (warp != 0) return;
 
-  const RowPre pre = load_pre<T, MODE>(a, row, rowp, lane);
   pdl_wait();
   if (MODE == MODE_ROUTE) {
     const int64_t nclusters = gridDim.x / C;
