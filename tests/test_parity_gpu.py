@@ -229,6 +229,32 @@ def test_route_matches_oracle(ctx, dtype, split):
     assert torch.equal(ship, ship2)
 
 
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+def test_every_launch_shape_of_the_automatic_policy(ctx, dtype):
+    """The automatic launch shape changes with the batch: clusters of 8, 4,
+    2 CTAs per row for small batches, one CTA per row (no cluster) from one
+    row per SM up to one wave of resident CTAs, the persistent kernel above.
+    Batches on both sides of each switch, against the oracle; features and
+    routing alike."""
+    _set(ctx)
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    # resident CTAs of the split kernel: 3 or 4 per SM on this GPU
+    sizes = sorted({1, 7, 37, 38, 39, 75, 76, 77, sms - 1, sms, sms + 1, 3 * sms, 4 * sms,
+                    4 * sms + 1, 5 * sms})
+    for i, n in enumerate(sizes):
+        lengths = [n // 2, n - n // 2] if n > 1 else [1]
+        x, ch, off, w, b = _batch(lengths, 2053, dtype, seed=300 + i)
+        o = oracle.route(as_oracle(x), ch.cpu().numpy(), off, w.astype(np.float64), b, 0.5)
+        dw, doff = torch.from_numpy(w).cuda(), torch.from_numpy(off).cuda()
+        score, ship, rf, agg = B.pr_route(ctx, x, ch, doff, dw, b, 0.5)
+        feat, top2, rfl = B.pr_token_features(ctx, x, ch, topk=20)
+        torch.cuda.synchronize()
+        _check_requests(score, ship, rf, agg, o, 0.5, "route n=%d" % n)
+        assert np.array_equal(top2.cpu().numpy(), o["idx"]), "top2 n=%d" % n
+        assert_close(feat.cpu().numpy()[:, [0, 1, 2, 3, 4, 6, 7]],
+                     o["feat"][:, [0, 1, 2, 3, 4, 6, 7]], "features n=%d" % n)
+
+
 def test_route_threshold_and_flags(ctx):
     """Zero weights give score 1/2, which ships at tau = 1/2 (ship iff p >= tau)."""
     lengths = [4, 6]
