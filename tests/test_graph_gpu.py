@@ -67,8 +67,13 @@ def test_route_calls_replay_in_a_graph(B, overlap):
         B.pr_ctx_destroy(ctx)
 
 
-def test_decode_trace_replays_in_a_graph(B):
-    n_slots, steps, V = 8, 60, 3000
+@pytest.mark.parametrize("n_slots,overlap", [(8, 0), (8, 1), (256, 0), (256, 1)])
+def test_decode_trace_replays_in_a_graph(B, n_slots, overlap):
+    """A decode trace captured in a CUDA graph gives the bits of the same
+    trace run call by call without overlap: with 8 slots (clusters of CTAs
+    per row) and with 256 (one CTA per row, two launches resident at once
+    when the overlap option lets the next step start early)."""
+    steps, V = 60, 3000
     g0 = np.random.default_rng(3)
     eos = (g0.random((steps, n_slots)) < 0.08).astype(np.uint8)
     rows = [random_rows(n_slots, V, torch.bfloat16, seed=700 + t) for t in range(steps)]
@@ -87,12 +92,14 @@ def test_decode_trace_replays_in_a_graph(B):
                 B.pr_decode_step(ctx, x, slot, ch, eos_d[t], w, -0.1, 0.5, score[t], ship[t],
                                  fl[t])
 
+        B.pr_ctx_set_option(ctx, B.PR_OPT_OVERLAP, 0)
         trace()
         torch.cuda.synchronize()
         ref = (score.clone(), ship.clone(), fl.clone())
         ref_state = B.pr_state_export(ctx)
         for t in (score, ship, fl):
             t.fill_(0)
+        B.pr_ctx_set_option(ctx, B.PR_OPT_OVERLAP, overlap)
         g = _capture(trace)
         g.replay()
         torch.cuda.synchronize()
