@@ -887,6 +887,18 @@ HEAD_FILES = ("pr_device.cuh", "pr_head.cuh", "pr_head_api.cu")
 HEAD_PROFILE = os.path.join(ROOT, "profiles", "head_attn_f32_full_response.md")
 # fp32 CUDA-core peak: 152 SMs x 128 FMA lanes x 2 flop x 2,070 MHz (maximum SM clock)
 FP32_PEAK_TFLOPS = 152 * 128 * 2 * 2.070e9 / 1e12
+# dense TF32 tensor rate against dense bf16, nominal (1.1 / 2.25 PFLOP/s)
+TF32_PER_BF16 = 1.1 / 2.25
+
+
+def tf32_peak():
+    """(TF/s, source): the measured bf16 burst rate x the nominal TF32 ratio."""
+    peaks_file = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    peaks = json.load(open(peaks_file)) if os.path.exists(peaks_file) else {}
+    bf16 = float(peaks.get("bf16_tflops", 0.0) or 0.0)
+    if bf16 > 0:
+        return bf16 * TF32_PER_BF16, "measured bf16 burst (%.1f TF/s) x 1.1/2.25" % bf16
+    return 1900.0 * TF32_PER_BF16, "fallback bf16 1,900 TF/s x 1.1/2.25"
 
 
 def head_flops(lengths, n_layers: int):
@@ -1029,6 +1041,7 @@ def run_head_workload(args):
 
     step_flops, attn_flops = head_flops(lengths, n_layers)
     achieved = attn_flops / (attn_ms / 1e3) / 1e12
+    tf32_pk, tf32_src = tf32_peak()
     if rank == 0:
         req_hi = n_req  # the whole workload: under a second of oracle time
         lo, hi = 0, int(offsets[req_hi])
@@ -1048,11 +1061,13 @@ def run_head_workload(args):
                                        n_req, n_rows),
                        "l2": "256 MB written between timed steps (flush)",
                        "n_layers": n_layers},
-            "roofline": {"bound": "alu", "achieved": achieved, "peak": FP32_PEAK_TFLOPS,
-                         "unit": "TFLOP/s", "frac": achieved / FP32_PEAK_TFLOPS,
+            "roofline": {"bound": "tensor", "achieved": achieved, "peak": tf32_pk,
+                         "unit": "TFLOP/s", "frac": achieved / tf32_pk,
                          "traffic": profiled_file_traffic(HEAD_PROFILE, HEAD_FILES),
                          "kernel": "head_attn",
-                         "peak_source": "derived: 152 SMs x 128 fp32 FMA lanes x 2 x 2.07 GHz",
+                         "peak_source": tf32_src + "; the contractions run as three TF32 "
+                                        "products per fp32 product",
+                         "fp32_cuda_core_frac": achieved / FP32_PEAK_TFLOPS,
                          "algorithmic_flops_per_launch": attn_flops,
                          "avg_launch_ms": attn_ms,
                          "step_flops": step_flops,

@@ -310,8 +310,13 @@ int64_t pr_head_param_count(int32_t n_layers);
  *                  W_2[64][128] b_2[64] g2[64] be2[64]
  *                w_out[64] b_out
  *   score, ship, req_flags   device [n_req]            (outputs)
- * The batch runs layer by layer in 2 n_layers + 3 launches on `stream`; all
- * arithmetic is fp32 in a fixed order, so results are bit-reproducible.  The
+ * The batch runs layer by layer in 2 n_layers + 3 launches on `stream`.  The
+ * attention's two contractions run on the tensor cores (tcgen05) with each
+ * fp32 operand split into two TF32 parts and three products per product
+ * (errors below 2^-21 of a product); everything else is fp32 on the CUDA
+ * cores; all sums run in a fixed order, so results are bit-reproducible.  A
+ * bounded wait on the tensor cores that runs out raises PR_FLAG_TIMEOUT in
+ * the context's flag word (that call's outputs are invalid).  The
  * context holds a device scratch of 1 KB per row, allocated (or grown) by the
  * first call with more rows than before -- that call synchronises the device;
  * calls on different streams must not overlap (they share that scratch).

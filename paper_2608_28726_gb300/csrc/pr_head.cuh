@@ -11,14 +11,16 @@
 //                row-local work between two attentions, fused per tile --
 //                O = A W_o^T + b_o, H = LN1(H + O), F = W_2 ReLU(W_1 H + b_1) + b_2,
 //                H = LN2(H + F), then the next layer's QKV = H W_qkv^T + b_qkv
-//   head_attn    one CTA per (request, head): softmax(Q K^T / 4) V with the
-//                keys and values staged in shared memory, online softmax
+//   head_attn    one CTA per (request, head, 128-query block): softmax(Q K^T / 4) V
+//                on the tensor cores (tcgen05, TF32 operands split in two for
+//                fp32 accuracy), online softmax over 128-key chunks
 //   head_pool    one CTA per request: fixed-order mean over t, sigmoid layer
 // Activations live in a scratch of 256 floats per row (H | Q | K | V; the
 // attention output overwrites Q), which stays in L2 for batches of tens of
-// MB.  All arithmetic is fp32 on the CUDA cores (fp32 FMA, no tensor-core
-// rounding) and every sum runs in a fixed order, so results are reproducible
-// bit for bit.
+// MB.  The row kernels run fp32 FMAs on the CUDA cores; the attention's two
+// contractions run on the tensor cores with each fp32 operand split into two
+// TF32 parts (three products per product), which keeps fp32-level accuracy.
+// Every sum runs in a fixed order, so results are reproducible bit for bit.
 #pragma once
 
 #include "pr_device.cuh"
@@ -431,145 +433,480 @@ __global__ void __launch_bounds__(NT, MODE == HR_QKV ? 2 : 1) head_rows(const He
   cp_async_wait<0>();
 }
 
-constexpr int HAW = 4;          // warps per head_attn CTA
-constexpr int HKT = 32 * HAW;   // keys per shared-memory tile: 32 per warp
-constexpr int HQS = 16;         // CTAs per (request, head)
+// ---- head_attn: softmax(Q K^T / 4) V on the tensor cores ----------------------------
+//
+// CTA (request, head, z) takes the 128-query blocks z, z + HA_QZ, ... of its
+// request; thread i owns query i of the block and TMEM lane i.  The keys pass
+// in chunks of 64.  Per chunk two tcgen05.mma kind::tf32 contractions run with
+// fp32 accumulators in TMEM: S = Q K^T (M = 128 queries, N = the chunk's keys
+// rounded up to 16, K = 16) and O_c = P V (M = 128, K = the chunk's keys
+// rounded up to 8).  Every fp32 operand x is split into x_hi = tf32(x) and
+// x_lo = x - x_hi, and a product is taken as a_hi b_hi + a_hi b_lo +
+// a_lo b_hi: the dropped a_lo b_lo and the tensor core's truncation of x_lo
+// to TF32 are below 2^-21 of the product, so the contractions keep fp32-level
+// accuracy on TF32 units.  The value operand is [V_hi | V_lo] side by side
+// (N = 32), so each K step of P V is two MMAs, P_hi [V_hi | V_lo] and
+// P_lo [V_hi | V_lo] (the P_lo V_lo half is never read), and O_c is the sum
+// of the accumulator's two halves.
+//
+// Between the two contractions each thread reads its row of S, keeps the
+// running maximum and sum (base 2, online over the chunks), writes P_hi back
+// over S in TMEM (the A operand of the first MMA of a K step) and P_lo to
+// shared memory (the second), and after P V folds O_c into its running
+// output; the next chunk's keys and values are loaded while the P V MMAs
+// run.  A CTA holds 128 TMEM columns and 50 KB of shared memory, so four run
+// on an SM and one's MMAs overlap another's softmax.  One elected thread
+// issues the MMAs; every wait on their completion is bounded.
+//
+// TMEM columns: S / P_hi 0-63, O_c 64-95, Q_hi 96-111, Q_lo 112-127.
+// Shared memory: the key operand and P_lo in the K-major canonical layout
+// without swizzle (core matrices of 8 rows x 16 bytes, consecutive along K at
+// 128 bytes, 8-row groups at the stride byte offset); [V_hi | V_lo]^T in the
+// 128-byte swizzled K-major layout (8 rows x 128 bytes per 1,024-byte atom,
+// the 16-byte piece c of row r stored at piece c ^ r), so that the 32 lanes
+// writing one dimension of 32 consecutive keys hit 32 different banks.
+constexpr int HA_M = 128;                       // queries per block = TMEM lanes = threads
+constexpr int HA_NC = 64;                       // keys per chunk
+constexpr int HA_QZ = 8;                        // CTAs per (request, head)
+constexpr uint32_t HA_TMEM_COLS = 128;
+constexpr uint32_t HA_O_COL = HA_NC;            // O_c: [V_hi | V_lo] products, 32 columns
+constexpr uint32_t HA_QH_COL = HA_O_COL + 2 * HDH;
+constexpr uint32_t HA_QL_COL = HA_QH_COL + HDH;
+constexpr int HA_K_SBO = (HDH / 4) * 128;       // key rows of 16 values: 4 core matrices
+constexpr int HA_P_SBO = (HA_NC / 4) * 128;     // P_lo rows of 64 keys: 16 core matrices
+constexpr int HA_VT_ROWS = 2 * HDH;             // [V_hi | V_lo]^T rows
+constexpr int HA_VT_ATOM = HA_VT_ROWS * 128;    // 32 keys of all rows: 4 swizzle atoms
+// shared memory (bytes from the 1,024-aligned base)
+constexpr int HA_VT = 0;
+constexpr int HA_K_HI = HA_VT + (HA_NC / 32) * HA_VT_ATOM;
+constexpr int HA_K_LO = HA_K_HI + HA_NC * HDH * 4;
+constexpr int HA_P_LO = HA_K_LO + HA_NC * HDH * 4;
+constexpr int HA_BAR = HA_P_LO + HA_M * HA_NC * 4;  // mbarrier: MMA completion
+constexpr int HA_TSLOT = HA_BAR + 8;                // TMEM base from tcgen05.alloc
+constexpr size_t HA_SMEM = HA_TSLOT + 8 + 1024;     // + alignment of the base
+constexpr int HA_CTAS_PER_SM = 4;
+static_assert(HA_CTAS_PER_SM * (HA_SMEM + 1024) <= 233472, "shared memory of four CTAs");
+static_assert(HA_CTAS_PER_SM * HA_TMEM_COLS <= 512 && HA_QL_COL + HDH <= HA_TMEM_COLS,
+              "TMEM columns");
+static_assert(HA_VT % 1024 == 0 && HA_VT_ATOM % 1024 == 0, "swizzle atoms are 1,024-aligned");
+static_assert(HA_NC == 64, "a thread reads its scores in two groups of 32 columns");
+// instruction descriptors of tcgen05.mma kind::tf32: fp32 accumulator (bits
+// 4-5 = 1), TF32 A and B (bits 7-9, 10-12 = 2), both K-major (bits 15, 16 =
+// 0), N / 8 in bits 17-22, M / 16 in bits 24-28
+constexpr uint32_t HA_IDESC_S = (1u << 4) | (2u << 7) | (2u << 10) |
+                                ((uint32_t)(HA_M >> 4) << 24);  // N (<= 64) set per chunk
+constexpr uint32_t HA_IDESC_O = (1u << 4) | (2u << 7) | (2u << 10) |
+                                ((uint32_t)(HA_VT_ROWS >> 3) << 17) | ((uint32_t)(HA_M >> 4) << 24);
+constexpr uint64_t HA_WAIT_NS = 2000000000ull;  // a wait gives up after 2 s
+constexpr uint32_t HA_ERR_TIMEOUT = 32u;        // PR_FLAG_TIMEOUT in the context flag word
 
-// CTA (request, head, z) takes the 32-query blocks z, z + 8, z + 16, ...; a
-// lane owns one query.  For each block all keys and values of the head pass
-// through shared memory in tiles of 128; warp w scores keys 32 w .. 32 w + 31
-// of every tile, 16 at a time, keeping a running maximum, sum and output (in
-// base 2: the queries carry the factor log2(e) / 4).  The four warps' partial
-// states are merged in warp order at the end of the block.
-__global__ void __launch_bounds__(HAW * 32) head_attn(const HeadArgs a) {
-  __shared__ __align__(16) float4 ks[HKT][HDH / 4];
-  __shared__ __align__(16) float4 vs[HKT][HDH / 4];
-  __shared__ float part[HAW][HDH + 2][32];
-  pdl_trigger();
-  pdl_wait();
-  int64_t lo, hi;
-  if (!head_request(a, blockIdx.x, lo, hi)) return;
-  const int hh = blockIdx.y, z = blockIdx.z;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int T = (int)(hi - lo);
-  float* scr = a.scratch + lo * HSCR;
-  const int nqb = (T + 31) >> 5;
-  constexpr float QSCALE = 0.25f * L2E;  // 1 / sqrt(16), in base 2
-
-  for (int qb = z; qb < nqb; qb += HQS) {
-    const int t = qb * 32 + lane;
-    const bool on = t < T;
-    float2 q2[HDH / 2], acc2[HDH / 2];  // (dimension 2e, 2e + 1) pairs
-    {
-      const float4* qp = reinterpret_cast<const float4*>(scr + (int64_t)(on ? t : 0) * HSCR + HD +
-                                                         hh * HDH);
+__device__ __forceinline__ uint32_t ha_saddr(const void* p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+// byte offset of (row, 4-value piece j) in the canonical layout without swizzle
+__device__ __forceinline__ uint32_t ha_kmaj(int row, int j, int sbo) {
+  return (uint32_t)((row >> 3) * sbo + j * 128 + (row & 7) * 16);
+}
+// byte offset of (row, key k) in the swizzled [V_hi | V_lo]^T operand
+__device__ __forceinline__ uint32_t ha_vt(int row, int k) {
+  const int r = row & 7, c = (k >> 2) & 7;
+  return (uint32_t)(HA_VT + (k >> 5) * HA_VT_ATOM + (row >> 3) * 1024 + r * 128 + ((c ^ r) << 4) +
+                    (k & 3) * 4);
+}
+// matrix descriptors: start >> 4 in bits 0-13, leading byte offset >> 4 in
+// bits 16-29, stride byte offset >> 4 in bits 32-45, version 1 in bits
+// 46-47, layout in bits 61-63 (0: no swizzle, 2: 128-byte swizzle)
+__device__ __forceinline__ uint64_t ha_desc(uint32_t saddr, uint32_t sbo) {
+  return (uint64_t)((saddr >> 4) & 0x3fffu) | ((uint64_t)(128u >> 4) << 16) |
+         ((uint64_t)((sbo >> 4) & 0x3fffu) << 32) | ((uint64_t)1 << 46);
+}
+__device__ __forceinline__ uint64_t ha_desc_sw128(uint32_t saddr) {
+  return (uint64_t)((saddr >> 4) & 0x3fffu) | ((uint64_t)1 << 16) |
+         ((uint64_t)(1024u >> 4) << 32) | ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+// tf32(x) rounded to nearest (ties away): the 13 low mantissa bits cleared
+// after adding half of their range; exact for finite x, and x - tf32(x) is
+// exact in fp32
+__device__ __forceinline__ float ha_hi(float x) {
+  return __uint_as_float((__float_as_uint(x) + 0x1000u) & 0xffffe000u);
+}
+__device__ __forceinline__ void ha_split(const float4 x, float4& h, float4& l) {
+  h = make_float4(ha_hi(x.x), ha_hi(x.y), ha_hi(x.z), ha_hi(x.w));
+  l = make_float4(x.x - h.x, x.y - h.y, x.z - h.z, x.w - h.w);
+}
+__device__ __forceinline__ void ha_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void ha_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+// generic-proxy shared-memory writes become visible to the tensor cores
+__device__ __forceinline__ void ha_fence_async() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+// D (+)= A B^T, A and B from shared memory
+__device__ __forceinline__ void ha_mma(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc,
+                                       uint32_t acc) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.u32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n\t}" ::"r"(d),
+      "l"(a), "l"(b), "r"(idesc), "r"(acc)
+      : "memory");
+}
+// D (+)= A B^T, A from TMEM (lane = row, one column per K value)
+__device__ __forceinline__ void ha_mma_ta(uint32_t d, uint32_t a, uint64_t b, uint32_t idesc,
+                                          uint32_t acc) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.u32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::tf32 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d),
+      "r"(a), "l"(b), "r"(idesc), "r"(acc)
+      : "memory");
+}
+__device__ __forceinline__ void ha_commit(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                   bar)
+               : "memory");
+}
+__device__ __forceinline__ bool ha_try(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ uint64_t ha_clock() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+// bounded wait for the phase with the given parity: false once HA_WAIT_NS
+// nanoseconds have passed without it
+__device__ __forceinline__ bool ha_wait(uint32_t bar, uint32_t parity) {
+  if (ha_try(bar, parity)) return true;
+  const uint64_t t0 = ha_clock();
+  for (uint32_t i = 1;; ++i) {
+    if (ha_try(bar, parity)) return true;
+    if ((i & 255u) == 0u && ha_clock() - t0 > HA_WAIT_NS) return false;
+  }
+}
+// 32 / 16 consecutive fp32 columns of this warp's 32 TMEM lanes (lane = row)
+__device__ __forceinline__ void ha_ld32(uint32_t taddr, float (&v)[32]) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
+        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
+        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 #pragma unroll
-      for (int d = 0; d < HDH / 4; ++d) {
-        const float4 v = qp[d];
-        q2[2 * d] = make_float2(v.x * QSCALE, v.y * QSCALE);
-        q2[2 * d + 1] = make_float2(v.z * QSCALE, v.w * QSCALE);
+  for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+}
+__device__ __forceinline__ void ha_ld16(uint32_t taddr, float (&v)[16]) {
+  uint32_t r[16];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(r[j]);
+}
+__device__ __forceinline__ void ha_st32(uint32_t taddr, const float (&v)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
+      "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, "
+      "%17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(
+          taddr),
+      "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])),
+      "r"(__float_as_uint(v[3])), "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])),
+      "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])), "r"(__float_as_uint(v[8])),
+      "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])),
+      "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])),
+      "r"(__float_as_uint(v[15])), "r"(__float_as_uint(v[16])), "r"(__float_as_uint(v[17])),
+      "r"(__float_as_uint(v[18])), "r"(__float_as_uint(v[19])), "r"(__float_as_uint(v[20])),
+      "r"(__float_as_uint(v[21])), "r"(__float_as_uint(v[22])), "r"(__float_as_uint(v[23])),
+      "r"(__float_as_uint(v[24])), "r"(__float_as_uint(v[25])), "r"(__float_as_uint(v[26])),
+      "r"(__float_as_uint(v[27])), "r"(__float_as_uint(v[28])), "r"(__float_as_uint(v[29])),
+      "r"(__float_as_uint(v[30])), "r"(__float_as_uint(v[31]))
+      : "memory");
+}
+
+__device__ __forceinline__ void ha_st16(uint32_t taddr, const float4 (&v)[4]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+      "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16};" ::"r"(taddr),
+      "r"(__float_as_uint(v[0].x)), "r"(__float_as_uint(v[0].y)), "r"(__float_as_uint(v[0].z)),
+      "r"(__float_as_uint(v[0].w)), "r"(__float_as_uint(v[1].x)), "r"(__float_as_uint(v[1].y)),
+      "r"(__float_as_uint(v[1].z)), "r"(__float_as_uint(v[1].w)), "r"(__float_as_uint(v[2].x)),
+      "r"(__float_as_uint(v[2].y)), "r"(__float_as_uint(v[2].z)), "r"(__float_as_uint(v[2].w)),
+      "r"(__float_as_uint(v[3].x)), "r"(__float_as_uint(v[3].y)), "r"(__float_as_uint(v[3].z)),
+      "r"(__float_as_uint(v[3].w))
+      : "memory");
+}
+
+// P = 2^(s QSCALE - mn) over 32 of this thread's score columns (col0 = the
+// first one's index in the chunk): P_hi back into TMEM over S, P_lo into
+// shared memory, the row sum into ls
+template <bool FULL>
+__device__ __forceinline__ void ha_softmax32(float (&v)[32], int col0, int nk, float qscale,
+                                             float mn, float& ls, uint8_t* plo_row, int row,
+                                             uint32_t taddr) {
+#pragma unroll
+  for (int j4 = 0; j4 < 8; ++j4) {
+    float pl[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int j = 4 * j4 + e;
+      float p = ex2(fmaf(v[j], qscale, -mn));
+      if (!FULL) p = col0 + j < nk ? p : 0.f;
+      ls += p;
+      const float ph = ha_hi(p);
+      v[j] = ph;
+      pl[e] = p - ph;
+    }
+    *reinterpret_cast<float4*>(plo_row + ha_kmaj(row, (col0 >> 2) + j4, HA_P_SBO)) =
+        make_float4(pl[0], pl[1], pl[2], pl[3]);
+  }
+  ha_st32(taddr, v);
+}
+
+__global__ void __launch_bounds__(HA_M, HA_CTAS_PER_SM) head_attn(const HeadArgs a) {
+  extern __shared__ uint8_t ha_raw[];
+  const int tid = threadIdx.x, warp = tid >> 5;
+  int64_t lo, hi;
+  // the offsets are inputs of the call, complete before its first kernel
+  const int T = head_request(a, blockIdx.x, lo, hi) ? (int)(hi - lo) : 0;
+  const int nqb = (T + HA_M - 1) / HA_M;
+  if ((int)blockIdx.z >= nqb) {
+    pdl_trigger();
+    return;
+  }
+  const int hh = blockIdx.y;
+  float* scr = a.scratch + lo * HSCR;
+  // staging: key kr = tid % 64 of a chunk, its K (part 0) or V (part 1) row
+  const int kr = tid & (HA_NC - 1), part = tid >> 6;
+  const float* kv_src = scr + 2 * HD + part * HD + hh * HDH;
+  float4 pre[HDH / 4];
+  float4 qv[HDH / 4];
+  auto load_row = [&](int k0) {
+    const int k = k0 + kr;
+    const bool on = k < T;  // rows past the request are zero; their scores are masked
+    const float4* src = reinterpret_cast<const float4*>(kv_src + (int64_t)(on ? k : 0) * HSCR);
+#pragma unroll
+    for (int j = 0; j < HDH / 4; ++j) pre[j] = on ? src[j] : make_float4(0.f, 0.f, 0.f, 0.f);
+  };
+  auto load_q = [&](int qb) {
+    const int q = qb * HA_M + tid;
+    const bool on = q < T;
+    const float4* src =
+        reinterpret_cast<const float4*>(scr + (int64_t)(on ? q : 0) * HSCR + HD + hh * HDH);
+#pragma unroll
+    for (int j = 0; j < HDH / 4; ++j) qv[j] = on ? src[j] : make_float4(0.f, 0.f, 0.f, 0.f);
+  };
+  // the first block's loads are in flight while the CTA takes its TMEM
+  pdl_wait();
+  load_q(blockIdx.z);
+  load_row(0);
+  const uint32_t raw = ha_saddr(ha_raw);
+  const uint32_t sb = (raw + 1023u) & ~1023u;  // swizzle atoms need a 1,024-aligned base
+  uint8_t* sm = ha_raw + (sb - raw);
+  const uint32_t bar = sb + HA_BAR;
+  if (tid == 0) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(bar) : "memory");
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  // TMEM is taken before the next kernel may start (the trigger below), so a
+  // later kernel of the stream never holds the columns this CTA waits for
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     sb + HA_TSLOT),
+                 "r"(HA_TMEM_COLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  ha_fence_before();
+  __syncthreads();
+  ha_fence_after();
+  const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(sm + HA_TSLOT);
+  pdl_trigger();
+  const uint32_t tq = tmem + ((uint32_t)(warp * 32) << 16);  // this warp's lane quarter
+  constexpr float QSCALE = 0.25f * L2E;  // 1 / sqrt(16), in base 2
+  uint32_t phase = 0;
+  bool ok = true;
+
+  auto store_row = [&]() {
+    // the row index is re-read here so that the compiler does not keep the
+    // 32 store addresses of the swizzled operand live across the chunk loop
+    int rr;
+    asm volatile("mov.b32 %0, %1;" : "=r"(rr) : "r"(kr));
+    const uint32_t vbase = (uint32_t)((rr >> 5) * HA_VT_ATOM + (rr & 3) * 4);
+    const uint32_t vc = (uint32_t)((rr >> 2) & 7);
+#pragma unroll
+    for (int j = 0; j < HDH / 4; ++j) {
+      float4 h, l;
+      ha_split(pre[j], h, l);
+      if (part == 0) {
+        *reinterpret_cast<float4*>(sm + HA_K_HI + ha_kmaj(rr, j, HA_K_SBO)) = h;
+        *reinterpret_cast<float4*>(sm + HA_K_LO + ha_kmaj(rr, j, HA_K_SBO)) = l;
+      } else {
+        const float hv[4] = {h.x, h.y, h.z, h.w}, lv[4] = {l.x, l.y, l.z, l.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {  // rows d (V_hi) and 16 + d (V_lo), key rr
+          const int d = 4 * j + e;
+          const uint32_t off = vbase + (uint32_t)((d >> 3) * 1024 + (d & 7) * 128) +
+                               ((vc ^ (uint32_t)(d & 7)) << 4);
+          *reinterpret_cast<float*>(sm + HA_VT + off) = hv[e];
+          *reinterpret_cast<float*>(sm + HA_VT + 2 * 1024 + off) = lv[e];
+        }
       }
     }
+  };
+
+  for (int qb = blockIdx.z; qb < nqb && ok; qb += HA_QZ) {
+    const int q = qb * HA_M + tid;
+    if (qb != (int)blockIdx.z) {
+      load_q(qb);
+      load_row(0);
+    }
+    {  // the block's queries into TMEM, split
+      float4 qh[HDH / 4], ql[HDH / 4];
 #pragma unroll
-    for (int e = 0; e < HDH / 2; ++e) acc2[e] = make_float2(0.f, 0.f);
+      for (int j = 0; j < HDH / 4; ++j) ha_split(qv[j], qh[j], ql[j]);
+      ha_st16(tq + HA_QH_COL, qh);
+      ha_st16(tq + HA_QL_COL, ql);
+      asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+    }
+    store_row();
+    float o[HDH];
+#pragma unroll
+    for (int d = 0; d < HDH; ++d) o[d] = 0.f;
     float m = -INFINITY, l = 0.f;
 
-    for (int k0 = 0; k0 < T; k0 += HKT) {
-      const int nk = min(HKT, T - k0);
+    for (int k0 = 0; k0 < T; k0 += HA_NC) {
+      const int nk = min(HA_NC, T - k0);
+      ha_fence_async();
+      ha_fence_before();
       __syncthreads();
-      // the whole tile is written: rows past nk are zero, so the branch-free
-      // loops below read finite values there (their scores are masked)
-      for (int i = tid; i < HKT * 8; i += HAW * 32) {
-        const int kr = i >> 3, pc = i & 7;  // pieces 0-3: K, 4-7: V
-        const bool ok = kr < nk;
-        const float* src = scr + (int64_t)(k0 + (ok ? kr : 0)) * HSCR + 2 * HD + hh * HDH;
-        float4* dst = pc < 4 ? &ks[kr][pc] : &vs[kr][pc - 4];
-        cp_async16(reinterpret_cast<float*>(dst), src + (pc < 4 ? 4 * pc : HD + 4 * (pc - 4)),
-                   ok);
+      ha_fence_after();
+      if (tid == 0) {
+        // S = Q K^T over the chunk's keys rounded up to 16 (N), K = 8 per instruction
+        const uint32_t idesc = HA_IDESC_S | ((uint32_t)(((nk + 15) & ~15) >> 3) << 17);
+        // descriptors of the first K step (a K step adds its byte offset >> 4)
+        const uint64_t dk_hi = ha_desc(sb + HA_K_HI, HA_K_SBO);
+        const uint64_t dk_lo = ha_desc(sb + HA_K_LO, HA_K_SBO);
+#pragma unroll
+        for (int s = 0; s < HDH / 8; ++s) {
+          const uint64_t ko = (256u * s) >> 4;
+          ha_mma_ta(tmem, tmem + HA_QH_COL + 8u * s, dk_hi + ko, idesc, s);
+          ha_mma_ta(tmem, tmem + HA_QH_COL + 8u * s, dk_lo + ko, idesc, 1u);
+          ha_mma_ta(tmem, tmem + HA_QL_COL + 8u * s, dk_hi + ko, idesc, 1u);
+        }
+        ha_commit(bar);
       }
-      cp_async_commit();
-      cp_async_wait<0>();
+      if (!__syncthreads_and(ha_wait(bar, phase))) {
+        ok = false;  // the phase stays: the teardown waits for it again
+        break;
+      }
+      phase ^= 1u;
+      ha_fence_after();
+
+      // this query's 64 scores in two groups of 32 columns; the second group
+      // is skipped when the chunk has no key there (the P V MMAs below stop
+      // at the chunk's keys too).  The first group is read twice (for the
+      // maximum, then for P), so that only 32 scores are held at a time.
+      float va[32], vb[32];
+      const bool full = nk == HA_NC, gb = nk > 32;
+      float mx = -INFINITY;
+      ha_ld32(tq, va);
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (full || j < nk) mx = fmaxf(mx, va[j]);
+      if (gb) {
+        ha_ld32(tq + 32, vb);
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+          if (full || 32 + j < nk) mx = fmaxf(mx, vb[j]);
+      }
+      const float mn = fmaxf(m, mx * QSCALE);
+      float ls = 0.f;
+      if (full) {
+        ha_softmax32<true>(vb, 32, nk, QSCALE, mn, ls, sm + HA_P_LO, tid, tq + 32);
+        ha_ld32(tq, va);
+        ha_softmax32<true>(va, 0, nk, QSCALE, mn, ls, sm + HA_P_LO, tid, tq);
+      } else {
+        if (gb) ha_softmax32<false>(vb, 32, nk, QSCALE, mn, ls, sm + HA_P_LO, tid, tq + 32);
+        ha_ld32(tq, va);
+        ha_softmax32<false>(va, 0, nk, QSCALE, mn, ls, sm + HA_P_LO, tid, tq);
+      }
+      asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+      const float f = ex2(m - mn);  // 0 on the first chunk (m = -inf)
+      l = fmaf(l, f, ls);
+      m = mn;
+      ha_fence_async();
+      ha_fence_before();
       __syncthreads();
-      const int kb = 32 * warp, ke = min(nk, kb + 32);
-      for (int j0 = kb; j0 < ke; j0 += 16) {
-        const int jn = min(16, ke - j0);
-        const float4(*kt)[HDH / 4] = ks + j0;
-        const float4(*vt)[HDH / 4] = vs + j0;
-        float sc[16];
-#pragma unroll
-        for (int jj = 0; jj < 16; ++jj) {
-          float2 d2 = make_float2(0.f, 0.f);  // even / odd dimensions
-#pragma unroll
-          for (int p = 0; p < 4; ++p) {
-            const float4 k4 = kt[jj][p];
-            d2 = __ffma2_rn(q2[2 * p], make_float2(k4.x, k4.y), d2);
-            d2 = __ffma2_rn(q2[2 * p + 1], make_float2(k4.z, k4.w), d2);
-          }
-          sc[jj] = jj < jn ? d2.x + d2.y : -INFINITY;
+      ha_fence_after();
+      if (tid == 0) {
+        const int ns = (nk + 7) >> 3;  // K steps up to the chunk's last key
+        const uint64_t dp_lo = ha_desc(sb + HA_P_LO, HA_P_SBO);
+        const uint64_t dvt = ha_desc_sw128(sb + HA_VT);
+#pragma unroll 4
+        for (int s = 0; s < ns; ++s) {  // O_c = P [V_hi | V_lo], K = 8 keys per instruction
+          const uint64_t vo = (uint64_t)((s >> 2) * HA_VT_ATOM + (s & 3) * 32) >> 4;
+          const uint64_t po = (256u * s) >> 4;
+          ha_mma_ta(tmem + HA_O_COL, tmem + 8u * s, dvt + vo, HA_IDESC_O, s);
+          ha_mma(tmem + HA_O_COL, dp_lo + po, dvt + vo, HA_IDESC_O, 1u);
         }
-        float mt = sc[0];
-#pragma unroll
-        for (int jj = 1; jj < 16; ++jj) mt = fmaxf(mt, sc[jj]);
-        const float mn = fmaxf(m, mt);
-        const float f = ex2(m - mn);
-        l *= f;
-        const float2 f2 = make_float2(f, f);
-#pragma unroll
-        for (int e = 0; e < HDH / 2; ++e) acc2[e] = __fmul2_rn(acc2[e], f2);
-        float pr[16];
-#pragma unroll
-        for (int jj = 0; jj < 16; ++jj) pr[jj] = ex2(sc[jj] - mn);  // 0 for masked keys
-        float ls = 0.f;
-#pragma unroll
-        for (int jj = 0; jj < 16; ++jj) ls += pr[jj];
-        l += ls;
-#pragma unroll
-        for (int jj = 0; jj < 16; ++jj) {
-          const float2 p2 = make_float2(pr[jj], pr[jj]);
-#pragma unroll
-          for (int pp = 0; pp < 4; ++pp) {
-            const float4 v4 = vt[jj][pp];
-            acc2[2 * pp] = __ffma2_rn(p2, make_float2(v4.x, v4.y), acc2[2 * pp]);
-            acc2[2 * pp + 1] = __ffma2_rn(p2, make_float2(v4.z, v4.w), acc2[2 * pp + 1]);
-          }
-        }
-        m = mn;
+        ha_commit(bar);
       }
-    }
-    // merge the four partial states (a warp that saw no key has m = -inf, l = 0)
-    part[warp][0][lane] = m;
-    part[warp][1][lane] = l;
-#pragma unroll
-    for (int e = 0; e < HDH / 2; ++e) {
-      part[warp][2 + 2 * e][lane] = acc2[e].x;
-      part[warp][3 + 2 * e][lane] = acc2[e].y;
-    }
-    __syncthreads();
-    if (warp == 0 && on) {
-      float M = part[0][0][lane];
-#pragma unroll
-      for (int w2 = 1; w2 < HAW; ++w2) M = fmaxf(M, part[w2][0][lane]);
-      float fw[HAW], L = 0.f;
-#pragma unroll
-      for (int w2 = 0; w2 < HAW; ++w2) {
-        fw[w2] = ex2(part[w2][0][lane] - M);
-        L = fmaf(part[w2][1][lane], fw[w2], L);
+      // the next chunk's rows are loaded while the P V MMAs run
+      if (k0 + HA_NC < T) load_row(k0 + HA_NC);
+      if (!__syncthreads_and(ha_wait(bar, phase))) {
+        ok = false;
+        break;
       }
-      const float inv = 1.f / L;
-      float4* op = reinterpret_cast<float4*>(scr + (int64_t)t * HSCR + HD + hh * HDH);
+      phase ^= 1u;
+      ha_fence_after();
+      {  // O = f O + O_c, O_c the sum of the [V_hi | V_lo] halves
+        float oc[32];
+        ha_ld32(tq + HA_O_COL, oc);
 #pragma unroll
-      for (int d4 = 0; d4 < HDH / 4; ++d4) {
-        float o[4];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          float v = 0.f;
-#pragma unroll
-          for (int w2 = 0; w2 < HAW; ++w2) v = fmaf(part[w2][2 + 4 * d4 + e][lane], fw[w2], v);
-          o[e] = v * inv;
-        }
-        op[d4] = make_float4(o[0], o[1], o[2], o[3]);
+        for (int d = 0; d < HDH; ++d) o[d] = fmaf(o[d], f, oc[d] + oc[HDH + d]);
       }
+      if (k0 + HA_NC < T) store_row();
     }
+    if (ok && q < T) {
+      const float inv = 1.f / l;
+      float4* op = reinterpret_cast<float4*>(scr + (int64_t)q * HSCR + HD + hh * HDH);
+#pragma unroll
+      for (int j = 0; j < HDH / 4; ++j)
+        op[j] = make_float4(o[4 * j] * inv, o[4 * j + 1] * inv, o[4 * j + 2] * inv,
+                            o[4 * j + 3] * inv);
+    }
+  }
+  if (!ok) {
+    if (tid == 0) atomicOr(a.ctx_flags, HA_ERR_TIMEOUT);
+    ha_wait(bar, phase);  // the MMAs still pending, bounded as well
+  }
+  ha_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    ha_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                 "r"(HA_TMEM_COLS)
+                 : "memory");
   }
 }
 

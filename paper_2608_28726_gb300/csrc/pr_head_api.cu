@@ -74,6 +74,8 @@ pr_status pr_head_score(pr_ctx* c, const float* feat, const uint32_t* row_flags,
     PR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, prk::head_rows<prk::HR_MID>, prk::NT,
                                                           prk::HEAD_ROWS_SMEM_FULL));
     c->head_bps_full = n > 0 ? n : 1;
+    PR_CUDA(cudaFuncSetAttribute(prk::head_attn, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)prk::HA_SMEM));
     c->head_ready = true;
   }
   if (n_rows > c->head_scr_rows) {
@@ -126,8 +128,8 @@ pr_status pr_head_score(pr_ctx* c, const float* feat, const uint32_t* row_flags,
     if (st != PR_OK) return st;
     for (int l = 0; l < n_layers; ++l) {
       st = launch_head(c, reinterpret_cast<const void*>(&prk::head_attn),
-                       dim3((unsigned)n_req, prk::HHEADS, prk::HQS), dim3(prk::HAW * 32), 0, s,
-                       true, a);
+                       dim3((unsigned)n_req, prk::HHEADS, prk::HA_QZ), dim3(prk::HA_M),
+                       prk::HA_SMEM, s, true, a);
       if (st != PR_OK) return st;
       a.lcur = layer(l);
       const bool last = l + 1 == n_layers;

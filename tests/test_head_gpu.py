@@ -85,6 +85,12 @@ def test_head_long_requests(B, ctx):
     check(B, ctx, [1024, 1000, 513], 2, seed=4300)
 
 
+def test_head_requests_past_one_round_of_query_blocks(B, ctx):
+    """T = 2,100 and 1,300: more 128-query blocks than CTAs per (request,
+    head), so a CTA takes a second block; 17 key chunks with a ragged last one."""
+    check(B, ctx, [2100, 1, 1300, 128], 2, seed=4350)
+
+
 def test_head_thresholds(B, ctx):
     g = np.random.Generator(np.random.PCG64(7))
     lengths = g.integers(1, 80, size=40, endpoint=True)
