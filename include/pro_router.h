@@ -311,10 +311,11 @@ int64_t pr_head_param_count(int32_t n_layers);
  *                w_out[64] b_out
  *   score, ship, req_flags   device [n_req]            (outputs)
  * The batch runs layer by layer in 2 n_layers + 3 launches on `stream`.  The
- * attention's two contractions run on the tensor cores (tcgen05) with each
- * fp32 operand split into two TF32 parts and three products per product
- * (errors below 2^-21 of a product); everything else is fp32 on the CUDA
- * cores; all sums run in a fixed order, so results are bit-reproducible.  A
+ * contractions (the attention's Q K^T and P V, the projections and the
+ * feed-forward) run on the tensor cores (tcgen05) with each fp32 operand
+ * split into two TF32 parts and three products per product (errors below
+ * 2^-21 of a product); the softmax, LayerNorm and the rest are fp32 on the
+ * CUDA cores; all sums run in a fixed order, so results are bit-reproducible.  A
  * bounded wait on the tensor cores that runs out raises PR_FLAG_TIMEOUT in
  * the context's flag word (that call's outputs are invalid).  The
  * context holds a device scratch of 1 KB per row, allocated (or grown) by the

@@ -46,7 +46,6 @@ struct pr_ctx {
   float* head_scr = nullptr;
   int64_t head_scr_rows = 0;
   bool head_ready = false;
-  int head_bps_qkv = 1, head_bps_full = 1;  // resident head_rows CTAs per SM
   // pr_selective_metrics: sort workspace for up to sel_cap scores, grown on demand
   void* sel_ws = nullptr;
   int64_t sel_cap = 0;

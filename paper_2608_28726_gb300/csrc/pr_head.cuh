@@ -7,19 +7,18 @@
 // The batch runs layer by layer, so that every step spreads over all SMs
 // whatever the mix of request lengths:
 //   head_embed   one CTA per request: H = W_in x_t + b_in + PE(t)
-//   head_rows    persistent CTAs over 64-row tiles of the whole batch: all the
-//                row-local work between two attentions, fused per tile --
+//   head_rows    one CTA per 128-row tile of the whole batch: all the row-local
+//                work between two attentions, fused per tile --
 //                O = A W_o^T + b_o, H = LN1(H + O), F = W_2 ReLU(W_1 H + b_1) + b_2,
 //                H = LN2(H + F), then the next layer's QKV = H W_qkv^T + b_qkv
-//   head_attn    one CTA per (request, head, 128-query block): softmax(Q K^T / 4) V
-//                on the tensor cores (tcgen05, TF32 operands split in two for
-//                fp32 accuracy), online softmax over 128-key chunks
+//   head_attn    one CTA per (request, head, 128-query block): softmax(Q K^T / 4) V,
+//                online softmax over 64-key chunks
 //   head_pool    one CTA per request: fixed-order mean over t, sigmoid layer
 // Activations live in a scratch of 256 floats per row (H | Q | K | V; the
 // attention output overwrites Q), which stays in L2 for batches of tens of
-// MB.  The row kernels run fp32 FMAs on the CUDA cores; the attention's two
-// contractions run on the tensor cores with each fp32 operand split into two
-// TF32 parts (three products per product), which keeps fp32-level accuracy.
+// MB.  Every contraction runs on the tensor cores with each fp32 operand split
+// into two TF32 parts (three products per product), which keeps fp32-level
+// accuracy; softmax, LayerNorm and the rest run in fp32 on the CUDA cores.
 // Every sum runs in a fixed order, so results are reproducible bit for bit.
 #pragma once
 
@@ -76,130 +75,9 @@ struct HeadArgs {
   const float* lnext;
 };
 
-// ---- shared-memory layout of head_rows (floats) ---------------------------------------
-constexpr int HTR = 64;                 // rows per tile
-constexpr int LDA64 = HD + 4;           // padded row of a 64-wide operand
-constexpr int LDA128 = HFF + 4;         // padded row of a 128-wide operand
-constexpr int HS_WQKV = 0;                             // W_qkv [192][68]
-constexpr int HS_VEC = HS_WQKV + 3 * HD * LDA64;       // b_qkv | b_o g1 be1 | b_1 | b_2 g2 be2
-constexpr int HS_VEC_N = 3 * HD + 3 * HD + HFF + 3 * HD;
-constexpr int HS_X0 = HS_VEC + HS_VEC_N;               // activation tile [64][68]
-constexpr int HS_X1 = HS_X0 + HTR * LDA64;             // activation tile [64][68]
-constexpr int HS_QKV_END = HS_X1 + HTR * LDA64;        // end of the QKV-only layout
-constexpr int HS_WO = HS_QKV_END;                      // W_o [64][68]
-constexpr int HS_W1 = HS_WO + HD * LDA64;              // W_1 [128][68]
-constexpr int HS_W2 = HS_W1 + HFF * LDA64;             // W_2 [64][132]
-constexpr int HS_HID = HS_W2 + HD * LDA128;            // hidden tile [64][132]
-constexpr int HS_END = HS_HID + HTR * LDA128;
-constexpr size_t HEAD_ROWS_SMEM_QKV = (size_t)HS_QKV_END * sizeof(float);
-constexpr size_t HEAD_ROWS_SMEM_FULL = (size_t)HS_END * sizeof(float);
-static_assert(HEAD_ROWS_SMEM_FULL <= 227 * 1024, "head_rows shared memory");
-// vector offsets inside HS_VEC
-constexpr int HV_BQKV = 0, HV_BO = 192, HV_G1 = 256, HV_BE1 = 320, HV_B1 = 384, HV_B2 = 512,
-              HV_G2 = 576, HV_BE2 = 640;
-
 constexpr int HR_QKV = 0, HR_MID = 1, HR_LAST = 2;
 
 // ---- small helpers ------------------------------------------------------------------------
-
-__device__ __forceinline__ void cp_async16(float* dst_smem, const float* src, bool valid) {
-  const uint32_t d = (uint32_t)__cvta_generic_to_shared(dst_smem);
-  const int n = valid ? 16 : 0;  // 0: the 16 bytes are zero-filled, nothing is read
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(d), "l"(src), "r"(n)
-               : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
-}
-
-// copy an N x K row-major matrix into shared rows of LD floats (16-byte pieces)
-template <int N, int K, int LD>
-__device__ __forceinline__ void stage_matrix(float* dst, const float* __restrict__ src) {
-  constexpr int Q = K / 4;
-  for (int c = threadIdx.x; c < N * Q; c += NT) {
-    const int n = c / Q, q = c - n * Q;
-    cp_async16(dst + n * LD + 4 * q, src + n * K + 4 * q, true);
-  }
-}
-
-// rows [row0, row0 + 64) of scratch columns [col, col + 64) into a [64][68]
-// tile; rows at or past n_rows are zero
-__device__ __forceinline__ void load_tile(float* dst, const float* scr, int64_t row0,
-                                          int64_t n_rows, int col) {
-  for (int c = threadIdx.x; c < HTR * (HD / 4); c += NT) {
-    const int r = c >> 4, q = c & 15;
-    const bool ok = row0 + r < n_rows;
-    const float* src = scr + (ok ? (row0 + r) : 0) * HSCR + col + 4 * q;
-    cp_async16(dst + r * LDA64 + 4 * q, src, ok);
-  }
-}
-
-// acc[i][j] = sum_k A[4 ty + i][k] * W[tx + 16 j][k] over k < K: thread
-// (tx, ty) = (tid % 16, tid / 16) owns rows 4 ty .. 4 ty + 3 and columns
-// tx + 16 j.  Operands are read as float4 along k; with rows padded by four
-// floats both reads are free of bank conflicts.  Each output keeps two
-// partial sums (even and odd k, in k order) in one packed fp32x2 FMA chain
-// and adds them at the end.
-template <int CPT, int K, int LDA, int LDW>
-__device__ __forceinline__ void tile_mm(const float* A, const float* W, float (&acc)[4][CPT],
-                                        int tx, int ty) {
-  float2 acc2[4][CPT];
-#pragma unroll
-  for (int i = 0; i < 4; ++i)
-#pragma unroll
-    for (int j = 0; j < CPT; ++j) acc2[i][j] = make_float2(0.f, 0.f);
-  const float* a0 = A + 4 * ty * LDA;
-  const float* w0 = W + tx * LDW;
-#pragma unroll 2
-  for (int k = 0; k < K; k += 4) {
-    float4 a[4];
-#pragma unroll
-    for (int i = 0; i < 4; ++i) a[i] = *reinterpret_cast<const float4*>(a0 + i * LDA + k);
-#pragma unroll
-    for (int j = 0; j < CPT; ++j) {
-      const float4 b = *reinterpret_cast<const float4*>(w0 + 16 * j * LDW + k);
-      const float2 b01 = make_float2(b.x, b.y), b23 = make_float2(b.z, b.w);
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        acc2[i][j] = __ffma2_rn(make_float2(a[i].x, a[i].y), b01, acc2[i][j]);
-        acc2[i][j] = __ffma2_rn(make_float2(a[i].z, a[i].w), b23, acc2[i][j]);
-      }
-    }
-  }
-#pragma unroll
-  for (int i = 0; i < 4; ++i)
-#pragma unroll
-    for (int j = 0; j < CPT; ++j) acc[i][j] = acc2[i][j].x + acc2[i][j].y;
-}
-
-// LayerNorm of the thread's four rows held as v[i][j] (columns tx + 16 j); a
-// row's 64 values sit in the 16 lanes of one half-warp
-__device__ __forceinline__ void rows_layer_norm(float (&v)[4][4], const float* g,
-                                                const float* be, int tx) {
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    float s = (v[i][0] + v[i][1]) + (v[i][2] + v[i][3]);
-#pragma unroll
-    for (int o = 8; o > 0; o >>= 1) s += __shfl_xor_sync(FULL, s, o);
-    const float mu = s * (1.f / HD);
-    float q = 0.f;
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      v[i][j] -= mu;
-      q = fmaf(v[i][j], v[i][j], q);
-    }
-#pragma unroll
-    for (int o = 8; o > 0; o >>= 1) q += __shfl_xor_sync(FULL, q, o);
-    const float inv = 1.f / sqrtf(q * (1.f / HD) + HLN_EPS);
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const int c = tx + 16 * j;
-      v[i][j] = fmaf(v[i][j] * inv, g[c], be[c]);
-    }
-  }
-}
 
 // Sinusoidal encoding of position t for the column pair (2i, 2i + 1):
 // sin(t f) and cos(t f), f = 10000^(-2i / 64).  The angle is kept in
@@ -283,154 +161,6 @@ __global__ void __launch_bounds__(NT) head_embed(const HeadArgs a) {
       *reinterpret_cast<float2*>(scr + (int64_t)t * HSCR + j0) = make_float2(v0 + sn, v1 + cs);
     }
   }
-}
-
-template <int MODE>
-__global__ void __launch_bounds__(NT, MODE == HR_QKV ? 2 : 1) head_rows(const HeadArgs a) {
-  extern __shared__ __align__(16) float hs[];
-  const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
-  const int64_t ntiles = (a.n_rows + HTR - 1) / HTR;
-  float* sV = hs + HS_VEC;
-  float* xin = hs + HS_X0;   // the tile's input (H for QKV-only, the attention output otherwise)
-  float* xmid = hs + HS_X1;  // LN1 output; then the next tile's input
-  const int in_col = (MODE == HR_QKV) ? 0 : HD;
-
-  // The weights do not depend on the previous kernel: their copies start
-  // before the dependency wait (with programmatic dependent launch they
-  // overlap the previous kernel's tail); the first tile is loaded after it.
-  pdl_trigger();
-  if (MODE != HR_QKV) {
-    stage_matrix<HD, HD, LDA64>(hs + HS_WO, a.lcur + HL_WO);
-    stage_matrix<HFF, HD, LDA64>(hs + HS_W1, a.lcur + HL_W1);
-    stage_matrix<HD, HFF, LDA128>(hs + HS_W2, a.lcur + HL_W2);
-  }
-  if (MODE != HR_LAST) stage_matrix<3 * HD, HD, LDA64>(hs + HS_WQKV, a.lnext + HL_WQKV);
-  pdl_wait();
-  load_tile(xin, a.scratch, (int64_t)blockIdx.x * HTR, a.n_rows, in_col);
-  cp_async_commit();
-  for (int i = tid; i < HS_VEC_N; i += NT) {
-    float v = 0.f;
-    if (i < 192) {
-      if (MODE != HR_LAST) v = __ldg(a.lnext + HL_BQKV + i);
-    } else if (MODE != HR_QKV) {
-      const float* L = a.lcur;
-      if (i < 256) v = __ldg(L + HL_BO + (i - 192));
-      else if (i < 320) v = __ldg(L + HL_G1 + (i - 256));
-      else if (i < 384) v = __ldg(L + HL_BE1 + (i - 320));
-      else if (i < 512) v = __ldg(L + HL_B1 + (i - 384));
-      else if (i < 576) v = __ldg(L + HL_B2 + (i - 512));
-      else if (i < 640) v = __ldg(L + HL_G2 + (i - 576));
-      else v = __ldg(L + HL_BE2 + (i - 640));
-    }
-    sV[i] = v;
-  }
-
-  for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
-    const int64_t row0 = tile * HTR;
-    const int64_t next = tile + gridDim.x;
-    float h[4][4];
-    if (MODE != HR_QKV) {
-      // residual H of the thread's rows (issued early, used after GEMM_o)
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const int64_t row = row0 + 4 * ty + i;
-        const bool ok = row < a.n_rows;
-        const float* src = a.scratch + (ok ? row : 0) * HSCR;
-#pragma unroll
-        for (int j = 0; j < 4; ++j) h[i][j] = ok ? src[tx + 16 * j] : 0.f;
-      }
-      cp_async_wait<0>();
-      __syncthreads();
-
-      // O = A W_o^T + b_o ; H = LN1(H + O)
-      float acc[4][4];
-      tile_mm<4, HD, LDA64, LDA64>(xin, hs + HS_WO, acc, tx, ty);
-#pragma unroll
-      for (int i = 0; i < 4; ++i)
-#pragma unroll
-        for (int j = 0; j < 4; ++j) h[i][j] += acc[i][j] + sV[HV_BO + tx + 16 * j];
-      rows_layer_norm(h, sV + HV_G1, sV + HV_BE1, tx);
-#pragma unroll
-      for (int i = 0; i < 4; ++i)
-#pragma unroll
-        for (int j = 0; j < 4; ++j) xmid[(4 * ty + i) * LDA64 + tx + 16 * j] = h[i][j];
-      __syncthreads();
-
-      // hidden = ReLU(H W_1^T + b_1)
-      {
-        float acc1[4][8];
-        tile_mm<8, HD, LDA64, LDA64>(xmid, hs + HS_W1, acc1, tx, ty);
-        float* hid = hs + HS_HID;
-#pragma unroll
-        for (int i = 0; i < 4; ++i)
-#pragma unroll
-          for (int j = 0; j < 8; ++j)
-            hid[(4 * ty + i) * LDA128 + tx + 16 * j] =
-                fmaxf(acc1[i][j] + sV[HV_B1 + tx + 16 * j], 0.f);
-      }
-      __syncthreads();
-      // xmid is free: prefetch the next tile's input into it
-      if (next < ntiles) load_tile(xmid, a.scratch, next * HTR, a.n_rows, in_col);
-      cp_async_commit();
-
-      // H = LN2(H + hidden W_2^T + b_2)
-      float acc2[4][4];
-      tile_mm<4, HFF, LDA128, LDA128>(hs + HS_HID, hs + HS_W2, acc2, tx, ty);
-#pragma unroll
-      for (int i = 0; i < 4; ++i)
-#pragma unroll
-        for (int j = 0; j < 4; ++j) h[i][j] += acc2[i][j] + sV[HV_B2 + tx + 16 * j];
-      rows_layer_norm(h, sV + HV_G2, sV + HV_BE2, tx);
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const int64_t row = row0 + 4 * ty + i;
-        if (row < a.n_rows) {
-          float* dst = a.scratch + row * HSCR;
-#pragma unroll
-          for (int j = 0; j < 4; ++j) dst[tx + 16 * j] = h[i][j];
-        }
-      }
-      if (MODE == HR_MID) {
-        // xin (consumed by GEMM_o two barriers ago) takes H for the QKV GEMM
-#pragma unroll
-        for (int i = 0; i < 4; ++i)
-#pragma unroll
-          for (int j = 0; j < 4; ++j) xin[(4 * ty + i) * LDA64 + tx + 16 * j] = h[i][j];
-        __syncthreads();
-      }
-    } else {
-      cp_async_wait<0>();
-      __syncthreads();
-      // xmid is free (nothing in this mode writes it): prefetch the next tile
-      if (next < ntiles) load_tile(xmid, a.scratch, next * HTR, a.n_rows, in_col);
-      cp_async_commit();
-    }
-
-    if (MODE != HR_LAST) {
-      // QKV = H W_qkv^T + b_qkv, written to scratch columns [64, 256), in two
-      // halves of 96 columns
-#pragma unroll
-      for (int half = 0; half < 2; ++half) {
-        float acc3[4][6];
-        tile_mm<6, HD, LDA64, LDA64>(xin, hs + HS_WQKV + half * 96 * LDA64, acc3, tx, ty);
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const int64_t row = row0 + 4 * ty + i;
-          if (row < a.n_rows) {
-            float* dst = a.scratch + row * HSCR + HD + half * 96;
-#pragma unroll
-            for (int j = 0; j < 6; ++j)
-              dst[tx + 16 * j] = acc3[i][j] + sV[HV_BQKV + half * 96 + tx + 16 * j];
-          }
-        }
-      }
-    }
-    __syncthreads();  // every read of xin is done before it becomes the prefetch buffer
-    float* t_ = xin;
-    xin = xmid;
-    xmid = t_;
-  }
-  cp_async_wait<0>();
 }
 
 // ---- head_attn: softmax(Q K^T / 4) V on the tensor cores ----------------------------
@@ -906,6 +636,430 @@ __global__ void __launch_bounds__(HA_M, HA_CTAS_PER_SM) head_attn(const HeadArgs
     ha_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
                  "r"(HA_TMEM_COLS)
+                 : "memory");
+  }
+}
+
+// ---- head_rows: the row-local block on the tensor cores -----------------------------
+//
+// CTA i takes the 128-row tile i of the whole batch; thread t owns row t and
+// TMEM lane t.  The block's four GEMMs run as tcgen05.mma kind::tf32 with the
+// same split as the attention (x = x_hi + x_lo, three products per product,
+// fp32-level accuracy): the activations are the A operand in TMEM (one column
+// per K value, written by their own row's thread), the weights the B operand
+// in shared memory (K-major canonical layout without swizzle), fp32
+// accumulators in TMEM.  Between the GEMMs each thread reads its row of the
+// accumulator and does the row-local work in registers, LayerNorm included:
+//   MID / LAST: O = A W_o^T (A: the attention output), H1 = LN1(H + O + b_o),
+//               F = ReLU(H1 W_1^T + b_1), H2 = LN2(H1 + F W_2^T + b_2) -> H
+//   MID / QKV:  QKV = H W_qkv^T + b_qkv -> Q, K, V (H = H2, or the embedding)
+// The weights are split and staged by the threads before the dependency wait
+// (they are inputs of the call), so with programmatic dependent launch they
+// overlap the previous kernel; W_qkv of a MID launch is loaded into registers
+// then and stored over W_o and W_1 once their GEMMs are done.  TMEM columns
+// (512, one CTA per SM): A operands hi / lo at 0-63 / 64-127 (K = 64) or
+// 0-127 / 128-255 (the hidden layer, K = 128); accumulators at 256 (W_1: 128
+// columns; W_2: 64; W_qkv: 192) and 384 (W_o: 64); H1 kept at 448-511 for
+// the second residual.  One elected thread issues the MMAs; every wait is
+// bounded.
+constexpr int HT_M = 128;                           // rows per tile = TMEM lanes
+constexpr int HT_NT = 2 * HT_M;                     // threads: two per row (column halves)
+constexpr uint32_t HT_TMEM_COLS = 512;
+constexpr uint32_t HT_A_HI = 0, HT_A_LO = 64;       // K = 64 A operands
+constexpr uint32_t HT_F_HI = 0, HT_F_LO = 128;      // the hidden layer (K = 128)
+constexpr uint32_t HT_D = 256;                      // W_1, W_2, W_qkv accumulators
+constexpr uint32_t HT_DO = 384;                     // W_o accumulator
+constexpr uint32_t HT_H1 = 448;                     // H1, fp32
+// shared memory (bytes): weights split in two, each matrix [N][K] hi then lo
+constexpr int HT_WO = 0;                            // W_o, 2 x 16 KB
+constexpr int HT_W1 = HT_WO + 2 * HD * HD * 4;      // W_1, 2 x 32 KB
+constexpr int HT_W2 = HT_W1 + 2 * HFF * HD * 4;     // W_2, 2 x 32 KB
+constexpr int HT_WEND = HT_W2 + 2 * HD * HFF * 4;   // 160 KB
+constexpr int HT_WQKV = 0;                          // W_qkv, 2 x 48 KB, over W_o and W_1
+static_assert(HT_WQKV + 2 * 3 * HD * HD * 4 <= HT_W2, "W_qkv fits over W_o and W_1");
+constexpr int HT_VEC = HT_WEND;                     // b_qkv | b_o g1 be1 | b_1 | b_2 g2 be2
+constexpr int HT_VEC_N = 3 * HD + 3 * HD + HFF + 3 * HD;
+// the tile's 64-wide input / output rows, staged for coalesced global access
+constexpr int HT_LDX = HD + 4;                      // padded row (floats): conflict-free per row
+constexpr int HT_X = HT_VEC + HT_VEC_N * 4;
+// the QKV output tile, staged over the weights once their GEMMs are done
+constexpr int HT_LDQ = 3 * HD + 4;
+constexpr int HT_Q = 0;
+static_assert(HT_Q + HT_M * HT_LDQ * 4 <= HT_VEC, "the QKV tile fits over the weights");
+constexpr int HT_XCH = HT_X + HT_M * HT_LDX * 4;    // row sums of the two halves [2][2][128]
+constexpr int HT_BAR = HT_XCH + 4 * HT_M * 4;       // mbarrier: MMA completion
+constexpr int HT_TSLOT = HT_BAR + 8;
+constexpr size_t HT_SMEM = HT_TSLOT + 8;
+static_assert(HT_SMEM <= 227 * 1024, "head_rows shared memory");
+static_assert(HT_BAR % 8 == 0, "mbarrier alignment");
+// vector offsets inside HT_VEC
+constexpr int HV_BQKV = 0, HV_BO = 192, HV_G1 = 256, HV_BE1 = 320, HV_B1 = 384, HV_B2 = 512,
+              HV_G2 = 576, HV_BE2 = 640;
+
+// tf32 instruction descriptor for M = 128 and the given N
+__host__ __device__ constexpr uint32_t ht_idesc(int n) {
+  return (1u << 4) | (2u << 7) | (2u << 10) | ((uint32_t)(n >> 3) << 17) |
+         ((uint32_t)(HT_M >> 4) << 24);
+}
+
+// float4 piece c of an [N][K] weight matrix: source row n, values 4 j .. 4 j + 3,
+// stored at float 4 c of the canonical layout (core matrices of 8 rows x 4
+// values, consecutive along K, 8-row groups one after another)
+template <int N, int K>
+__device__ __forceinline__ void ht_piece_src(int c, int& n, int& j) {
+  constexpr int Q = K / 4;
+  const int g = c >> 3;
+  n = ((g / Q) << 3) | (c & 7);
+  j = g % Q;
+}
+// this thread's pieces of W, raw, into the matrix's lo half (cp.async: all in
+// flight at once); ht_split_w then splits them in place once they have landed
+template <int N, int K>
+__device__ __forceinline__ void ht_copy_w(uint8_t* dst, const float* __restrict__ src) {
+  constexpr int IT = N * K / 4 / HT_NT;
+#pragma unroll
+  for (int i = 0; i < IT; ++i) {
+    const int c = threadIdx.x + i * HT_NT;
+    int n, j;
+    ht_piece_src<N, K>(c, n, j);
+    const uint32_t d = ha_saddr(dst + N * K * 4 + 16 * c);
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(d), "l"(src + n * K + 4 * j)
+                 : "memory");
+  }
+}
+template <int N, int K>
+__device__ __forceinline__ void ht_split_w(uint8_t* dst) {
+  constexpr int IT = N * K / 4 / HT_NT;
+#pragma unroll
+  for (int i = 0; i < IT; ++i) {
+    const int c = threadIdx.x + i * HT_NT;
+    float4* lo = reinterpret_cast<float4*>(dst + N * K * 4) + c;
+    float4 h, l;
+    ha_split(*lo, h, l);
+    reinterpret_cast<float4*>(dst)[c] = h;
+    *lo = l;
+  }
+}
+
+// D (+)= A B^T over K: A_hi / A_lo in TMEM columns, B = W (N rows, hi then lo)
+// in shared memory; three products per K step of 8
+template <int N, int K>
+__device__ __forceinline__ void ht_gemm(uint32_t d, uint32_t a_hi, uint32_t a_lo, uint32_t w) {
+  constexpr uint32_t SBO = (K / 4) * 128;
+  const uint64_t bh = ha_desc(w, SBO), bl = ha_desc(w + N * K * 4, SBO);
+#pragma unroll
+  for (int s = 0; s < K / 8; ++s) {
+    const uint64_t ko = (256u * s) >> 4;
+    ha_mma_ta(d, a_hi + 8u * s, bh + ko, ht_idesc(N), s);
+    ha_mma_ta(d, a_hi + 8u * s, bl + ko, ht_idesc(N), 1u);
+    ha_mma_ta(d, a_lo + 8u * s, bh + ko, ht_idesc(N), 1u);
+  }
+}
+
+// 32 values split in two and written to TMEM as A-operand columns
+__device__ __forceinline__ void ht_put_split(uint32_t t_hi, uint32_t t_lo, const float* v) {
+  float h[32], l[32];
+#pragma unroll
+  for (int j = 0; j < 32; ++j) {
+    h[j] = ha_hi(v[j]);
+    l[j] = v[j] - h[j];
+  }
+  ha_st32(t_hi, h);
+  ha_st32(t_lo, l);
+}
+
+// LayerNorm of a row whose 64 values are held by two threads, 32 each (half
+// hf holds columns 32 hf ..): the halves' partial sums meet in shared memory
+// and are added in half order, so both threads see the same statistics
+__device__ __forceinline__ void ht_layer_norm(float (&v)[32], const float* g, const float* be,
+                                              float* xch, int r, int hf) {
+  float s4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+  for (int j = 0; j < 32; ++j) s4[j & 3] += v[j];
+  xch[hf * HT_M + r] = (s4[0] + s4[1]) + (s4[2] + s4[3]);
+  __syncthreads();
+  const float mu = (xch[r] + xch[HT_M + r]) * (1.f / HD);
+  float q4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+  for (int j = 0; j < 32; ++j) {
+    v[j] -= mu;
+    q4[j & 3] = fmaf(v[j], v[j], q4[j & 3]);
+  }
+  xch[(2 + hf) * HT_M + r] = (q4[0] + q4[1]) + (q4[2] + q4[3]);
+  __syncthreads();
+  const float inv =
+      1.f / sqrtf((xch[2 * HT_M + r] + xch[3 * HT_M + r]) * (1.f / HD) + HLN_EPS);
+#pragma unroll
+  for (int j = 0; j < 32; ++j) v[j] = fmaf(v[j] * inv, g[32 * hf + j], be[32 * hf + j]);
+}
+
+// rows [row0, row0 + 128) of scratch columns [col, col + 64) into the staging
+// tile with cp.async, sixteen threads per row (coalesced); rows past the batch
+// are zero-filled
+__device__ __forceinline__ void ht_load_rows(uint8_t* sm, const float* scr, int64_t row0,
+                                             int64_t n_rows, int col) {
+#pragma unroll
+  for (int i = 0; i < HT_M * (HD / 4) / HT_NT; ++i) {
+    const int c = threadIdx.x + i * HT_NT;
+    const int r = c >> 4, q = c & 15;
+    const bool ok = row0 + r < n_rows;
+    const float* src = scr + (ok ? row0 + r : 0) * HSCR + col + 4 * q;
+    const uint32_t d = ha_saddr(sm + HT_X + (r * HT_LDX + 4 * q) * 4);
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(d), "l"(src),
+                 "r"(ok ? 16 : 0)
+                 : "memory");
+  }
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+// the staging tile back to scratch columns [col, col + 64), coalesced
+__device__ __forceinline__ void ht_store_rows(const uint8_t* sm, float* scr, int64_t row0,
+                                              int64_t n_rows, int col) {
+#pragma unroll
+  for (int i = 0; i < HT_M * (HD / 4) / HT_NT; ++i) {
+    const int c = threadIdx.x + i * HT_NT;
+    const int r = c >> 4, q = c & 15;
+    if (row0 + r < n_rows)
+      *reinterpret_cast<float4*>(scr + (row0 + r) * HSCR + col + 4 * q) =
+          *reinterpret_cast<const float4*>(sm + HT_X + (r * HT_LDX + 4 * q) * 4);
+  }
+}
+
+template <int MODE>
+__global__ void __launch_bounds__(HT_NT, 1) head_rows(const HeadArgs a) {
+  extern __shared__ __align__(16) uint8_t ht_sm[];
+  const int tid = threadIdx.x, warp = tid >> 5;
+  const int r = tid & (HT_M - 1);  // the row (TMEM lane) ...
+  const int hf = tid >> 7;         // ... and the half of its columns this thread takes
+  const uint32_t sb = ha_saddr(ht_sm);
+  const uint32_t bar = sb + HT_BAR;
+  float* sV = reinterpret_cast<float*>(ht_sm + HT_VEC);
+  float* xch = reinterpret_cast<float*>(ht_sm + HT_XCH);
+  // this thread's half of its row in the staging tile (8 pieces of 16 bytes)
+  float4* xrow = reinterpret_cast<float4*>(ht_sm + HT_X) + r * (HT_LDX / 4) + 8 * hf;
+  const int64_t row0 = (int64_t)blockIdx.x * HT_M;
+
+  // the weights and vectors are inputs of the call: staged before the wait,
+  // their copies in flight while the CTA takes its TMEM
+  constexpr int WQ_IT = 3 * HD * HD / 4 / HT_NT;
+  float4 wq_hold[MODE == HR_MID ? WQ_IT : 1];
+  if (MODE == HR_QKV) ht_copy_w<3 * HD, HD>(ht_sm + HT_WQKV, a.lnext + HL_WQKV);
+  if (MODE != HR_QKV) {
+    ht_copy_w<HD, HD>(ht_sm + HT_WO, a.lcur + HL_WO);
+    ht_copy_w<HFF, HD>(ht_sm + HT_W1, a.lcur + HL_W1);
+    ht_copy_w<HD, HFF>(ht_sm + HT_W2, a.lcur + HL_W2);
+  }
+  asm volatile("cp.async.commit_group;" ::: "memory");
+  if (MODE == HR_MID) {  // W_qkv waits in registers until W_o and W_1 are done
+#pragma unroll
+    for (int i = 0; i < WQ_IT; ++i) {
+      int n, j;
+      ht_piece_src<3 * HD, HD>(tid + i * HT_NT, n, j);
+      wq_hold[i] = __ldg(reinterpret_cast<const float4*>(a.lnext + HL_WQKV + n * HD) + j);
+    }
+  }
+  if (tid == 0) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(bar) : "memory");
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  // TMEM is taken before the next kernel may start (the trigger below), so a
+  // later kernel of the stream never holds the columns this CTA waits for
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     sb + HT_TSLOT),
+                 "r"(HT_TMEM_COLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+#pragma unroll
+  for (int k = 0; k < (HT_VEC_N + HT_NT - 1) / HT_NT; ++k) {
+    const int i = tid + k * HT_NT;
+    if (i >= HT_VEC_N) break;
+    float v = 0.f;
+    if (i < 192) {
+      if (MODE != HR_LAST) v = __ldg(a.lnext + HL_BQKV + i);
+    } else if (MODE != HR_QKV) {
+      const float* L = a.lcur;
+      if (i < 256) v = __ldg(L + HL_BO + (i - 192));
+      else if (i < 320) v = __ldg(L + HL_G1 + (i - 256));
+      else if (i < 384) v = __ldg(L + HL_BE1 + (i - 320));
+      else if (i < 512) v = __ldg(L + HL_B1 + (i - 384));
+      else if (i < 576) v = __ldg(L + HL_B2 + (i - 512));
+      else if (i < 640) v = __ldg(L + HL_G2 + (i - 576));
+      else v = __ldg(L + HL_BE2 + (i - 640));
+    }
+    sV[i] = v;
+  }
+  asm volatile("cp.async.wait_all;" ::: "memory");  // this thread's pieces, split in place
+  if (MODE == HR_QKV) ht_split_w<3 * HD, HD>(ht_sm + HT_WQKV);
+  if (MODE != HR_QKV) {
+    ht_split_w<HD, HD>(ht_sm + HT_WO);
+    ht_split_w<HFF, HD>(ht_sm + HT_W1);
+    ht_split_w<HD, HFF>(ht_sm + HT_W2);
+  }
+  ha_fence_before();
+  __syncthreads();
+  ha_fence_after();
+  const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(ht_sm + HT_TSLOT);
+  const uint32_t tq = tmem + ((uint32_t)((warp & 3) * 32) << 16);  // this warp's lane quarter
+  const uint32_t c32 = 32u * hf;                                    // this half's first column
+  pdl_trigger();
+  pdl_wait();
+
+  // the tile's input rows (the attention output over Q for MID / LAST, H for
+  // QKV), then this thread's half row as the first GEMM's A operand
+  ht_load_rows(ht_sm, a.scratch, row0, a.n_rows, MODE == HR_QKV ? 0 : HD);
+  asm volatile("cp.async.wait_all;" ::: "memory");
+  __syncthreads();
+  auto read_half = [&](float (&x)[32]) {
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const float4 v = xrow[j];
+      x[4 * j] = v.x;
+      x[4 * j + 1] = v.y;
+      x[4 * j + 2] = v.z;
+      x[4 * j + 3] = v.w;
+    }
+  };
+  {
+    float x[32];
+    read_half(x);
+    ht_put_split(tq + HT_A_HI + c32, tq + HT_A_LO + c32, x);
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+  }
+  uint32_t phase = 0;
+  bool ok = true;
+  // all threads' operands written -> one thread issues the MMAs -> every
+  // thread waits (bounded) for their completion; `during` runs meanwhile
+  auto mma_step = [&](auto issue, auto during) -> bool {
+    ha_fence_async();
+    ha_fence_before();
+    __syncthreads();
+    ha_fence_after();
+    if (tid == 0) {
+      issue();
+      ha_commit(bar);
+    }
+    during();
+    if (!__syncthreads_and(ha_wait(bar, phase))) return false;
+    phase ^= 1u;
+    ha_fence_after();
+    return true;
+  };
+  auto nothing = [] {};
+
+  if (MODE != HR_QKV) {
+    float h[32];
+    // O = A W_o^T, while the residual H comes into the staging tile
+    ok = mma_step(
+        [&] { ht_gemm<HD, HD>(tmem + HT_DO, tmem + HT_A_HI, tmem + HT_A_LO, sb + HT_WO); },
+        [&] { ht_load_rows(ht_sm, a.scratch, row0, a.n_rows, 0); });
+    asm volatile("cp.async.wait_all;" ::: "memory");
+    __syncthreads();
+    if (ok) {
+      // H1 = LN1(H + O + b_o): kept in TMEM for the second residual and split
+      // as the A operand of W_1
+      read_half(h);
+      {
+        float d[32];
+        ha_ld32(tq + HT_DO + c32, d);
+#pragma unroll
+        for (int j = 0; j < 32; ++j) h[j] += d[j] + sV[HV_BO + c32 + j];
+      }
+      ht_layer_norm(h, sV + HV_G1, sV + HV_BE1, xch, r, hf);
+      ha_st32(tq + HT_H1 + c32, h);
+      ht_put_split(tq + HT_A_HI + c32, tq + HT_A_LO + c32, h);
+      asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+      ok = mma_step(
+          [&] { ht_gemm<HFF, HD>(tmem + HT_D, tmem + HT_A_HI, tmem + HT_A_LO, sb + HT_W1); },
+          nothing);
+    }
+    if (ok) {
+      if (MODE == HR_MID) {  // W_o and W_1 are done: W_qkv over them
+#pragma unroll
+        for (int i = 0; i < WQ_IT; ++i) {
+          float4 hh, ll;
+          ha_split(wq_hold[i], hh, ll);
+          reinterpret_cast<float4*>(ht_sm + HT_WQKV)[tid + i * HT_NT] = hh;
+          reinterpret_cast<float4*>(ht_sm + HT_WQKV + 3 * HD * HD * 4)[tid + i * HT_NT] = ll;
+        }
+      }
+      // F = ReLU(H1 W_1^T + b_1), split as the A operand of W_2 (64 columns a half)
+#pragma unroll
+      for (int c = 0; c < HFF / 64; ++c) {
+        const uint32_t col = 64u * hf + 32u * c;
+        float d[32];
+        ha_ld32(tq + HT_D + col, d);
+#pragma unroll
+        for (int j = 0; j < 32; ++j) d[j] = fmaxf(d[j] + sV[HV_B1 + col + j], 0.f);
+        ht_put_split(tq + HT_F_HI + col, tq + HT_F_LO + col, d);
+      }
+      asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+      ok = mma_step(
+          [&] { ht_gemm<HD, HFF>(tmem + HT_D, tmem + HT_F_HI, tmem + HT_F_LO, sb + HT_W2); },
+          nothing);
+    }
+    if (ok) {
+      // H2 = LN2(H1 + F W_2^T + b_2) -> H, through the staging tile
+      {
+        float d[32], rr[32];
+        ha_ld32(tq + HT_D + c32, d);
+        ha_ld32(tq + HT_H1 + c32, rr);
+#pragma unroll
+        for (int j = 0; j < 32; ++j) h[j] = rr[j] + (d[j] + sV[HV_B2 + c32 + j]);
+      }
+      ht_layer_norm(h, sV + HV_G2, sV + HV_BE2, xch, r, hf);
+#pragma unroll
+      for (int j = 0; j < 8; ++j)
+        xrow[j] = make_float4(h[4 * j], h[4 * j + 1], h[4 * j + 2], h[4 * j + 3]);
+      if (MODE == HR_MID) {
+        ht_put_split(tq + HT_A_HI + c32, tq + HT_A_LO + c32, h);
+        asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+      }
+      __syncthreads();
+      ht_store_rows(ht_sm, a.scratch, row0, a.n_rows, 0);
+    }
+  }
+  if (MODE != HR_LAST && ok) {
+    // QKV = H W_qkv^T + b_qkv -> scratch columns [64, 256), through a
+    // staging tile over the weights (their MMAs are done); 96 columns a half
+    ok = mma_step(
+        [&] { ht_gemm<3 * HD, HD>(tmem + HT_D, tmem + HT_A_HI, tmem + HT_A_LO, sb + HT_WQKV); },
+        nothing);
+    if (ok) {
+      float4* qrow = reinterpret_cast<float4*>(ht_sm + HT_Q) + r * (HT_LDQ / 4);
+#pragma unroll
+      for (int c = 0; c < 3; ++c) {
+        const uint32_t col = 96u * hf + 32u * c;
+        float d[32];
+        ha_ld32(tq + HT_D + col, d);
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+          qrow[col / 4 + j] = make_float4(d[4 * j] + sV[HV_BQKV + col + 4 * j],
+                                          d[4 * j + 1] + sV[HV_BQKV + col + 4 * j + 1],
+                                          d[4 * j + 2] + sV[HV_BQKV + col + 4 * j + 2],
+                                          d[4 * j + 3] + sV[HV_BQKV + col + 4 * j + 3]);
+      }
+      __syncthreads();
+#pragma unroll 4
+      for (int i = 0; i < HT_M * (3 * HD / 4) / HT_NT; ++i) {  // 48 pieces of 16 bytes a row
+        const int f = tid + i * HT_NT;
+        const int rw = f / (3 * HD / 4), q = f - rw * (3 * HD / 4);
+        if (row0 + rw < a.n_rows)
+          *reinterpret_cast<float4*>(a.scratch + (row0 + rw) * HSCR + HD + 4 * q) =
+              reinterpret_cast<const float4*>(ht_sm + HT_Q)[rw * (HT_LDQ / 4) + q];
+      }
+    }
+  }
+  if (!ok) {
+    if (tid == 0) atomicOr(a.ctx_flags, HA_ERR_TIMEOUT);
+    ha_wait(bar, phase);  // the MMAs still pending, bounded as well
+  }
+  ha_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    ha_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                 "r"(HT_TMEM_COLS)
                  : "memory");
   }
 }

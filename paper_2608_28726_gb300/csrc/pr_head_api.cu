@@ -59,21 +59,11 @@ pr_status pr_head_score(pr_ctx* c, const float* feat, const uint32_t* row_flags,
   if (st != PR_OK) return st;
   if (!c->head_ready) {
     PR_CUDA(cudaFuncSetAttribute(prk::head_rows<prk::HR_QKV>,
-                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)prk::HEAD_ROWS_SMEM_QKV));
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, (int)prk::HT_SMEM));
     PR_CUDA(cudaFuncSetAttribute(prk::head_rows<prk::HR_MID>,
-                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)prk::HEAD_ROWS_SMEM_FULL));
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, (int)prk::HT_SMEM));
     PR_CUDA(cudaFuncSetAttribute(prk::head_rows<prk::HR_LAST>,
-                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)prk::HEAD_ROWS_SMEM_FULL));
-    int n = 0;
-    PR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, prk::head_rows<prk::HR_QKV>, prk::NT,
-                                                          prk::HEAD_ROWS_SMEM_QKV));
-    c->head_bps_qkv = n > 0 ? n : 1;
-    PR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, prk::head_rows<prk::HR_MID>, prk::NT,
-                                                          prk::HEAD_ROWS_SMEM_FULL));
-    c->head_bps_full = n > 0 ? n : 1;
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, (int)prk::HT_SMEM));
     PR_CUDA(cudaFuncSetAttribute(prk::head_attn, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)prk::HA_SMEM));
     c->head_ready = true;
@@ -117,14 +107,13 @@ pr_status pr_head_score(pr_ctx* c, const float* feat, const uint32_t* row_flags,
                    dim3((unsigned)n_req, prk::HES), blk, 0, s, c->overlap != 0, a);
   if (st != PR_OK) return st;
   if (n_rows > 0) {
-    const int64_t ntiles = (n_rows + prk::HTR - 1) / prk::HTR;
-    const unsigned g_qkv = (unsigned)std::min<int64_t>(ntiles, (int64_t)c->num_sms * c->head_bps_qkv);
-    const unsigned g_full =
-        (unsigned)std::min<int64_t>(ntiles, (int64_t)c->num_sms * c->head_bps_full);
+    // one CTA per 128-row tile (the row kernels hold all 512 TMEM columns of an SM)
+    const unsigned ntiles = (unsigned)((n_rows + prk::HT_M - 1) / prk::HT_M);
+    const dim3 rblk(prk::HT_NT);
     a.lcur = nullptr;
     a.lnext = layer(0);
-    st = launch_head(c, reinterpret_cast<const void*>(&prk::head_rows<prk::HR_QKV>), dim3(g_qkv), blk,
-                     prk::HEAD_ROWS_SMEM_QKV, s, true, a);
+    st = launch_head(c, reinterpret_cast<const void*>(&prk::head_rows<prk::HR_QKV>), dim3(ntiles),
+                     rblk, prk::HT_SMEM, s, true, a);
     if (st != PR_OK) return st;
     for (int l = 0; l < n_layers; ++l) {
       st = launch_head(c, reinterpret_cast<const void*>(&prk::head_attn),
@@ -136,7 +125,7 @@ pr_status pr_head_score(pr_ctx* c, const float* feat, const uint32_t* row_flags,
       a.lnext = last ? nullptr : layer(l + 1);
       const void* k = last ? reinterpret_cast<const void*>(&prk::head_rows<prk::HR_LAST>)
                            : reinterpret_cast<const void*>(&prk::head_rows<prk::HR_MID>);
-      st = launch_head(c, k, dim3(g_full), blk, prk::HEAD_ROWS_SMEM_FULL, s, true, a);
+      st = launch_head(c, k, dim3(ntiles), rblk, prk::HT_SMEM, s, true, a);
       if (st != PR_OK) return st;
     }
   }
