@@ -91,6 +91,15 @@ def test_head_requests_past_one_round_of_query_blocks(B, ctx):
     check(B, ctx, [2100, 1, 1300, 128], 2, seed=4350)
 
 
+def test_head_more_row_tiles_than_sms(B, ctx):
+    """About 30,000 rows: more 128-row tiles than SMs, so the row kernels run
+    in more than one wave of CTAs (each holds a whole SM's TMEM)."""
+    g = np.random.Generator(np.random.PCG64(4400))
+    lengths = g.integers(100, 200, size=200, endpoint=True)
+    assert lengths.sum() > 128 * 160
+    check(B, ctx, lengths, 2, seed=4401)
+
+
 def test_head_thresholds(B, ctx):
     g = np.random.Generator(np.random.PCG64(7))
     lengths = g.integers(1, 80, size=40, endpoint=True)
