@@ -237,6 +237,7 @@ def run_reference(args):
 
 # ---- timing, parity and the per-configuration records of the verifier ------------------
 
+T_START = time.time()
 MIN_TIMED_S = 1.5  # each timed measurement repeats its K-step loop until this much device time
 TOL_RTOL, TOL_ATOL, SHIP_BAND = 1e-4, 1e-5, 1e-6  # the verifier's parity bar
 
@@ -401,7 +402,15 @@ def measure_route_config(name, B, dev, stream, K, warm, world, sampler, threads,
         for _ in range(warm):
             step()
         torch.cuda.synchronize(dev)
-        return timed_repeats(step, K, stream, dev, world, B)
+        # steps per timed loop: K, or fewer for steps of many milliseconds (a
+        # loop of about half a second; the loop still repeats until
+        # MIN_TIMED_S of device time, at least three times)
+        t0 = time.perf_counter()
+        step()
+        torch.cuda.synchronize(dev)
+        k_eff = max(3, min(K, int(0.5 / max(time.perf_counter() - t0, 1e-6))))
+        state["k"] = k_eff
+        return timed_repeats(step, k_eff, stream, dev, world, B)
 
     iso, _, _ = timed(0)
     per, win, launches = timed(1)
@@ -460,7 +469,7 @@ def measure_route_config(name, B, dev, stream, K, warm, world, sampler, threads,
                         wl.n_rows, wl.vocab)
     rec = _route_rec(wl, name, desc, timing, ms, statistics.median(iso), stream_ms,
                      algorithmic_bytes(wl) if name != "tiny" else algorithmic_bytes(wl),
-                     wl.n_rows, world, clocks, launches, K, reps, parity, graph)
+                     wl.n_rows, world, clocks, launches, state["k"], reps, parity, graph)
     rec["generation_s"] = gen_s
     rec["l2"] = ("8 rotated copies (360 MB) larger than L2" if name == "tiny" else
                  "inputs (%.1f GB) larger than L2 (129 MB), no flush" % (need / 1e9))
@@ -640,6 +649,11 @@ def measure_noalloc(B, x, ch, wl, dev, stream, K, warm, world, n_req: int = 26):
 CONFIG_NAMES = {"c1": "tiny", "c3": "decode", "c4": "ragged", "c5": "wide"}
 
 
+def progress(msg: str):
+    """A progress line on stderr with the seconds since the bench started."""
+    print("[bench %.1f s] %s" % (time.time() - T_START, msg), file=sys.stderr, flush=True)
+
+
 def run_gb300(args):
     rank, world, local = dist_env()
     if world > 1:
@@ -672,6 +686,7 @@ def run_gb300(args):
     warm = max(3, args.warmup)
     min_s = min(0.05, MIN_TIMED_S) if args.skip_host else MIN_TIMED_S
 
+    progress("headline workload generated")
     # (1) isolated launches: one launch at a time (no overlap between steps)
     B.pr_ctx_set_option(ctx, B.PR_OPT_OVERLAP, 0)
     for _ in range(warm):
@@ -699,6 +714,7 @@ def run_gb300(args):
         B.pr_ctx_destroy(ctx)
         return 0
 
+    progress("headline timed")
     # end to end from pinned host memory through the public C ABI (without
     # the clock sampler's nvidia-smi process beside it)
     sampler.stop()
@@ -739,6 +755,7 @@ def run_gb300(args):
     peak, peak_src = measured_peak()
     cores = os.cpu_count() or 1
 
+    progress("end to end timed")
     line = None
     configs = {}
     noalloc = None
@@ -763,6 +780,7 @@ def run_gb300(args):
     B.pr_ctx_destroy(ctx)
     del x, ch
     torch.cuda.empty_cache()
+    progress("headline parity, CPU baseline and pr_route_noalloc done")
 
     if rank == 0 and world == 1 and args.configs != "none":
         for key in [k.strip() for k in args.configs.split(",") if k.strip()]:
@@ -777,6 +795,7 @@ def run_gb300(args):
             except (RuntimeError, torch.cuda.OutOfMemoryError) as e:
                 torch.cuda.empty_cache()
                 configs[key] = {"workload": name, "value": None, "error": str(e).splitlines()[0]}
+            progress("config %s (%s) done" % (key, name))
     sampler.stop()
 
     if rank == 0:
