@@ -1670,6 +1670,91 @@ def run_selective_workload(args):
     return 0
 
 
+def run_prescore_workload(args):
+    """The prompt pre-scorer of Eq. 2 on the host CPU (the paper keeps it off
+    the accelerator): a vocabulary fitted on 20,000 seeded synthetic prompts,
+    then batches of 100,000 prompts scored with all host threads."""
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    from paper_2608_28726_gb300 import build as prbuild
+    prbuild.build()
+    from paper_2608_28726_gb300 import binding as B
+    from oracle import prescore as op
+    docs, _ = W.prompts(20000, seed=9401)
+    prompts, images = W.prompts(100000, seed=9402)
+    t0 = time.perf_counter()
+    ps = B.pr_prescorer_fit(docs, min_df=2)
+    fit_s = time.perf_counter() - t0
+    V = B.pr_prescorer_vocab_size(ps)
+    w, b = W.prescore_weights(V)
+    cores = os.cpu_count() or 1
+    import ctypes
+    _bs, arr = B._texts(prompts)  # the host arrays the C call reads, built once
+    n = len(prompts)
+    p_lib, z_lib = np.empty(n, np.float32), np.empty(n, np.float32)
+
+    def call(n_threads=0, count=n):
+        st = B._lib.pr_prescorer_score(ps, ctypes.cast(arr, ctypes.c_void_p), images.ctypes.data,
+                                       count, w.ctypes.data, float(b), n_threads,
+                                       p_lib.ctypes.data, z_lib.ctypes.data)
+        assert st == 0, st
+
+    for _ in range(max(1, args.warmup)):
+        call()
+    reps, t_start = [], time.perf_counter()
+    while len(reps) < 3 or time.perf_counter() - t_start < MIN_TIMED_S:
+        t0 = time.perf_counter()
+        call()
+        reps.append(time.perf_counter() - t0)
+    sec = statistics.median(reps)
+    t0 = time.perf_counter()
+    call(n_threads=1, count=20000)
+    one_core = 20000 / (time.perf_counter() - t0)
+    # through the Python binding, its argument marshalling included
+    t0 = time.perf_counter()
+    p_api, _ = B.pr_prescorer_score(ps, prompts, images, w, b)
+    api_sec = time.perf_counter() - t0
+    call()
+    # parity and the float64 oracle's own speed on a sample
+    n_s = 2000
+    m = op.fit(docs, min_df=2)
+    t0 = time.perf_counter()
+    p_or, z_or = op.score(m, prompts[:n_s], images[:n_s], w.astype(np.float64), b)
+    oracle_s = time.perf_counter() - t0
+    z_or = np.asarray(z_or)
+    ok = bool(np.all(np.abs(z_lib[:n_s] - z_or) <= 1e-5 + 1e-6 * np.abs(z_or)) and
+              np.all(np.abs(p_lib[:n_s] - np.asarray(p_or)) <= 1e-6) and
+              np.array_equal(p_api, p_lib))
+    text_bytes = sum(len(x) for x in prompts)
+    B.pr_prescorer_destroy(ps)
+    line = {
+        "metric": "pre-scored prompts/sec (Eq. 2 prompt pre-scorer, host CPU)",
+        "value": len(prompts) / sec, "unit": "prompts/s", "n_gpus": 0, "steps": len(reps),
+        "warmup": max(1, args.warmup), "ms_per_step": sec * 1e3, "higher_is_better": True,
+        "scaling": "none", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": "100,000 seeded synthetic prompts (mean %.0f bytes), vocabulary "
+                               "of %d terms fitted on 20,000 others (min_df 2)" % (
+                                   text_bytes / len(prompts), V),
+                   "threads": cores, "fit_s": fit_s,
+                   "note": "host CPU by design (Section 3.1 keeps the pre-scorer off the "
+                           "accelerator): no GPU and no GPU roofline"},
+        "roofline": {"bound": "host", "achieved": text_bytes / sec / 1e6, "unit": "MB/s of prompt "
+                     "text", "peak": None, "frac": None, "one_core_prompts_per_s": one_core},
+        "cpu_baseline": {"value": n_s / oracle_s, "unit": "prompts/s", "cores": 1,
+                         "kind": "oracle", "sample": "prompts 0..%d, float64 Python oracle"
+                                                     % (n_s - 1)},
+        "e2e": {"value": len(prompts) / api_sec, "unit": "prompts/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0,
+                "api": "binding.pr_prescorer_score from Python strings (encoding and "
+                       "argument arrays included); value times the C call alone"},
+        "gpu_launches": 0,
+        "parity": {"prompts_checked": n_s, "ok": ok},
+    }
+    print(json.dumps(gate_on_parity(line)))
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -1678,7 +1763,7 @@ def main():
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--workload", default=WORKLOAD,
                     choices=["full", "tiny", "ragged", "wide", "decode", "head", "selective",
-                             "quantile", "lmhead"],
+                             "quantile", "lmhead", "prescore"],
                     help="full (default, the headline line), one of the other verifier "
                          "workloads, head (the transformer scorer head), quantile (the "
                          "quantile-summary MLP), selective (calibration and ranking metrics) "
@@ -1719,6 +1804,8 @@ def main():
         return run_head_workload(args)
     if args.workload == "selective":
         return run_selective_workload(args)
+    if args.workload == "prescore":
+        return run_prescore_workload(args)
     if args.workload == "quantile":
         return run_quantile_workload(args)
     if args.workload == "lmhead":

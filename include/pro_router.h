@@ -504,6 +504,54 @@ pr_status pr_route_noalloc(const void* logits, pr_dtype dt, int64_t n_rows, int6
                            int32_t n_req, const float* w, float b, float tau, float* score,
                            uint8_t* ship, uint32_t* req_flags, float* agg, void* stream);
 
+/* ---- the prompt pre-scorer (host CPU) ----------------------------------------------- */
+
+/*
+ * Pro-Router's first stage (Section 3.1, Eq. 2): before any token is
+ * generated a logistic regression over cheap prompt features guides the
+ * request, p_pre(x) = sigmoid(w . phi(x) + b), phi(x) = [TF-IDF vector of the
+ * prompt text, image count, prompt length].  The paper keeps this step off
+ * the accelerator; these calls run on the host CPU and touch no device.
+ *
+ * Readings of what the paper leaves open: a token is a maximal run of word
+ * bytes ([0-9A-Za-z_] and every byte >= 0x80) at least two bytes long, ASCII
+ * letters lowercased; the vocabulary is every term of the fitting corpus with
+ * document frequency >= min_df, columns in byte order of the terms; tf is the
+ * raw count, idf = ln((1 + n) / (1 + df)) + 1 (n documents), the row tf * idf
+ * is scaled to unit Euclidean length (a prompt without vocabulary terms has a
+ * zero row); the length is the prompt's token count (in or out of the
+ * vocabulary).  Sums run in double precision in ascending column order.
+ *
+ * pr_prescorer_fit: vocabulary and idf of n_docs NUL-terminated texts (host
+ *   pointers, read during the call only).  *out receives a new pre-scorer,
+ *   owned by the caller (pr_prescorer_destroy).  PR_ERR_INVALID_ARG for a
+ *   NULL text, n_docs < 0 or min_df < 1; PR_ERR_NO_MEMORY if an allocation fails.
+ * pr_prescorer_vocab_size: V, the number of TF-IDF columns (-1 for NULL).
+ * pr_prescorer_term: the term of a column (NUL-terminated, owned by the
+ *   pre-scorer), NULL outside [0, V).
+ * pr_prescorer_features: phi of one prompt: the nonzero TF-IDF entries in
+ *   ascending column order into columns / values (host arrays of cap
+ *   entries), their count into *nnz and the token count into *length;
+ *   PR_ERR_INVALID_ARG (with *nnz set) when cap is too small.
+ * pr_prescorer_score: for each of n prompts (host NUL-terminated texts) with
+ *   n_images[i] >= 0 images, score[i] = p_pre and, if logit is not NULL,
+ *   logit[i] = w . phi + b.  w: host float [V + 2] (V TF-IDF weights, then the
+ *   image-count weight, then the length weight).  n_threads host threads (0:
+ *   all hardware threads); the results do not depend on it.  Thread-safe for
+ *   concurrent calls on one pre-scorer (it is only read).
+ */
+typedef struct pr_prescorer pr_prescorer;
+pr_status pr_prescorer_fit(const char* const* docs, int32_t n_docs, int32_t min_df,
+                           pr_prescorer** out);
+void pr_prescorer_destroy(pr_prescorer* ps);
+int64_t pr_prescorer_vocab_size(const pr_prescorer* ps);
+const char* pr_prescorer_term(const pr_prescorer* ps, int64_t column);
+pr_status pr_prescorer_features(const pr_prescorer* ps, const char* prompt, int32_t cap,
+                                int32_t* columns, float* values, int32_t* nnz, int64_t* length);
+pr_status pr_prescorer_score(const pr_prescorer* ps, const char* const* prompts,
+                             const int32_t* n_images, int32_t n, const float* w, float b,
+                             int32_t n_threads, float* score, float* logit);
+
 /* ---- diagnostics ------------------------------------------------------------------ */
 
 /* Static description of a status code. */

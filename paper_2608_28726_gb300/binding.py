@@ -33,7 +33,9 @@ EXPORTS = (
     "pr_state_export", "pr_state_import", "pr_status_string", "pr_last_cuda_error",
     "pr_launch_count", "pr_route_noalloc", "pr_head_param_count", "pr_head_score",
     "pr_ctx_kernel_times", "pr_selective_metrics", "pr_quantile_score", "pr_lmhead_features",
-    "pr_selftest_wait", "pr_lmhead_decode_step", "pr_last_error",
+    "pr_selftest_wait", "pr_lmhead_decode_step", "pr_last_error", "pr_prescorer_fit",
+    "pr_prescorer_destroy", "pr_prescorer_vocab_size", "pr_prescorer_term",
+    "pr_prescorer_features", "pr_prescorer_score",
 )
 
 if not os.path.exists(LIB):
@@ -70,6 +72,10 @@ _SIGS = {
     "pr_head_score": [_P, _P, _P, _I64, _P, _I32, _P, _I32, _F32, _P, _P, _P, _P],
     "pr_state_export": [_P, _P, ctypes.POINTER(_SZ)],
     "pr_state_import": [_P, _P, _SZ],
+    "pr_prescorer_fit": [_P, _I32, _I32, ctypes.POINTER(_P)],
+    "pr_prescorer_features": [_P, ctypes.c_char_p, _I32, _P, _P, ctypes.POINTER(_I32),
+                              ctypes.POINTER(_I64)],
+    "pr_prescorer_score": [_P, _P, _P, _I32, _P, _F32, _I32, _P, _P],
 }
 for _name, _args in _SIGS.items():
     _fn = getattr(_lib, _name)
@@ -83,6 +89,12 @@ _lib.pr_launch_count.argtypes = []
 _lib.pr_launch_count.restype = ctypes.c_uint64
 _lib.pr_head_param_count.argtypes = [_I32]
 _lib.pr_head_param_count.restype = _I64
+_lib.pr_prescorer_destroy.argtypes = [_P]
+_lib.pr_prescorer_destroy.restype = None
+_lib.pr_prescorer_vocab_size.argtypes = [_P]
+_lib.pr_prescorer_vocab_size.restype = _I64
+_lib.pr_prescorer_term.argtypes = [_P, _I64]
+_lib.pr_prescorer_term.restype = ctypes.c_char_p
 
 
 class PRError(RuntimeError):
@@ -561,3 +573,63 @@ def pr_selftest_wait(ctx, limit_ns: int) -> bool:
     done = _I32(-1)
     _check(_lib.pr_selftest_wait(ctx, int(limit_ns), ctypes.byref(done)), "pr_selftest_wait")
     return done.value == 1
+
+
+# ---- the prompt pre-scorer (host CPU; Section 3.1, Eq. 2) ---------------------------------
+
+def _texts(texts):
+    """Host array of NUL-terminated byte strings (kept alive by the caller)."""
+    bs = [t.encode() if isinstance(t, str) else bytes(t) for t in texts]
+    if any(b"\0" in b for b in bs):
+        raise PRError(PR_ERR_INVALID_ARG, "prescorer", "a text holds a NUL byte")
+    arr = (ctypes.c_char_p * max(1, len(bs)))(*bs)
+    return bs, arr
+
+
+def pr_prescorer_fit(docs, min_df: int = 1):
+    """Vocabulary and smoothed idf of a corpus (str or bytes texts)."""
+    bs, arr = _texts(docs)
+    out = _P()
+    _check(_lib.pr_prescorer_fit(ctypes.cast(arr, _P), len(bs), int(min_df), ctypes.byref(out)),
+           "pr_prescorer_fit")
+    return out.value
+
+
+def pr_prescorer_destroy(ps):
+    _lib.pr_prescorer_destroy(ps)
+
+
+def pr_prescorer_vocab_size(ps) -> int:
+    return int(_lib.pr_prescorer_vocab_size(ps))
+
+
+def pr_prescorer_term(ps, column: int):
+    return _lib.pr_prescorer_term(ps, int(column))
+
+
+def pr_prescorer_features(ps, prompt, cap: int = 4096):
+    """(columns int32, values float32, token count) of one prompt."""
+    p = prompt.encode() if isinstance(prompt, str) else bytes(prompt)
+    cols = np.empty(max(1, cap), np.int32)
+    vals = np.empty(max(1, cap), np.float32)
+    nnz, length = _I32(), _I64()
+    _check(_lib.pr_prescorer_features(ps, p, int(cap), cols.ctypes.data, vals.ctypes.data,
+                                      ctypes.byref(nnz), ctypes.byref(length)),
+           "pr_prescorer_features")
+    return cols[:nnz.value].copy(), vals[:nnz.value].copy(), int(length.value)
+
+
+def pr_prescorer_score(ps, prompts, n_images, w, b: float, n_threads: int = 0):
+    """(p_pre float32 [n], logit float32 [n]) on the host; w: float32 [V + 2]."""
+    bs, arr = _texts(prompts)
+    n = len(bs)
+    img = np.ascontiguousarray(n_images, np.int32)
+    wv = np.ascontiguousarray(w, np.float32)
+    if img.shape != (n,) or wv.shape != (pr_prescorer_vocab_size(ps) + 2,):
+        raise PRError(PR_ERR_INVALID_ARG, "pr_prescorer_score", "n_images or w has the wrong size")
+    score = np.empty(max(1, n), np.float32)
+    logit = np.empty(max(1, n), np.float32)
+    _check(_lib.pr_prescorer_score(ps, ctypes.cast(arr, _P), img.ctypes.data, n, wv.ctypes.data,
+                                   float(b), int(n_threads), score.ctypes.data, logit.ctypes.data),
+           "pr_prescorer_score")
+    return score[:n], logit[:n]

@@ -1,0 +1,221 @@
+// The prompt pre-scorer (Pro-Router, Section 3.1, Eq. 2) on the host CPU, as
+// the paper keeps it off the accelerator:
+//
+//   p_pre(x) = sigmoid(w . phi(x) + b),  phi(x) = [TF-IDF(prompt), image count, length]
+//
+// pr_prescorer_fit builds the vocabulary and the smoothed idf of a corpus;
+// pr_prescorer_score scores a batch of prompts, in parallel over host
+// threads.  Readings of what the paper leaves open (the same as the float64
+// reference used by the tests):
+//   * a token is a maximal run of word bytes ([0-9A-Za-z_] and every byte >=
+//     0x80) at least two bytes long, ASCII letters lowercased;
+//   * the vocabulary holds every corpus term with document frequency >=
+//     min_df, columns in byte order of the terms;
+//   * tf = raw count, idf = ln((1 + n) / (1 + df)) + 1, the row scaled to unit
+//     Euclidean length (a row without vocabulary terms stays zero);
+//   * length = the prompt's token count; w = V TF-IDF weights, then the
+//     image-count weight, then the length weight.
+// Sums run in double precision in ascending column order.
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <new>
+#include <string>
+#include <thread>
+#include <unordered_map>
+#include <unordered_set>
+#include <utility>
+#include <vector>
+
+#include "pro_router.h"
+
+struct pr_prescorer {
+  std::vector<std::string> terms;                   // column -> term, byte order
+  std::unordered_map<std::string, int32_t> column;  // term -> column
+  std::vector<double> idf;
+  int64_t n_docs = 0;
+};
+
+namespace {
+
+inline bool word_byte(unsigned char c) {
+  return (c >= '0' && c <= '9') || (c >= 'a' && c <= 'z') || (c >= 'A' && c <= 'Z') || c == '_' ||
+         c >= 0x80;
+}
+
+// calls f(token) for every token of the NUL-terminated text
+template <class F>
+void for_each_token(const char* text, F&& f) {
+  std::string tok;
+  for (const unsigned char* p = reinterpret_cast<const unsigned char*>(text);; ++p) {
+    const unsigned char c = *p;
+    if (c != 0 && word_byte(c)) {
+      tok.push_back((c >= 'A' && c <= 'Z') ? char(c + ('a' - 'A')) : char(c));
+      continue;
+    }
+    if (tok.size() >= 2) f(tok);
+    tok.clear();
+    if (c == 0) break;
+  }
+}
+
+struct Row {
+  std::vector<std::pair<int32_t, double>> v;  // (column, value), ascending column
+  int64_t length = 0;
+};
+
+void tfidf_row(const pr_prescorer& ps, const char* prompt, Row& row) {
+  std::unordered_map<int32_t, int64_t> counts;
+  row.length = 0;
+  for_each_token(prompt, [&](const std::string& t) {
+    ++row.length;
+    const auto it = ps.column.find(t);
+    if (it != ps.column.end()) ++counts[it->second];
+  });
+  row.v.clear();
+  row.v.reserve(counts.size());
+  for (const auto& kc : counts) row.v.emplace_back(kc.first, (double)kc.second * ps.idf[kc.first]);
+  std::sort(row.v.begin(), row.v.end());
+  double ss = 0.0;
+  for (const auto& e : row.v) ss += e.second * e.second;
+  if (ss > 0.0) {
+    const double inv = 1.0 / std::sqrt(ss);
+    for (auto& e : row.v) e.second *= inv;
+  }
+}
+
+double row_logit(const pr_prescorer& ps, const Row& row, int32_t n_images, const float* w,
+                 float b) {
+  const size_t V = ps.terms.size();
+  double z = (double)b;
+  for (const auto& e : row.v) z += (double)w[e.first] * e.second;
+  z += (double)w[V] * (double)n_images + (double)w[V + 1] * (double)row.length;
+  return z;
+}
+
+double sigmoid(double z) {
+  if (z >= 0.0) return 1.0 / (1.0 + std::exp(-z));
+  const double e = std::exp(z);
+  return e / (1.0 + e);
+}
+
+}  // namespace
+
+extern "C" {
+
+pr_status pr_prescorer_fit(const char* const* docs, int32_t n_docs, int32_t min_df,
+                           pr_prescorer** out) {
+  if (!out) return PR_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (n_docs < 0 || (n_docs > 0 && !docs) || min_df < 1) return PR_ERR_INVALID_ARG;
+  for (int32_t i = 0; i < n_docs; ++i)
+    if (!docs[i]) return PR_ERR_INVALID_ARG;
+  try {
+    std::unordered_map<std::string, int64_t> df;
+    std::unordered_set<std::string> seen;
+    for (int32_t i = 0; i < n_docs; ++i) {
+      seen.clear();
+      for_each_token(docs[i], [&](const std::string& t) {
+        if (seen.insert(t).second) ++df[t];
+      });
+    }
+    pr_prescorer* ps = new pr_prescorer;
+    for (const auto& tc : df)
+      if (tc.second >= min_df) ps->terms.push_back(tc.first);
+    std::sort(ps->terms.begin(), ps->terms.end());  // byte order (std::string compares as unsigned char)
+    ps->idf.resize(ps->terms.size());
+    ps->column.reserve(ps->terms.size());
+    for (size_t j = 0; j < ps->terms.size(); ++j) {
+      ps->column.emplace(ps->terms[j], (int32_t)j);
+      ps->idf[j] = std::log((1.0 + (double)n_docs) / (1.0 + (double)df[ps->terms[j]])) + 1.0;
+    }
+    ps->n_docs = n_docs;
+    *out = ps;
+    return PR_OK;
+  } catch (const std::bad_alloc&) {
+    return PR_ERR_NO_MEMORY;
+  }
+}
+
+void pr_prescorer_destroy(pr_prescorer* ps) { delete ps; }
+
+int64_t pr_prescorer_vocab_size(const pr_prescorer* ps) {
+  return ps ? (int64_t)ps->terms.size() : -1;
+}
+
+const char* pr_prescorer_term(const pr_prescorer* ps, int64_t column) {
+  if (!ps || column < 0 || column >= (int64_t)ps->terms.size()) return nullptr;
+  return ps->terms[(size_t)column].c_str();
+}
+
+pr_status pr_prescorer_features(const pr_prescorer* ps, const char* prompt, int32_t cap,
+                                int32_t* columns, float* values, int32_t* nnz, int64_t* length) {
+  if (!ps || !prompt || cap < 0 || !nnz || !length || (cap > 0 && (!columns || !values)))
+    return PR_ERR_INVALID_ARG;
+  try {
+    Row row;
+    tfidf_row(*ps, prompt, row);
+    *nnz = (int32_t)row.v.size();
+    *length = row.length;
+    if ((int64_t)row.v.size() > cap) return PR_ERR_INVALID_ARG;
+    for (size_t i = 0; i < row.v.size(); ++i) {
+      columns[i] = row.v[i].first;
+      values[i] = (float)row.v[i].second;
+    }
+    return PR_OK;
+  } catch (const std::bad_alloc&) {
+    return PR_ERR_NO_MEMORY;
+  }
+}
+
+pr_status pr_prescorer_score(const pr_prescorer* ps, const char* const* prompts,
+                             const int32_t* n_images, int32_t n, const float* w, float b,
+                             int32_t n_threads, float* score, float* logit) {
+  if (!ps || n < 0 || !w || n_threads < 0) return PR_ERR_INVALID_ARG;
+  if (n == 0) return PR_OK;
+  if (!prompts || !n_images || !score) return PR_ERR_INVALID_ARG;
+  for (int32_t i = 0; i < n; ++i)
+    if (!prompts[i] || n_images[i] < 0) return PR_ERR_INVALID_ARG;
+  int nt = n_threads > 0 ? n_threads : (int)std::max(1u, std::thread::hardware_concurrency());
+  nt = std::max(1, std::min(nt, n));
+  bool failed = false;
+  auto work = [&](int32_t lo, int32_t hi, bool* fail) {
+    try {
+      Row row;
+      for (int32_t i = lo; i < hi; ++i) {
+        tfidf_row(*ps, prompts[i], row);
+        const double z = row_logit(*ps, row, n_images[i], w, b);
+        score[i] = (float)sigmoid(z);
+        if (logit) logit[i] = (float)z;
+      }
+    } catch (const std::bad_alloc&) {
+      *fail = true;
+    }
+  };
+  if (nt == 1) {
+    work(0, n, &failed);
+    return failed ? PR_ERR_NO_MEMORY : PR_OK;
+  }
+  std::vector<std::thread> th;
+  std::vector<char> fails((size_t)nt, 0);
+  try {
+    th.reserve((size_t)nt);
+    for (int t = 0; t < nt; ++t) {
+      const int32_t lo = (int32_t)((int64_t)n * t / nt), hi = (int32_t)((int64_t)n * (t + 1) / nt);
+      th.emplace_back([&, lo, hi, t] {
+        bool f = false;
+        work(lo, hi, &f);
+        fails[(size_t)t] = f;
+      });
+    }
+  } catch (...) {
+    for (auto& x : th) x.join();
+    return PR_ERR_NO_MEMORY;
+  }
+  for (auto& x : th) x.join();
+  for (char f : fails)
+    if (f) return PR_ERR_NO_MEMORY;
+  return PR_OK;
+}
+
+}  // extern "C"

@@ -373,3 +373,79 @@ def lmhead_inputs(n_rows: int, d: int = 3584, vocab: int = 151936, seed: int = 8
                          (2.0 / d ** 0.5)).to(torch.bfloat16)
     chosen = torch.randint(0, vocab, (n_rows,), generator=g, device=dev, dtype=torch.int32)
     return hidden, weight, chosen
+
+
+# ---- prompts for the pre-scorer (Section 3.1, Eq. 2) --------------------------------------
+#
+# The paper's prompts (benchmark questions with images) are not available;
+# these stand in for them: a seeded vocabulary of VOCAB pseudo-words (random
+# lowercase strings of 3-10 letters), words drawn with Zipf(1.07) frequencies
+# over the vocabulary's ranks, prompt lengths clip(round(lognormal(ln 30,
+# 0.7)), 3, 400) words, about 10% of words capitalised, punctuation after 10%
+# of words, a number token for 3%, a one-letter word (which no token keeps)
+# for 5%, a word with a non-ASCII letter for 1%; image counts 0 (30%), 1
+# (55%), 2 (10%) or 3-5 (5%).
+
+PROMPT_VOCAB = 20000
+
+
+def _pseudo_words(n: int, seed: int) -> list[bytes]:
+    """n distinct random lowercase words of 3-10 letters (a drawn length is
+    raised by one after every eight collisions, so the loop always ends)."""
+    g = np.random.Generator(np.random.PCG64(seed))
+    lens = g.integers(3, 10, size=n, endpoint=True)
+    letters = np.frombuffer(b"abcdefghijklmnopqrstuvwxyz", np.uint8)
+    words, seen = [], set()
+    for L in lens:
+        tries = 0
+        while True:
+            w = bytes(letters[g.integers(0, 26, size=int(L) + tries // 8)])
+            if w not in seen:
+                seen.add(w)
+                words.append(w)
+                break
+            tries += 1
+    return words
+
+
+def prompts(n: int, seed: int = 9001) -> tuple[list[bytes], np.ndarray]:
+    """n seeded synthetic prompts (UTF-8 bytes) and their image counts."""
+    words = _pseudo_words(PROMPT_VOCAB, seed + 1)
+    ranks = np.arange(1, PROMPT_VOCAB + 1, dtype=np.float64)
+    pz = ranks ** -1.07
+    pz /= pz.sum()
+    g = np.random.Generator(np.random.PCG64(seed))
+    lengths = np.clip(np.round(np.exp(g.normal(np.log(30.0), 0.7, size=n))), 3, 400).astype(int)
+    out = []
+    for L in lengths:
+        idx = g.choice(PROMPT_VOCAB, size=L, p=pz)
+        u = g.random((L, 6))
+        parts = []
+        for k in range(L):
+            w = words[idx[k]]
+            if u[k, 0] < 0.10:
+                w = w[:1].upper() + w[1:]
+            if u[k, 1] < 0.03:
+                w = b"%d" % int(u[k, 2] * 1000)
+            elif u[k, 1] < 0.08:
+                w = w[:1]
+            elif u[k, 1] < 0.09:
+                w = w + "é".encode()
+            if u[k, 3] < 0.10:
+                w = w + b".,?!:;"[int(u[k, 4] * 6):][:1]
+            parts.append(w)
+        out.append(b" ".join(parts))
+    c = g.random(n)
+    images = np.where(c < 0.30, 0, np.where(c < 0.85, 1, np.where(c < 0.95, 2,
+                                                                   3 + (c * 1000).astype(int) % 3)))
+    return out, images.astype(np.int32)
+
+
+def prescore_weights(vocab: int, seed: int = 9101) -> tuple[np.ndarray, float]:
+    """Stand-in weights of the pre-scorer's logistic regression (the trained
+    ones are not available): V TF-IDF weights N(0, 1), the image-count weight
+    N(0, 0.3^2), the length weight N(0, 0.01^2), then b ~ N(0, 0.1^2)."""
+    g = np.random.Generator(np.random.PCG64(seed))
+    w = np.concatenate([g.normal(0.0, 1.0, vocab), g.normal(0.0, 0.3, 1),
+                        g.normal(0.0, 0.01, 1)]).astype(np.float32)
+    return w, float(g.normal(0.0, 0.1))
