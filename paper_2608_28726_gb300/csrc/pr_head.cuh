@@ -237,12 +237,6 @@ __device__ __forceinline__ uint32_t ha_saddr(const void* p) {
 __device__ __forceinline__ uint32_t ha_kmaj(int row, int j, int sbo) {
   return (uint32_t)((row >> 3) * sbo + j * 128 + (row & 7) * 16);
 }
-// byte offset of (row, key k) in the swizzled [V_hi | V_lo]^T operand
-__device__ __forceinline__ uint32_t ha_vt(int row, int k) {
-  const int r = row & 7, c = (k >> 2) & 7;
-  return (uint32_t)(HA_VT + (k >> 5) * HA_VT_ATOM + (row >> 3) * 1024 + r * 128 + ((c ^ r) << 4) +
-                    (k & 3) * 4);
-}
 // matrix descriptors: start >> 4 in bits 0-13, leading byte offset >> 4 in
 // bits 16-29, stride byte offset >> 4 in bits 32-45, version 1 in bits
 // 46-47, layout in bits 61-63 (0: no swizzle, 2: 128-byte swizzle)
@@ -323,7 +317,7 @@ __device__ __forceinline__ bool ha_wait(uint32_t bar, uint32_t parity) {
     if ((i & 255u) == 0u && ha_clock() - t0 > HA_WAIT_NS) return false;
   }
 }
-// 32 / 16 consecutive fp32 columns of this warp's 32 TMEM lanes (lane = row)
+// 32 consecutive fp32 columns of this warp's 32 TMEM lanes (lane = row)
 __device__ __forceinline__ void ha_ld32(uint32_t taddr, float (&v)[32]) {
   uint32_t r[32];
   asm volatile(
@@ -339,19 +333,6 @@ __device__ __forceinline__ void ha_ld32(uint32_t taddr, float (&v)[32]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 #pragma unroll
   for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
-}
-__device__ __forceinline__ void ha_ld16(uint32_t taddr, float (&v)[16]) {
-  uint32_t r[16];
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
-      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
-        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
-        "=r"(r[14]), "=r"(r[15])
-      : "r"(taddr));
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-#pragma unroll
-  for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(r[j]);
 }
 __device__ __forceinline__ void ha_st32(uint32_t taddr, const float (&v)[32]) {
   asm volatile(
