@@ -30,6 +30,7 @@ constexpr int SEL_TILE = SEL_NT * SEL_IPT;  // items per tile
 constexpr int SR_IPT = 16;                  // items per thread in the radix passes: longer
 constexpr int SR_TILE = SEL_NT * SR_IPT;    // digit runs per tile, half the tile counts
 constexpr int SEL_RADIX = 256;
+constexpr int SEL_FEW_DIGITS = 16;          // a pass with at most this many digits ranks by match.any
 constexpr uint32_t SEL_NONFINITE = 0xffffffffu;
 
 struct SelResult {        // written by sel_finish, copied to the host
@@ -192,26 +193,38 @@ __global__ void __launch_bounds__(SEL_NT) sel_scan_digit(uint32_t* __restrict__ 
 // takes tiles b, b + grid, b + 2 grid, ..., and loads the next tile's keys,
 // labels and offsets while it ranks and writes the current one.  Warp w owns
 // items [w * 512, (w + 1) * 512) of a tile in 16 rounds of 32 consecutive
-// items; the lanes holding the same digit in a round are found with
-// match.any and ranked by lane, rounds in order, so the tile order of equal
-// digits is kept.  The tile is then laid out in shared memory in digit order
+// items; the lanes holding the same digit in a round are found (with
+// match.any, or with eight ballots, see sel_scatter) and ranked by lane,
+// rounds in order, so the tile order of equal digits is kept.  The tile is then laid out in shared memory in digit order
 // and written out in that order: each digit's run goes to consecutive
 // addresses.  Indices are 32-bit (n < 2^31).
-__global__ void __launch_bounds__(SEL_NT) sel_scatter(const uint32_t* __restrict__ key_in,
+struct SelScatterSmem {
+  uint32_t wcnt[SEL_NT / 32][SEL_RADIX];
+  uint32_t gbase[SEL_RADIX];  // global position of the tile's first item of digit d,
+                              // minus the digit's offset inside the tile
+  uint32_t toff[SEL_RADIX];   // offset of digit d inside the tile
+  uint32_t ws[SEL_NT / 32], ws2[SEL_NT / 32];
+  uint32_t sk[SR_TILE];
+  uint8_t sv[SR_TILE];
+};
+
+template <bool BALLOT>
+__device__ __forceinline__ void sel_scatter_body(const uint32_t* __restrict__ key_in,
                                                       const uint8_t* __restrict__ val_in,
                                                       int64_t n64, int shift,
                                                       const uint32_t* __restrict__ counts,
                                                       int64_t ntiles64,
                                                       const uint32_t* __restrict__ total,
                                                       uint32_t* __restrict__ key_out,
-                                                      uint8_t* __restrict__ val_out) {
-  __shared__ uint32_t wcnt[SEL_NT / 32][SEL_RADIX];
-  __shared__ uint32_t gbase[SEL_RADIX];  // global position of the tile's first item of digit d,
-                                         // minus the digit's offset inside the tile
-  __shared__ uint32_t toff[SEL_RADIX];   // offset of digit d inside the tile
-  __shared__ uint32_t ws[SEL_NT / 32], ws2[SEL_NT / 32];
-  __shared__ uint32_t sk[SR_TILE];
-  __shared__ uint8_t sv[SR_TILE];
+                                                      uint8_t* __restrict__ val_out,
+                                                      SelScatterSmem& sh) {
+  auto& wcnt = sh.wcnt;
+  auto& gbase = sh.gbase;
+  auto& toff = sh.toff;
+  auto& ws = sh.ws;
+  auto& ws2 = sh.ws2;
+  auto& sk = sh.sk;
+  auto& sv = sh.sv;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const uint32_t n = (uint32_t)n64, ntiles = (uint32_t)ntiles64;
   constexpr int PER_WARP = SR_TILE / (SEL_NT / 32);
@@ -249,7 +262,18 @@ __global__ void __launch_bounds__(SEL_NT) sel_scatter(const uint32_t* __restrict
     for (int r = 0; r < SR_IPT; ++r) {
       const bool ok = base + r * 32 + lane < n;
       const uint32_t d = (k[r] >> shift) & 0xff;
-      const unsigned peers = __match_any_sync(FULL, ok ? d : SEL_RADIX);  // SEL_RADIX: no item
+      unsigned peers;  // the lanes holding digit d (lanes without an item group apart)
+      if (!BALLOT) {
+        peers = __match_any_sync(FULL, ok ? d : SEL_RADIX);  // SEL_RADIX: no item
+      } else {
+        peers = __ballot_sync(FULL, ok);
+        if (!ok) peers = ~peers;
+#pragma unroll
+        for (int bit = 0; bit < 8; ++bit) {
+          const unsigned bal = __ballot_sync(FULL, (d >> bit) & 1u);
+          peers &= ((d >> bit) & 1u) ? bal : ~bal;
+        }
+      }
       const uint32_t rank = __popc(peers & lt);
       const uint32_t before = ok ? wcnt[warp][d] : 0u;
       __syncwarp();
@@ -318,6 +342,28 @@ __global__ void __launch_bounds__(SEL_NT) sel_scatter(const uint32_t* __restrict
     }
     bt = btn;
   }
+}
+
+// The warp ranking's method: match.any costs more the more distinct digits a
+// warp holds, eight ballots (one per digit bit) cost the same for any mix.
+// A pass whose keys hold few digits (the top byte of scores that share an
+// exponent range) takes match.any, the others the ballots; the choice is one
+// branch around the whole body, so each method compiles on its own.
+__global__ void __launch_bounds__(SEL_NT) sel_scatter(const uint32_t* __restrict__ key_in,
+                                                      const uint8_t* __restrict__ val_in,
+                                                      int64_t n64, int shift,
+                                                      const uint32_t* __restrict__ counts,
+                                                      int64_t ntiles64,
+                                                      const uint32_t* __restrict__ total,
+                                                      uint32_t* __restrict__ key_out,
+                                                      uint8_t* __restrict__ val_out) {
+  __shared__ SelScatterSmem sh;
+  if (__syncthreads_count(total[threadIdx.x] != 0u) <= SEL_FEW_DIGITS)
+    sel_scatter_body<false>(key_in, val_in, n64, shift, counts, ntiles64, total, key_out, val_out,
+                            sh);
+  else
+    sel_scatter_body<true>(key_in, val_in, n64, shift, counts, ntiles64, total, key_out, val_out,
+                           sh);
 }
 
 // per tile: inclusive prefix of the labels inside the tile (first n_f items)
