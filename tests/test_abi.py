@@ -40,6 +40,21 @@ def test_binding_covers_the_header(lib):
     assert sorted(binding.EXPORTS) == declared_functions()
 
 
+def test_header_is_plain_c(tmp_path):
+    """The boundary is a C ABI: the header compiles as strict C99 with no
+    CUDA or C++ header behind it."""
+    import shutil
+    import subprocess
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    src = tmp_path / "use.c"
+    src.write_text('#include "pro_router.h"\nint main(void) { return pr_launch_count() > 0; }\n')
+    subprocess.run([cc, "-std=c99", "-Wall", "-Wextra", "-pedantic", "-Werror", "-I",
+                    os.path.dirname(HEADER), "-c", str(src), "-o", str(tmp_path / "use.o")],
+                   check=True)
+
+
 def test_library_targets_sm_103a_only():
     assert prbuild.ARCH == ["-gencode", "arch=compute_103a,code=sm_103a"]
 
