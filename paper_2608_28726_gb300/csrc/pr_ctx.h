@@ -49,6 +49,8 @@ struct pr_ctx {
   // pr_selective_metrics: sort workspace for up to sel_cap scores, grown on demand
   void* sel_ws = nullptr;
   int64_t sel_cap = 0;
+  // its persistent radix scatter: resident CTAs per SM; 0 = not set up yet
+  int sel_scatter_bps = 0;
   // pr_lmhead_features: per-(row, split) states, grown on demand
   void* lm_parts = nullptr;
   size_t lm_parts_bytes = 0;

@@ -97,15 +97,14 @@ pr_status pr_selective_metrics(pr_ctx* c, const float* scores, const uint8_t* la
   const int64_t ntiles = (n + prk::SEL_TILE - 1) / prk::SEL_TILE;
   const unsigned g_tiles = (unsigned)ntiles;
   // the scatter is persistent: one wave of resident CTAs
-  static int scatter_bps = 0;
-  if (scatter_bps == 0) {
+  if (c->sel_scatter_bps == 0) {
     int b = 0;
     PR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, prk::sel_scatter, prk::SEL_NT, 0));
-    scatter_bps = b > 0 ? b : 1;
+    c->sel_scatter_bps = b > 0 ? b : 1;
   }
   const int64_t rtiles = (n + prk::SR_TILE - 1) / prk::SR_TILE;  // tiles of the radix passes
   const unsigned g_scatter =
-      (unsigned)std::min<int64_t>(rtiles, (int64_t)c->num_sms * scatter_bps);
+      (unsigned)std::min<int64_t>(rtiles, (int64_t)c->num_sms * c->sel_scatter_bps);
   int launches = 0;
   // after each launch: count it, check it, and (PR_OPT_TIMING) record an event
   auto launched = [&]() -> pr_status {
