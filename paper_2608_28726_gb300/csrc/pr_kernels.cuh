@@ -631,7 +631,7 @@ __global__ void __launch_bounds__(NT, rows_min_blocks<T>()) verify_rows(const Ar
       const int32_t gi = t * TILE + (j % UNR) * NT + (int32_t)(id & 255u);
       if (t >= ntiles || gi >= ng) continue;
       const int32_t g = g0 + gi;
-      const uint4 wv = ALIGNED ? ld_stream(vp + g) : Tr::load_elems(rowp, (int64_t)g);
+      const uint4 wv = ALIGNED ? ld_reread(vp + g) : Tr::load_elems(rowp, (int64_t)g);
 #pragma unroll
       for (int e2 = 0; e2 < VEC; ++e2) {
         const float x = Tr::at(wv, e2);
@@ -784,9 +784,14 @@ struct SmemWS {
   uint32_t wl[2][NWARP][32];    // per-warp sorted per-thread maxima, ord() encoded
   float pm[2][NWARP], pS[2][NWARP], pU[2][NWARP];
   float cand_v[CCAP];           // finaliser: candidate tiles (value,
-  uint32_t cand_id[CCAP];       //   tile << 8 | thread)
+  uint32_t cand_id[CCAP];       //   tile << 8 | thread, | BEST_BIT for a thread's best tile)
   uint64_t ebuf[ECAP];          // finaliser: candidate element keys
+  uint4 best[2][UNR][NT];       // per thread: the groups of its best tile, as streamed
 };
+
+// A candidate that is its thread's best tile: the finaliser reads its groups
+// from SmemWS::best instead of re-reading the row (tile indices stay below 2^16).
+constexpr uint32_t BEST_BIT = 0x80000000u;
 
 // Row geometry shared by the streaming warps and the finaliser (C = 1).
 struct RowGeom {
@@ -886,7 +891,7 @@ __device__ __noinline__ void finalize_ws(const Args& a, SmemWS& sm, int b, int64
       const int p2 = n + __popc(b1) + __popc(b2 & lt);
       if (c1 && p1 < CCAP) {
         sm.cand_v[p1] = inf.x;
-        sm.cand_id[p1] = ((ids & 0xffffu) << 8) | t;
+        sm.cand_id[p1] = BEST_BIT | ((ids & 0xffffu) << 8) | t;
       }
       if (c2 && !c3 && p2 < CCAP) {
         sm.cand_v[p2] = inf.y;
@@ -927,22 +932,32 @@ __device__ __noinline__ void finalize_ws(const Args& a, SmemWS& sm, int b, int64
   }
   __syncwarp();
 
-  // ---- re-read the candidate tiles (issued first, so that sorting the
-  // candidates for theta overlaps the loads), then keep elements >= theta
+  // ---- the candidate tiles' groups: a thread's best tile from shared
+  // memory, the others re-read from the row (issued first, so that sorting
+  // the candidates for theta overlaps the loads); then keep elements >= theta
   const int total = fb ? 0 : n * UNR;
+  // group `it` of the candidates (UNR per candidate tile): its index in the
+  // row (or -1: none, or the partial last group) and its 16 bytes
+  auto cand_group = [&](int it, int32_t& gsel_q, uint4& w) {
+    gsel_q = -1;
+    w = NEG;
+    const uint32_t id = sm.cand_id[it >> 2];
+    if (id == TAIL_ID) return;
+    const int k = it & (UNR - 1), t = (int)(id & 255u);
+    const int32_t gi = (int32_t)((id & ~BEST_BIT) >> 8) * TILE + k * NT + t;
+    if (gi >= geo.gfull) return;
+    gsel_q = gi;
+    if (id & BEST_BIT) w = sm.best[b][k][t];
+    else w = ALIGNED ? ld_reread(vp + gi) : Tr::load_elems(rowp, gi);
+  };
   uint4 wv[4];
   int32_t gsel[4];
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
     const int it = q * 32 + lane;
     gsel[q] = -1;
-    if (it < total) {
-      const uint32_t id = sm.cand_id[it >> 2];
-      const int32_t gi = (int32_t)(id >> 8) * TILE + (it & (UNR - 1)) * NT + (int32_t)(id & 255u);
-      if (id != TAIL_ID && gi < geo.gfull) gsel[q] = gi;
-    }
     wv[q] = NEG;
-    if (gsel[q] >= 0) wv[q] = ALIGNED ? ld_stream(vp + gsel[q]) : Tr::load_elems(rowp, gsel[q]);
+    if (it < total) cand_group(it, gsel[q], wv[q]);
   }
 
   // ---- theta: the exact kc-th largest candidate value (theta1 if a thread
@@ -969,13 +984,8 @@ __device__ __noinline__ void finalize_ws(const Args& a, SmemWS& sm, int b, int64
         for (int q = 0; q < 4; ++q) {
           const int it = i0 + q * 32 + lane;
           gsel[q] = -1;
-          if (it < total && sm.cand_v[it >> 2] >= th) {
-            const uint32_t id = sm.cand_id[it >> 2];
-            const int32_t gi = (int32_t)(id >> 8) * TILE + (it & (UNR - 1)) * NT + (int32_t)(id & 255u);
-            if (id != TAIL_ID && gi < geo.gfull) gsel[q] = gi;
-          }
           wv[q] = NEG;
-          if (gsel[q] >= 0) wv[q] = ALIGNED ? ld_stream(vp + gsel[q]) : Tr::load_elems(rowp, gsel[q]);
+          if (it < total && sm.cand_v[it >> 2] >= th) cand_group(it, gsel[q], wv[q]);
         }
       }
 #pragma unroll
@@ -1142,6 +1152,10 @@ __global__ void __launch_bounds__(NT_WS, 3) verify_rows_ws(const Args a) {
       const float tmax = Tr::tile_max(cur);
       {
         const bool c1 = tmax > v1, c2 = tmax > v2;
+        if (c1) {  // a new best tile: keep its groups for the finaliser
+#pragma unroll
+          for (int k = 0; k < UNR; ++k) sm.best[b][k][tid] = cur[k];
+        }
         v3 = fmaxf(v3, fminf(tmax, v2));
         const float nv2 = c1 ? v1 : (c2 ? tmax : v2);
         const uint32_t ni2 = c1 ? i1 : (c2 ? (uint32_t)t : i2);
