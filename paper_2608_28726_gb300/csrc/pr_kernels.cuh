@@ -11,6 +11,17 @@
 
 namespace prk {
 
+// A scattered 16-byte re-read of a row already streamed: without the 256-byte
+// L2 prefetch of ld_stream, a load that misses L2 fetches one 32-byte sector
+// from DRAM instead of a 256-byte block.
+__device__ __forceinline__ uint4 ld_reread(const void* p) {
+  uint4 r;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+               : "l"(p));
+  return r;
+}
+
 // ---- pooling, scoring, ship rule (Section 3.1) -------------------------------------
 
 struct Pooled {
