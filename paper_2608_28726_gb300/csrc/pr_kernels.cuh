@@ -770,8 +770,9 @@ __global__ void __launch_bounds__(NT, rows_min_blocks<T>()) verify_rows(const Ar
 //
 // NWARP streaming warps read rows blockIdx.x, blockIdx.x + gridDim.x, ...; they
 // never wait on the per-row selection: at the end of a row they leave its tile
-// maxima, per-warp (m, S, U) and sorted per-thread maxima in one of two shared
-// buffers, signal the finaliser warp with a named barrier and go on (the next
+// maxima, per-warp (m, S, U), sorted per-thread maxima and each thread's best
+// tile in one of two shared buffers, signal the finaliser warp with a named
+// barrier and go on (the next
 // row's first tile is already in flight).  The finaliser warp turns a buffer
 // into the row's exact top-K, features and epilogue, then hands the buffer
 // back.  Named barriers (bar.arrive / bar.sync with NT + 32 threads) are the
@@ -825,7 +826,9 @@ struct RowGeom {
 // thread whose third-best value also reaches theta1 contributes all its
 // tiles, and then theta stays theta1 (exact, if slower).  Otherwise theta =
 // the kc-th largest candidate value.  Elements >= theta of the candidate
-// tiles are the only ones that can be among the top kc.
+// tiles are the only ones that can be among the top kc.  A best tile is read
+// from the copy the streaming thread left in shared memory; the other
+// candidate tiles are re-read from the row, which may have left L2 by then.
 template <typename T, int MODE, bool ALIGNED>
 __device__ __noinline__ void finalize_ws(const Args& a, SmemWS& sm, int b, int64_t row,
                                          const RowGeom& geo, const RowPre& pre, int lane) {

@@ -180,6 +180,70 @@ def test_persistent_many_rows_per_cta(ctx, dtype):
     _set(ctx)
 
 
+def _tile_pattern_rows(V, dtype, seed):
+    """Rows whose largest values sit where the persistent kernel's candidate
+    tiles come from different places.  Group g of a row belongs to tile
+    g // 1024 and thread g % 256 (four groups of 16 bytes per thread per
+    tile); a thread's best tile is read back from shared memory, its other
+    candidate tiles from the row."""
+    vec = 8 if dtype == torch.bfloat16 else 4
+    nt, unr = 256, 4
+    tile = nt * unr
+    ntiles = -(-(V // vec) // tile)
+    g = torch.Generator().manual_seed(seed)
+
+    def at(t, tid, k, e):
+        return ((t * tile + k * nt + tid) * vec + e)
+
+    rows = []
+    # one thread holds the top values in five tiles: a third tile >= theta1,
+    # so every tile of that thread is a candidate
+    r = torch.randn(V, generator=g)
+    for j, t in enumerate(range(0, ntiles, max(1, ntiles // 5))):
+        for k in range(unr):
+            v = at(t, 7, k, (j + k) % vec)
+            if v < V:
+                r[v] = 10.0 + j + 0.125 * k
+    rows.append(r)
+    # 24 threads with two strong tiles each: second-best tiles as candidates
+    r = torch.randn(V, generator=g)
+    for i in range(24):
+        for j, t in enumerate((1 + i % 3, ntiles - 2 - i % 4)):
+            v = at(t, 9 * i + 3, i % unr, i % vec)
+            if v < V:
+                r[v] = 8.0 + 0.0625 * i + 0.5 * j
+    rows.append(r)
+    # rising along the row: every tile beats its thread's best so far
+    rows.append(torch.linspace(-3.0, 3.0, V) + 0.01 * torch.randn(V, generator=g))
+    # falling: each thread's best tile is its first and must outlast the row
+    rows.append(torch.linspace(3.0, -3.0, V) + 0.01 * torch.randn(V, generator=g))
+    # the two largest values, tied, at the end of the last full tile and in
+    # the row's last element
+    r = torch.randn(V, generator=g)
+    r[V - 1] = 6.0
+    r[min(V // vec // tile * tile * vec, V) - 1] = 6.0
+    rows.append(r)
+    return torch.stack(rows).to(dtype)
+
+
+@pytest.mark.parametrize("dtype,V", [(torch.bfloat16, 151936), (torch.float32, 65549)])
+def test_persistent_candidate_paths(ctx, dtype, V):
+    """The persistent kernel's candidate tiles: a thread's best tile from shared
+    memory, its second-best and (for a thread with three tiles above theta1)
+    all its other tiles from the row, on both shared buffers (600 rows, more
+    than one per CTA)."""
+    _set(ctx, split=1)
+    x, ch = random_rows(600, V, dtype, seed=4242)
+    pat = _tile_pattern_rows(V, dtype, seed=4243)
+    for j in range(pat.size(0)):
+        for base in (0, 470):
+            x[base + 3 * j] = pat[j].cuda()
+    feat, top2, rf = B.pr_token_features(ctx, x, ch, topk=20)
+    of, oi, ofl = _oracle_rows(x, ch)
+    _check_features(feat, top2, rf, of, oi, ofl, "candidate paths V=%d" % V)
+    _set(ctx)
+
+
 def test_features_rho(ctx):
     lengths = [5, 1, 0, 9, 3]
     off = torch.tensor(np.concatenate([[0], np.cumsum(lengths)]), dtype=torch.int64).cuda()
