@@ -165,8 +165,8 @@ __global__ void __launch_bounds__(NT) head_embed(const HeadArgs a) {
 
 // ---- head_attn: softmax(Q K^T / 4) V on the tensor cores ----------------------------
 //
-// CTA (request, head, z) takes the 128-query blocks z, z + HA_QZ, ... of its
-// request; thread i owns query i of the block and TMEM lane i.  The keys pass
+// CTA (request, head, z) takes the 128-query blocks z, z + gridDim.z, ... of
+// its request; thread i owns query i of the block and TMEM lane i.  The keys pass
 // in chunks of 64.  Per chunk two tcgen05.mma kind::tf32 contractions run with
 // fp32 accumulators in TMEM: S = Q K^T (M = 128 queries, N = the chunk's keys
 // rounded up to 16, K = 16) and O_c = P V (M = 128, K = the chunk's keys
@@ -197,7 +197,8 @@ __global__ void __launch_bounds__(NT) head_embed(const HeadArgs a) {
 // writing one dimension of 32 consecutive keys hit 32 different banks.
 constexpr int HA_M = 128;                       // queries per block = TMEM lanes = threads
 constexpr int HA_NC = 64;                       // keys per chunk
-constexpr int HA_QZ = 8;                        // CTAs per (request, head)
+constexpr int HA_QZ_MIN = 4;                    // CTAs per (request, head): at least,
+constexpr int HA_QZ_MAX = 16;                   //   and at most
 constexpr uint32_t HA_TMEM_COLS = 128;
 constexpr uint32_t HA_O_COL = HA_NC;            // O_c: [V_hi | V_lo] products, 32 columns
 constexpr uint32_t HA_QH_COL = HA_O_COL + 2 * HDH;
@@ -485,7 +486,7 @@ __global__ void __launch_bounds__(HA_M, HA_CTAS_PER_SM) head_attn(const HeadArgs
     }
   };
 
-  for (int qb = blockIdx.z; qb < nqb && ok; qb += HA_QZ) {
+  for (int qb = blockIdx.z; qb < nqb && ok; qb += (int)gridDim.z) {
     const int q = qb * HA_M + tid;
     if (qb != (int)blockIdx.z) {
       load_q(qb);

@@ -115,10 +115,20 @@ pr_status pr_head_score(pr_ctx* c, const float* feat, const uint32_t* row_flags,
     st = launch_head(c, reinterpret_cast<const void*>(&prk::head_rows<prk::HR_QKV>), dim3(ntiles),
                      rblk, prk::HT_SMEM, s, true, a);
     if (st != PR_OK) return st;
+    // CTAs per (request, head): one per query block of a request of the mean
+    // length, at least HA_QZ_MIN.  A CTA whose request has no block z exits at
+    // once, but empty CTAs still slow the launch chain, and too few leave long
+    // requests' blocks in sequence (two layers, back-to-back calls: 64 requests
+    // of U{32..256} rows 72.3 us with 8 CTAs, 71.0 with 4; 1,024 lognormal
+    // requests 1.12 ms with 8, 1.07 with 4; four requests of 2,100 and 1,300
+    // rows 484 us with 8, 359 with 14).
+    const int64_t mean_t = n_rows / n_req;
+    const unsigned gz = (unsigned)std::min<int64_t>(
+        prk::HA_QZ_MAX, std::max<int64_t>(prk::HA_QZ_MIN, (mean_t + prk::HA_M - 1) / prk::HA_M));
     for (int l = 0; l < n_layers; ++l) {
       st = launch_head(c, reinterpret_cast<const void*>(&prk::head_attn),
-                       dim3((unsigned)n_req, prk::HHEADS, prk::HA_QZ), dim3(prk::HA_M),
-                       prk::HA_SMEM, s, true, a);
+                       dim3((unsigned)n_req, prk::HHEADS, gz), dim3(prk::HA_M), prk::HA_SMEM, s,
+                       true, a);
       if (st != PR_OK) return st;
       a.lcur = layer(l);
       const bool last = l + 1 == n_layers;

@@ -226,21 +226,26 @@ def _tile_pattern_rows(V, dtype, seed):
     return torch.stack(rows).to(dtype)
 
 
+@pytest.mark.parametrize("shift", [0, 1])
 @pytest.mark.parametrize("dtype,V", [(torch.bfloat16, 151936), (torch.float32, 65549)])
-def test_persistent_candidate_paths(ctx, dtype, V):
+def test_persistent_candidate_paths(ctx, dtype, V, shift):
     """The persistent kernel's candidate tiles: a thread's best tile from shared
     memory, its second-best and (for a thread with three tiles above theta1)
     all its other tiles from the row, on both shared buffers (600 rows, more
-    than one per CTA)."""
+    than one per CTA); with shift 1 the rows start off the 16-byte grid and
+    take the element-load path."""
     _set(ctx, split=1)
-    x, ch = random_rows(600, V, dtype, seed=4242)
+    pad = (-V) % 8 + 8  # a row stride of a multiple of 16 bytes
+    base, ch = random_rows(600, V + pad, dtype, seed=4242)
+    x = base[:, shift:shift + V]
+    ch = ch % V
     pat = _tile_pattern_rows(V, dtype, seed=4243)
     for j in range(pat.size(0)):
-        for base in (0, 470):
-            x[base + 3 * j] = pat[j].cuda()
+        for r0 in (0, 470):
+            x[r0 + 3 * j] = pat[j].cuda()
     feat, top2, rf = B.pr_token_features(ctx, x, ch, topk=20)
-    of, oi, ofl = _oracle_rows(x, ch)
-    _check_features(feat, top2, rf, of, oi, ofl, "candidate paths V=%d" % V)
+    of, oi, ofl = _oracle_rows(x.contiguous(), ch)
+    _check_features(feat, top2, rf, of, oi, ofl, "candidate paths V=%d shift=%d" % (V, shift))
     _set(ctx)
 
 
