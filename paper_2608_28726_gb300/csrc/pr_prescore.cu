@@ -16,6 +16,11 @@
 //   * length = the prompt's token count; w = V TF-IDF weights, then the
 //     image-count weight, then the length weight.
 // Sums run in double precision in ascending column order.
+//
+// Scoring a prompt hashes each token while it is read (64-bit FNV-1a over the
+// lowercased bytes), finds its column in an open-addressing table of the
+// vocabulary, and counts it in a per-thread dense array, so that no token is
+// copied into a string or a node-based map.
 #include <algorithm>
 #include <cmath>
 #include <cstring>
@@ -30,10 +35,13 @@
 #include "pro_router.h"
 
 struct pr_prescorer {
-  std::vector<std::string> terms;                   // column -> term, byte order
-  std::unordered_map<std::string, int32_t> column;  // term -> column
+  std::vector<std::string> terms;  // column -> term, byte order
   std::vector<double> idf;
   int64_t n_docs = 0;
+  // term -> column: open addressing, linear probing, at most half full
+  std::vector<uint64_t> slot_hash;
+  std::vector<int32_t> slot_col;  // -1: empty
+  uint64_t slot_mask = 0;
 };
 
 namespace {
@@ -43,6 +51,27 @@ inline bool word_byte(unsigned char c) {
          c >= 0x80;
 }
 
+constexpr uint64_t FNV_OFFSET = 1469598103934665603ull, FNV_PRIME = 1099511628211ull;
+
+inline uint64_t fnv1a(const char* p, size_t n) {
+  uint64_t h = FNV_OFFSET;
+  for (size_t i = 0; i < n; ++i) h = (h ^ (unsigned char)p[i]) * FNV_PRIME;
+  return h;
+}
+
+inline unsigned char lower(unsigned char c) {
+  return (c >= 'A' && c <= 'Z') ? (unsigned char)(c + ('a' - 'A')) : c;
+}
+
+// per byte: 0 outside a token (the NUL included), else the byte lowercased
+struct ByteClass {
+  unsigned char v[256];
+  ByteClass() {
+    for (int c = 0; c < 256; ++c) v[c] = (c != 0 && word_byte((unsigned char)c)) ? lower((unsigned char)c) : 0;
+  }
+};
+const ByteClass kByte;
+
 // calls f(token) for every token of the NUL-terminated text
 template <class F>
 void for_each_token(const char* text, F&& f) {
@@ -50,7 +79,7 @@ void for_each_token(const char* text, F&& f) {
   for (const unsigned char* p = reinterpret_cast<const unsigned char*>(text);; ++p) {
     const unsigned char c = *p;
     if (c != 0 && word_byte(c)) {
-      tok.push_back((c >= 'A' && c <= 'Z') ? char(c + ('a' - 'A')) : char(c));
+      tok.push_back((char)lower(c));
       continue;
     }
     if (tok.size() >= 2) f(tok);
@@ -59,23 +88,74 @@ void for_each_token(const char* text, F&& f) {
   }
 }
 
+// the column of the lowercased token tok[0, n) with hash h, or -1
+inline int32_t find_column(const pr_prescorer& ps, const unsigned char* tok, size_t n, uint64_t h) {
+  if (ps.slot_col.empty()) return -1;
+  for (uint64_t i = h & ps.slot_mask;; i = (i + 1) & ps.slot_mask) {
+    const int32_t c = ps.slot_col[i];
+    if (c < 0) return -1;
+    if (ps.slot_hash[i] == h) {
+      const std::string& t = ps.terms[(size_t)c];
+      if (t.size() == n && std::memcmp(t.data(), tok, n) == 0) return c;
+    }
+  }
+}
+
+void build_table(pr_prescorer& ps) {
+  size_t cap = 16;
+  while (cap < 2 * ps.terms.size()) cap <<= 1;
+  ps.slot_hash.assign(cap, 0ull);
+  ps.slot_col.assign(cap, -1);
+  ps.slot_mask = cap - 1;
+  for (size_t j = 0; j < ps.terms.size(); ++j) {
+    const uint64_t h = fnv1a(ps.terms[j].data(), ps.terms[j].size());
+    uint64_t i = h & ps.slot_mask;
+    while (ps.slot_col[i] >= 0) i = (i + 1) & ps.slot_mask;
+    ps.slot_hash[i] = h;
+    ps.slot_col[i] = (int32_t)j;
+  }
+}
+
 struct Row {
   std::vector<std::pair<int32_t, double>> v;  // (column, value), ascending column
   int64_t length = 0;
+  std::vector<int32_t> count;    // per column (all zero between prompts)
+  std::vector<int32_t> touched;  // columns counted in this prompt
+  std::vector<unsigned char> tok;
 };
 
 void tfidf_row(const pr_prescorer& ps, const char* prompt, Row& row) {
-  std::unordered_map<int32_t, int64_t> counts;
+  if (row.count.size() != ps.terms.size()) row.count.assign(ps.terms.size(), 0);
+  row.touched.clear();
   row.length = 0;
-  for_each_token(prompt, [&](const std::string& t) {
-    ++row.length;
-    const auto it = ps.column.find(t);
-    if (it != ps.column.end()) ++counts[it->second];
-  });
+  // maximal runs of word bytes, lowercased and hashed as they are read
+  size_t n = 0;
+  uint64_t h = FNV_OFFSET;
+  for (const unsigned char* p = reinterpret_cast<const unsigned char*>(prompt);; ++p) {
+    const unsigned char c = *p;
+    const unsigned char lc = kByte.v[c];
+    if (lc != 0) {
+      if (n == row.tok.size()) row.tok.resize(row.tok.empty() ? 64 : 2 * row.tok.size());
+      row.tok[n++] = lc;
+      h = (h ^ lc) * FNV_PRIME;
+      continue;
+    }
+    if (n >= 2) {
+      ++row.length;
+      const int32_t col = find_column(ps, row.tok.data(), n, h);
+      if (col >= 0 && row.count[(size_t)col]++ == 0) row.touched.push_back(col);
+    }
+    n = 0;
+    h = FNV_OFFSET;
+    if (c == 0) break;
+  }
+  std::sort(row.touched.begin(), row.touched.end());
   row.v.clear();
-  row.v.reserve(counts.size());
-  for (const auto& kc : counts) row.v.emplace_back(kc.first, (double)kc.second * ps.idf[kc.first]);
-  std::sort(row.v.begin(), row.v.end());
+  row.v.reserve(row.touched.size());
+  for (const int32_t col : row.touched) {
+    row.v.emplace_back(col, (double)row.count[(size_t)col] * ps.idf[(size_t)col]);
+    row.count[(size_t)col] = 0;
+  }
   double ss = 0.0;
   for (const auto& e : row.v) ss += e.second * e.second;
   if (ss > 0.0) {
@@ -124,12 +204,10 @@ pr_status pr_prescorer_fit(const char* const* docs, int32_t n_docs, int32_t min_
       if (tc.second >= min_df) ps->terms.push_back(tc.first);
     std::sort(ps->terms.begin(), ps->terms.end());  // byte order (std::string compares as unsigned char)
     ps->idf.resize(ps->terms.size());
-    ps->column.reserve(ps->terms.size());
-    for (size_t j = 0; j < ps->terms.size(); ++j) {
-      ps->column.emplace(ps->terms[j], (int32_t)j);
+    for (size_t j = 0; j < ps->terms.size(); ++j)
       ps->idf[j] = std::log((1.0 + (double)n_docs) / (1.0 + (double)df[ps->terms[j]])) + 1.0;
-    }
     ps->n_docs = n_docs;
+    build_table(*ps);
     *out = ps;
     return PR_OK;
   } catch (const std::bad_alloc&) {
