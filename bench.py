@@ -1690,12 +1690,12 @@ def run_prescore_workload(args):
     w, b = W.prescore_weights(V)
     cores = os.cpu_count() or 1
     import ctypes
-    _bs, arr = B._texts(prompts)  # the host arrays the C call reads, built once
+    _buf, ptrs, _ = B._texts(prompts)  # the host arrays the C call reads, built once
     n = len(prompts)
     p_lib, z_lib = np.empty(n, np.float32), np.empty(n, np.float32)
 
     def call(n_threads=0, count=n):
-        st = B._lib.pr_prescorer_score(ps, ctypes.cast(arr, ctypes.c_void_p), images.ctypes.data,
+        st = B._lib.pr_prescorer_score(ps, ptrs.ctypes.data, images.ctypes.data,
                                        count, w.ctypes.data, float(b), n_threads,
                                        p_lib.ctypes.data, z_lib.ctypes.data)
         assert st == 0, st

@@ -578,19 +578,33 @@ def pr_selftest_wait(ctx, limit_ns: int) -> bool:
 # ---- the prompt pre-scorer (host CPU; Section 3.1, Eq. 2) ---------------------------------
 
 def _texts(texts):
-    """Host array of NUL-terminated byte strings (kept alive by the caller)."""
-    bs = [t.encode() if isinstance(t, str) else bytes(t) for t in texts]
-    if any(b"\0" in b for b in bs):
+    """(buffer, pointers, n): the n texts as NUL-terminated byte strings side
+    by side in one host buffer, and a uint64 array of their addresses (the C
+    call's `const char* const*`).  The caller keeps both alive for the call."""
+    texts = list(texts)
+    n = len(texts)
+    if n == 0:
+        return b"", np.zeros(1, np.uint64), 0
+    if all(isinstance(t, str) for t in texts):
+        buf = ("\0".join(texts) + "\0").encode()
+    else:
+        buf = b"\0".join(t.encode() if isinstance(t, str) else bytes(t) for t in texts) + b"\0"
+    a = np.frombuffer(buf, np.uint8)
+    ends = np.flatnonzero(a == 0)
+    if ends.size != n:
         raise PRError(PR_ERR_INVALID_ARG, "prescorer", "a text holds a NUL byte")
-    arr = (ctypes.c_char_p * max(1, len(bs)))(*bs)
-    return bs, arr
+    ptrs = np.empty(n, np.uint64)
+    ptrs[0] = 0
+    ptrs[1:] = ends[:-1] + 1
+    ptrs += np.uint64(a.ctypes.data)
+    return buf, ptrs, n
 
 
 def pr_prescorer_fit(docs, min_df: int = 1):
     """Vocabulary and smoothed idf of a corpus (str or bytes texts)."""
-    bs, arr = _texts(docs)
+    buf, ptrs, n = _texts(docs)
     out = _P()
-    _check(_lib.pr_prescorer_fit(ctypes.cast(arr, _P), len(bs), int(min_df), ctypes.byref(out)),
+    _check(_lib.pr_prescorer_fit(ptrs.ctypes.data, n, int(min_df), ctypes.byref(out)),
            "pr_prescorer_fit")
     return out.value
 
@@ -621,15 +635,14 @@ def pr_prescorer_features(ps, prompt, cap: int = 4096):
 
 def pr_prescorer_score(ps, prompts, n_images, w, b: float, n_threads: int = 0):
     """(p_pre float32 [n], logit float32 [n]) on the host; w: float32 [V + 2]."""
-    bs, arr = _texts(prompts)
-    n = len(bs)
+    buf, ptrs, n = _texts(prompts)
     img = np.ascontiguousarray(n_images, np.int32)
     wv = np.ascontiguousarray(w, np.float32)
     if img.shape != (n,) or wv.shape != (pr_prescorer_vocab_size(ps) + 2,):
         raise PRError(PR_ERR_INVALID_ARG, "pr_prescorer_score", "n_images or w has the wrong size")
     score = np.empty(max(1, n), np.float32)
     logit = np.empty(max(1, n), np.float32)
-    _check(_lib.pr_prescorer_score(ps, ctypes.cast(arr, _P), img.ctypes.data, n, wv.ctypes.data,
+    _check(_lib.pr_prescorer_score(ps, ptrs.ctypes.data, img.ctypes.data, n, wv.ctypes.data,
                                    float(b), int(n_threads), score.ctypes.data, logit.ctypes.data),
            "pr_prescorer_score")
     return score[:n], logit[:n]
