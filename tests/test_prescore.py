@@ -118,3 +118,23 @@ def test_bad_arguments(B):
             B.pr_prescorer_features(ps, b"alpha beta", cap=1)
     finally:
         B.pr_prescorer_destroy(ps)
+
+
+def test_text_marshalling(B):
+    """The prompts reach the C call as NUL-terminated strings in one buffer,
+    addressed by a pointer array: str, bytes and non-ASCII text read back as
+    given; a NUL inside a text is refused."""
+    import ctypes
+    texts = ["plain text", b"raw bytes \xff\xfe", "naïve café", "", b"", "x" * 5000]
+    buf, ptrs, n = B._texts(texts)
+    assert n == len(texts) and ptrs.dtype == np.uint64
+    for t, p in zip(texts, ptrs):
+        want = t.encode() if isinstance(t, str) else t
+        assert ctypes.string_at(int(p)) == want
+    buf, ptrs, n = B._texts(["only", "strings"])
+    assert [ctypes.string_at(int(p)) for p in ptrs] == [b"only", b"strings"]
+    buf, ptrs, n = B._texts([])
+    assert n == 0
+    for bad in (["a\0b"], [b"a", b"\0"], ["ok", "no\0"]):
+        with pytest.raises(B.PRError):
+            B._texts(bad)
