@@ -102,7 +102,9 @@ typedef enum { PR_DTYPE_F32 = 0, PR_DTYPE_BF16 = 1 } pr_dtype;
 /* options (pr_ctx_set_option) */
 #define PR_OPT_TOPK 0        /* K of the top-K entropy for pr_route / pr_decode_step; default 20 */
 #define PR_OPT_TOPK_RENORM 1 /* 0 (default): raw p over the top K; 1: renormalised over the top K */
-#define PR_OPT_SPLIT 2       /* CTAs per row (thread-block cluster): 0 = automatic, or 1, 2, 4, 8 */
+#define PR_OPT_SPLIT 2       /* CTAs per row (thread-block cluster): 0 = automatic, or 1, 2, 4, 8;
+                                1 runs the persistent kernel (rows of more than 2^16 tiles of
+                                1,024 x 16 bytes take one CTA per row instead) */
 #define PR_OPT_OVERLAP 3     /* 1: a call may start while the previous kernel on its stream is
                                 still running (programmatic dependent launch): it reads its
                                 inputs at once and waits for that kernel before writing

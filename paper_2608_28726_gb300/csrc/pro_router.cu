@@ -92,24 +92,29 @@ pr_status ws_setup(pr_ctx* c, pr_dtype dt, int mode, bool aligned, int* bps) {
 //    against 13.9 us with the persistent kernel);
 //  * fewer rows: the largest split (<= 8) whose CTAs still fit in one wave;
 //  * more rows: the persistent kernel.
+// The persistent kernel keeps a thread's best tile indices in 16 bits, so rows
+// of more than 2^16 tiles (over 536 M bf16 or 268 M fp32 values) take one CTA
+// per row instead, the forced split 1 included.
 struct LaunchShape {
   int C;
   bool persistent;
 };
 
-LaunchShape choose_launch(pr_ctx* c, pr_dtype dt, int mode, int64_t n_rows) {
-  if (c->split == 1) return {1, true};
+LaunchShape choose_launch(pr_ctx* c, pr_dtype dt, int mode, int64_t n_rows, int64_t vocab) {
+  const int64_t groups = vocab / (dt == PR_DTYPE_BF16 ? 8 : 4);
+  const bool ws_fits = (groups + prk::TILE - 1) / prk::TILE <= 65536;
+  if (c->split == 1) return {1, ws_fits};
   if (c->split == 2 || c->split == 4 || c->split == 8) return {c->split, false};
   const int64_t slots = (int64_t)c->num_sms * blocks_per_sm(c, dt, mode);
   if (n_rows >= c->num_sms && n_rows <= slots) return {1, false};
   int s = 1;
   while (s < prk::MAXC && n_rows * (s * 2) <= slots) s <<= 1;
-  return {s, s == 1};
+  return {s, s == 1 && ws_fits};
 }
 
 pr_status launch_rows(pr_ctx* c, pr_dtype dt, int mode, const prk::Args& a, cudaStream_t st) {
   if (a.n_rows == 0) return PR_OK;
-  const LaunchShape shape = choose_launch(c, dt, mode, a.n_rows);
+  const LaunchShape shape = choose_launch(c, dt, mode, a.n_rows, a.vocab);
   const int C = shape.C;
   if (shape.persistent) {
     // persistent warp-specialised kernel: every SM gets its resident CTAs

@@ -249,6 +249,30 @@ def test_persistent_candidate_paths(ctx, dtype, V, shift):
     _set(ctx)
 
 
+def test_rows_past_the_persistent_kernels_tile_limit(ctx):
+    """Rows of more than 2^16 tiles (268,443,648 fp32 values, 1.07 GB a row)
+    leave the persistent kernel, whose tile indices are 16-bit, even with
+    split 1 forced; the largest values sit in the rows' last tiles."""
+    _set(ctx, split=1)
+    V = (1 << 28) + 2 * 4096
+    free, _ = torch.cuda.mem_get_info()
+    if free < 8 * V * 4:
+        pytest.skip("needs about 9 GB of free device memory")
+    g = torch.Generator(device="cuda")
+    g.manual_seed(5)
+    x = torch.randn(2, V, device="cuda", generator=g)
+    x[0, V - 1] = 40.0
+    x[0, V - 5000] = 39.0
+    x[1, 3] = 41.0
+    x[1, V - 2] = 42.0
+    ch = torch.tensor([V - 1, 7], dtype=torch.int32, device="cuda")
+    feat, top2, rf = B.pr_token_features(ctx, x, ch, topk=20)
+    of, oi, ofl = _oracle_rows(x, ch)
+    assert oi[0].tolist() == [V - 1, V - 5000] and oi[1].tolist() == [V - 2, 3]
+    _check_features(feat, top2, rf, of, oi, ofl, "rows of 65,538 tiles")
+    _set(ctx)
+
+
 def test_features_rho(ctx):
     lengths = [5, 1, 0, 9, 3]
     off = torch.tensor(np.concatenate([[0], np.cumsum(lengths)]), dtype=torch.int64).cuda()
