@@ -17,18 +17,18 @@
 //     image-count weight, then the length weight.
 // Sums run in double precision in ascending column order.
 //
-// Scoring a prompt hashes each token while it is read (64-bit FNV-1a over the
-// lowercased bytes), finds its column in an open-addressing table of the
-// vocabulary, and counts it in a per-thread dense array, so that no token is
-// copied into a string or a node-based map.
+// Both fitting and scoring hash each token while it is read (64-bit FNV-1a
+// over the lowercased bytes).  Fitting counts document frequencies in an
+// open-addressing table of the corpus's terms; scoring finds a token's column
+// in an open-addressing table of the vocabulary and counts it in a per-thread
+// dense array, so that no token is copied into a string or a node-based map.
 #include <algorithm>
 #include <cmath>
 #include <cstring>
+#include <memory>
 #include <new>
 #include <string>
 #include <thread>
-#include <unordered_map>
-#include <unordered_set>
 #include <utility>
 #include <vector>
 
@@ -72,21 +72,75 @@ struct ByteClass {
 };
 const ByteClass kByte;
 
-// calls f(token) for every token of the NUL-terminated text
+// calls f(tok, n, h) for every token of the NUL-terminated text: tok[0, n)
+// its lowercased bytes (in buf, reused), h their FNV-1a hash, both formed
+// as the bytes are read
 template <class F>
-void for_each_token(const char* text, F&& f) {
-  std::string tok;
+void scan_tokens(const char* text, std::vector<unsigned char>& buf, F&& f) {
+  size_t n = 0;
+  uint64_t h = FNV_OFFSET;
   for (const unsigned char* p = reinterpret_cast<const unsigned char*>(text);; ++p) {
     const unsigned char c = *p;
-    if (c != 0 && word_byte(c)) {
-      tok.push_back((char)lower(c));
+    const unsigned char lc = kByte.v[c];
+    if (lc != 0) {
+      if (n == buf.size()) buf.resize(buf.empty() ? 64 : 2 * buf.size());
+      buf[n++] = lc;
+      h = (h ^ lc) * FNV_PRIME;
       continue;
     }
-    if (tok.size() >= 2) f(tok);
-    tok.clear();
+    if (n >= 2) f(static_cast<const unsigned char*>(buf.data()), n, h);
+    n = 0;
+    h = FNV_OFFSET;
     if (c == 0) break;
   }
 }
+
+// The corpus's distinct terms while fitting: open addressing over the terms'
+// hashes, each term's document frequency and the last document that counted
+// it (a document counts a term once).
+struct TermCounter {
+  std::vector<std::string> terms;
+  std::vector<int64_t> df;
+  std::vector<int32_t> last_doc;
+  std::vector<uint64_t> slot_hash;
+  std::vector<int32_t> slot_id;  // -1: empty
+  uint64_t mask = 0;
+
+  TermCounter() { rehash(1024); }
+  void rehash(size_t cap) {
+    slot_hash.assign(cap, 0ull);
+    slot_id.assign(cap, -1);
+    mask = cap - 1;
+    for (size_t j = 0; j < terms.size(); ++j) {
+      const uint64_t h = fnv1a(terms[j].data(), terms[j].size());
+      uint64_t i = h & mask;
+      while (slot_id[i] >= 0) i = (i + 1) & mask;
+      slot_hash[i] = h;
+      slot_id[i] = (int32_t)j;
+    }
+  }
+  void count(const unsigned char* tok, size_t n, uint64_t h, int32_t doc) {
+    uint64_t i = h & mask;
+    for (;; i = (i + 1) & mask) {
+      const int32_t id = slot_id[i];
+      if (id < 0) break;
+      const std::string& t = terms[(size_t)id];
+      if (slot_hash[i] == h && t.size() == n && std::memcmp(t.data(), tok, n) == 0) {
+        if (last_doc[(size_t)id] != doc) {
+          last_doc[(size_t)id] = doc;
+          ++df[(size_t)id];
+        }
+        return;
+      }
+    }
+    terms.emplace_back(reinterpret_cast<const char*>(tok), n);
+    df.push_back(1);
+    last_doc.push_back(doc);
+    slot_hash[i] = h;
+    slot_id[i] = (int32_t)(terms.size() - 1);
+    if (2 * terms.size() > slot_id.size()) rehash(2 * slot_id.size());
+  }
+};
 
 // the column of the lowercased token tok[0, n) with hash h, or -1
 inline int32_t find_column(const pr_prescorer& ps, const unsigned char* tok, size_t n, uint64_t h) {
@@ -128,27 +182,11 @@ void tfidf_row(const pr_prescorer& ps, const char* prompt, Row& row) {
   if (row.count.size() != ps.terms.size()) row.count.assign(ps.terms.size(), 0);
   row.touched.clear();
   row.length = 0;
-  // maximal runs of word bytes, lowercased and hashed as they are read
-  size_t n = 0;
-  uint64_t h = FNV_OFFSET;
-  for (const unsigned char* p = reinterpret_cast<const unsigned char*>(prompt);; ++p) {
-    const unsigned char c = *p;
-    const unsigned char lc = kByte.v[c];
-    if (lc != 0) {
-      if (n == row.tok.size()) row.tok.resize(row.tok.empty() ? 64 : 2 * row.tok.size());
-      row.tok[n++] = lc;
-      h = (h ^ lc) * FNV_PRIME;
-      continue;
-    }
-    if (n >= 2) {
-      ++row.length;
-      const int32_t col = find_column(ps, row.tok.data(), n, h);
-      if (col >= 0 && row.count[(size_t)col]++ == 0) row.touched.push_back(col);
-    }
-    n = 0;
-    h = FNV_OFFSET;
-    if (c == 0) break;
-  }
+  scan_tokens(prompt, row.tok, [&](const unsigned char* tok, size_t n, uint64_t h) {
+    ++row.length;
+    const int32_t col = find_column(ps, tok, n, h);
+    if (col >= 0 && row.count[(size_t)col]++ == 0) row.touched.push_back(col);
+  });
   std::sort(row.touched.begin(), row.touched.end());
   row.v.clear();
   row.v.reserve(row.touched.size());
@@ -191,24 +229,27 @@ pr_status pr_prescorer_fit(const char* const* docs, int32_t n_docs, int32_t min_
   for (int32_t i = 0; i < n_docs; ++i)
     if (!docs[i]) return PR_ERR_INVALID_ARG;
   try {
-    std::unordered_map<std::string, int64_t> df;
-    std::unordered_set<std::string> seen;
-    for (int32_t i = 0; i < n_docs; ++i) {
-      seen.clear();
-      for_each_token(docs[i], [&](const std::string& t) {
-        if (seen.insert(t).second) ++df[t];
-      });
+    TermCounter tc;
+    std::vector<unsigned char> buf;
+    for (int32_t i = 0; i < n_docs; ++i)
+      scan_tokens(docs[i], buf,
+                  [&](const unsigned char* tok, size_t n, uint64_t h) { tc.count(tok, n, h, i); });
+    // the terms kept, in byte order (std::string compares as unsigned char)
+    std::vector<int32_t> keep;
+    for (size_t j = 0; j < tc.terms.size(); ++j)
+      if (tc.df[j] >= min_df) keep.push_back((int32_t)j);
+    std::sort(keep.begin(), keep.end(),
+              [&](int32_t x, int32_t y) { return tc.terms[(size_t)x] < tc.terms[(size_t)y]; });
+    std::unique_ptr<pr_prescorer> ps(new pr_prescorer);
+    ps->terms.reserve(keep.size());
+    ps->idf.reserve(keep.size());
+    for (const int32_t j : keep) {
+      ps->terms.push_back(std::move(tc.terms[(size_t)j]));
+      ps->idf.push_back(std::log((1.0 + (double)n_docs) / (1.0 + (double)tc.df[(size_t)j])) + 1.0);
     }
-    pr_prescorer* ps = new pr_prescorer;
-    for (const auto& tc : df)
-      if (tc.second >= min_df) ps->terms.push_back(tc.first);
-    std::sort(ps->terms.begin(), ps->terms.end());  // byte order (std::string compares as unsigned char)
-    ps->idf.resize(ps->terms.size());
-    for (size_t j = 0; j < ps->terms.size(); ++j)
-      ps->idf[j] = std::log((1.0 + (double)n_docs) / (1.0 + (double)df[ps->terms[j]])) + 1.0;
     ps->n_docs = n_docs;
     build_table(*ps);
-    *out = ps;
+    *out = ps.release();
     return PR_OK;
   } catch (const std::bad_alloc&) {
     return PR_ERR_NO_MEMORY;
