@@ -138,3 +138,24 @@ def test_text_marshalling(B):
     for bad in (["a\0b"], [b"a", b"\0"], ["ok", "no\0"]):
         with pytest.raises(B.PRError):
             B._texts(bad)
+
+
+def test_long_tokens_and_many_terms(B):
+    """Tokens longer than the scan's first buffer (64 bytes) and a corpus with
+    thousands of distinct terms (the fitting table grows several times)."""
+    long_a = b"a" * 300
+    long_b = b"Tok" + b"x" * 5000 + b"end"
+    docs = [b"w%05d common" % i for i in range(5000)] + [long_a + b" " + long_b, long_a]
+    ps = B.pr_prescorer_fit(docs, min_df=1)
+    try:
+        m = op.fit(docs, min_df=1)
+        V = B.pr_prescorer_vocab_size(ps)
+        assert V == len(m.terms) == 5000 + 3
+        assert [B.pr_prescorer_term(ps, j) for j in (0, V - 1)] == [m.terms[0], m.terms[-1]]
+        for p in (long_a, long_b + b" " + long_a + b" w00042", b"COMMON " + long_b.upper()):
+            cols, vals, length = B.pr_prescorer_features(ps, p)
+            row, _, olen = op.features(m, p, 0)
+            assert length == olen and cols.tolist() == sorted(row)
+            np.testing.assert_allclose(vals, [row[j] for j in sorted(row)], rtol=1e-6, atol=1e-7)
+    finally:
+        B.pr_prescorer_destroy(ps)
